@@ -1,0 +1,487 @@
+"""Plain CPU oracle for one GSQ optimisation step of a linear layer.
+
+TEST INFRASTRUCTURE ONLY.  This is the slow, obviously-correct restatement of
+the method that the CUDA path is checked against.  It shares no code with the
+CUDA path; only tests, the smoke check and the benchmark's CPU-baseline leg may
+import it.  Arithmetic is float64 (numpy) except where a floating-point value
+decides an integer (initial round-to-nearest codes, the initial scales that
+feed them, the K-Quant sub-scale codes): those decisions are taken in fp32,
+the precision the kernels use, so both sides decide identically.  Optimiser
+state is stored in fp32 between steps (the precision of the stored state on
+both sides); within a step everything is float64.
+
+What one step computes (paper references):
+  noise      g_k ~ Gumbel(0,1) per weight and level, fresh each step
+             (Alg. 1; §3.3 "Gradient accumulation")      -> philox.gumbel
+  relax      p = softmax((kappa*l + g)/tau)  (Alg. 1)
+  soft weight  w~ = sum_k p_k q_k  (Alg. 1 "return"); W^ = s_group * w~
+             with one scale per group of consecutive inputs (§3.2 constraint
+             set C_b-bit; §4.1 "Quantization configuration": symmetric,
+             group-wise, groups row-wise over consecutive entries)
+  loss       L = ||f(x; W^) - f(x; W)||_F^2 (Eq. 1) for a linear f:
+             sum_t ||(W^ - W) x_t||^2 = tr(D H D^T), D = W^ - W, H = X^T X
+  gradient   dL/dW^ = D (H + H^T); dL/ds_g = sum_{c in g} dL/dW^_c * w~_c;
+             dL/dl_k = (kappa/tau) * dL/dW^ * s * p_k (q_k - w~)  (softmax
+             Jacobian as written in the proof of the Lemma, App. B)
+  optimiser  Lion (§3.3 "Optimizer"; App. B; Table 5 hyper-parameters):
+             c = b1 m + (1-b1) g;  theta <- theta - lr (sign(c) + wd theta);
+             m <- b2 m + (1-b2) g
+  projection hard argmax of the noise-free logits (Alg. 2, final lines,
+             generalised from the binary threshold to K levels)
+  packing    symmetric group-wise b-bit codes + fp16 scale per group (§4.1),
+             or a two-level K-Quant-like super-block (§4.4, App. E).
+
+Readings where the paper is silent are listed at the top of the design notes
+(kappa multiplies the logit; summed, un-normalised loss; Philox stream; absmax
+initial scale; RTN code with +bias logit init; weight decay on logits only;
+sign(0) = 0; lowest index wins argmax ties; packing bit order; fp16 RNE).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Optional
+
+import numpy as np
+
+from . import philox
+
+SUB_BLOCK = 16      # K-Quant-like sub-block (one 6-bit sub-scale code)
+SUPER_BLOCK = 256   # K-Quant-like super-block (one fp16 d)
+
+
+# ----------------------------------------------------------------------------
+# problem and state
+# ----------------------------------------------------------------------------
+@dataclass
+class Problem:
+    """Static inputs of one layer problem (the paper's problem statement, Eq. 1)."""
+    E: int
+    R: int
+    C: int
+    grid: np.ndarray                    # K ascending levels (float64)
+    group: int                          # scale group size along the input dim
+    seed: int = 0
+    scale_mode: str = "group"           # "group" | "kquant2"
+    H: Optional[np.ndarray] = None      # [E, C, C] float64
+    X: Optional[np.ndarray] = None      # [E, T, C] float64 (loss taken literally over tokens)
+    lr_logits: float = 1e-4
+    lr_scales: float = 5e-5
+    beta1: float = 0.9
+    beta2: float = 0.95
+    wd_logits: float = 1.0
+    wd_scales: float = 0.0
+    noise: bool = True
+
+    @property
+    def K(self) -> int:
+        return int(len(self.grid))
+
+
+@dataclass
+class RowState:
+    """Optimiser state for a set of global rows (row id = e*R + r).
+
+    Rows are independent in everything but the scalar loss, so the oracle can
+    follow any subset of rows exactly."""
+    row_ids: np.ndarray                 # int64 [nr]
+    W: np.ndarray                       # float64 [nr, C] (values of the stored dtype)
+    logits: np.ndarray                  # float32 [K, nr, C]
+    scales: np.ndarray                  # float32 [nr, C // group]
+    m_logits: np.ndarray                # float32 [K, nr, C]
+    m_scales: np.ndarray                # float32 [nr, C // group]
+    kq_d: Optional[np.ndarray] = None   # float32 [nr, C // 256] (fp16 values) for kquant2
+    kq_sc: Optional[np.ndarray] = None  # int32 [nr, C // 16] for kquant2
+
+    def copy(self) -> "RowState":
+        return RowState(self.row_ids.copy(), self.W.copy(), self.logits.copy(),
+                        self.scales.copy(), self.m_logits.copy(), self.m_scales.copy(),
+                        None if self.kq_d is None else self.kq_d.copy(),
+                        None if self.kq_sc is None else self.kq_sc.copy())
+
+    def subset(self, idx) -> "RowState":
+        idx = np.asarray(idx)
+        return RowState(self.row_ids[idx].copy(), self.W[idx].copy(),
+                        self.logits[:, idx].copy(), self.scales[idx].copy(),
+                        self.m_logits[:, idx].copy(), self.m_scales[idx].copy(),
+                        None if self.kq_d is None else self.kq_d[idx].copy(),
+                        None if self.kq_sc is None else self.kq_sc[idx].copy())
+
+
+def flat_index(prob: Problem, row_ids: np.ndarray) -> np.ndarray:
+    """i = (e*R + r)*C + c for every weight of the given rows: [nr, C]."""
+    return row_ids.astype(np.int64)[:, None] * prob.C + np.arange(prob.C, dtype=np.int64)[None, :]
+
+
+def expand_scales(scales: np.ndarray, group: int) -> np.ndarray:
+    """Per-weight scale s_{r, floor(c/G)} as float64 [nr, C]."""
+    return np.repeat(scales.astype(np.float64), group, axis=1)
+
+
+# ----------------------------------------------------------------------------
+# forward: noise, relaxation, soft weight (Alg. 1, §3.2)
+# ----------------------------------------------------------------------------
+def relax(logits: np.ndarray, g, tau: float, kappa: float) -> np.ndarray:
+    """p_k = exp((kappa l_k + g_k)/tau) / sum_j exp((kappa l_j + g_j)/tau)  (Alg. 1).
+
+    Level axis first.  The common shift by max_j is the usual overflow guard and
+    leaves the ratio unchanged."""
+    z = (kappa * logits.astype(np.float64) + g) / tau
+    z = z - z.max(axis=0, keepdims=True)
+    e = np.exp(z)
+    return e / e.sum(axis=0, keepdims=True)
+
+
+def soft_value(p: np.ndarray, grid: np.ndarray) -> np.ndarray:
+    """w~ = sum_k p_k q_k (Alg. 1, soft sample over the grid)."""
+    return np.tensordot(np.asarray(grid, dtype=np.float64), p, axes=(0, 0))
+
+
+def noise(prob: Problem, st: RowState, t: int) -> np.ndarray:
+    if not prob.noise:
+        return np.zeros((prob.K, len(st.row_ids), prob.C))
+    return philox.gumbel(prob.seed, t, flat_index(prob, st.row_ids), prob.K)
+
+
+@dataclass
+class Forward:
+    g: np.ndarray
+    p: np.ndarray
+    wtil: np.ndarray
+    s: np.ndarray
+    What: np.ndarray
+    D: np.ndarray
+
+
+def forward(prob: Problem, st: RowState, t: int, tau: float, kappa: float) -> Forward:
+    g = noise(prob, st, t)
+    p = relax(st.logits, g, tau, kappa)
+    wtil = soft_value(p, prob.grid)
+    s = expand_scales(st.scales, prob.group)
+    What = s * wtil
+    return Forward(g=g, p=p, wtil=wtil, s=s, What=What, D=What - st.W)
+
+
+# ----------------------------------------------------------------------------
+# loss and its gradient w.r.t. the soft weight (Eq. 1 with a linear layer)
+# ----------------------------------------------------------------------------
+def loss_and_grad(prob: Problem, row_ids: np.ndarray, D: np.ndarray):
+    """L = sum_rows D_r H_e D_r^T and dL/dW^ = D (H_e + H_e^T), per expert e.
+
+    With calibration tokens (prob.X) the loss is taken literally as
+    sum_t ||D x_t||^2 and the gradient as 2 (D X^T) X."""
+    G = np.empty_like(D)
+    L = 0.0
+    experts = row_ids // prob.R
+    for e in np.unique(experts):
+        sel = experts == e
+        De = D[sel]
+        if prob.X is not None:
+            Xe = prob.X[e]
+            Y = De @ Xe.T                        # rows of (W^ - W) x_t, one column per token
+            L += float(np.sum(Y * Y))
+            G[sel] = 2.0 * (Y @ Xe)
+        else:
+            He = prob.H[e]
+            DH = De @ He
+            L += float(np.sum(DH * De))
+            G[sel] = De @ (He + He.T)
+    return L, G
+
+
+def loss_bruteforce(W: np.ndarray, What: np.ndarray, X: np.ndarray) -> float:
+    """sum over tokens of ||(W - W^) x_t||^2 with explicit Python loops (tiny inputs only)."""
+    R, C = W.shape
+    total = 0.0
+    for x in X:
+        for r in range(R):
+            acc = 0.0
+            for c in range(C):
+                acc += (W[r, c] - What[r, c]) * x[c]
+            total += acc * acc
+    return total
+
+
+# ----------------------------------------------------------------------------
+# backward (App. B softmax Jacobian) and Lion (§3.3, App. B)
+# ----------------------------------------------------------------------------
+def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float):
+    """dL/dl [K, nr, C] and dL/ds [nr, C/G]."""
+    q = np.asarray(prob.grid, dtype=np.float64)[:, None, None]
+    d_logits = (kappa / tau) * (G * fw.s)[None] * fw.p * (q - fw.wtil[None])
+    nr, C = G.shape
+    d_scales = (G * fw.wtil).reshape(nr, C // prob.group, prob.group).sum(axis=2)
+    return d_logits, d_scales
+
+
+def lion(theta32: np.ndarray, m32: np.ndarray, grad: np.ndarray, lr: float, b1: float,
+         b2: float, wd: float):
+    """One Lion update with decoupled weight decay (Chen et al. 2023, the
+    optimiser the paper adopts in §3.3); sign(0) = 0.  Returns fp32 state."""
+    theta = theta32.astype(np.float64)
+    m = m32.astype(np.float64)
+    c = b1 * m + (1.0 - b1) * grad
+    theta_new = theta - lr * (np.sign(c) + wd * theta)
+    m_new = b2 * m + (1.0 - b2) * grad
+    return theta_new.astype(np.float32), m_new.astype(np.float32)
+
+
+def scales_frozen(prob: Problem) -> bool:
+    return prob.lr_scales == 0.0 and prob.wd_scales == 0.0
+
+
+@dataclass
+class StepResult:
+    loss: float
+    fw: Forward
+    G: np.ndarray
+    d_logits: np.ndarray
+    d_scales: Optional[np.ndarray]
+
+
+def step(prob: Problem, st: RowState, t: int, tau: float, kappa: float,
+         update: bool = True) -> StepResult:
+    """One optimisation step t on the given rows (Alg. 2's loop body generalised
+    to K levels: sample, soft weight, loss, gradient, update).  Updates `st` in
+    place unless update=False; the reported loss is this step's forward loss."""
+    fw = forward(prob, st, t, tau, kappa)
+    L, G = loss_and_grad(prob, st.row_ids, fw.D)
+    d_logits, d_scales = backward(prob, fw, G, tau, kappa)
+    if scales_frozen(prob):
+        d_scales = None
+    if update:
+        st.logits, st.m_logits = lion(st.logits, st.m_logits, d_logits, prob.lr_logits,
+                                      prob.beta1, prob.beta2, prob.wd_logits)
+        if d_scales is not None:
+            st.scales, st.m_scales = lion(st.scales, st.m_scales, d_scales, prob.lr_scales,
+                                          prob.beta1, prob.beta2, prob.wd_scales)
+    return StepResult(loss=L, fw=fw, G=G, d_logits=d_logits, d_scales=d_scales)
+
+
+# ----------------------------------------------------------------------------
+# initialisation (readings: absmax scale, round-to-nearest code, +bias logit)
+# ----------------------------------------------------------------------------
+def f32_to_f16_bits(x) -> np.ndarray:
+    """IEEE 754 binary32 -> binary16, round to nearest, ties to even; returns uint16 bits.
+
+    Written from the format definition: 1 sign, 5 exponent (bias 15), 10
+    fraction bits; subnormal quantum 2^-24; magnitudes >= 65520 overflow to inf."""
+    x = np.asarray(x, dtype=np.float32)
+    a = np.abs(x.astype(np.float64))
+    sign = np.where(np.signbit(x), 0x8000, 0).astype(np.uint32)
+    out = np.zeros(x.shape, dtype=np.uint32)
+    nan = np.isnan(x)
+    big = (~nan) & (a >= 65520.0)
+    fin = (~nan) & (~big)
+    _, ex = np.frexp(np.where(fin & (a > 0), a, 1.0))
+    e = ex - 1                                        # a = m * 2^e with m in [1, 2)
+    e = np.maximum(e, -14)                            # below 2^-14 the quantum stays 2^-24
+    quantum = np.ldexp(1.0, e - 10)
+    v = np.rint(a / quantum) * quantum                # exact: a has <= 24 significant bits
+    v = np.where(fin, v, 0.0)
+    _, ev = np.frexp(np.where(v > 0, v, 1.0))
+    ev = ev - 1
+    normal = v >= 2.0 ** -14
+    exp_field = np.where(normal, ev + 15, 0)
+    frac = np.where(normal, v / np.ldexp(1.0, ev - 10) - 1024.0, v / 2.0 ** -24)
+    bits = (exp_field.astype(np.uint32) << 10) | frac.astype(np.uint32)
+    out = np.where(fin, bits, out)
+    out = np.where(big, 0x7C00, out)
+    out = np.where(nan, 0x7E00, out)
+    return (out | sign).astype(np.uint16)
+
+
+def f16_bits_to_f32(h) -> np.ndarray:
+    """binary16 bits -> float value (exact)."""
+    h = np.asarray(h, dtype=np.uint32)
+    s = np.where(h & 0x8000, -1.0, 1.0)
+    e = (h >> 10) & 0x1F
+    f = (h & 0x3FF).astype(np.float64)
+    v = np.where(e == 0, f * 2.0 ** -24, np.ldexp(1.0 + f / 1024.0, e.astype(np.int64) - 15))
+    v = np.where(e == 31, np.where(f == 0, np.inf, np.nan), v)
+    return (s * v).astype(np.float32)
+
+
+def rtn_codes(W32: np.ndarray, s32: np.ndarray, grid: np.ndarray) -> np.ndarray:
+    """Round-to-nearest grid index k0 = argmin_k |W/s - q_k| in fp32 (lowest k on
+    ties); a zero scale maps to the level of smallest magnitude."""
+    q32 = np.asarray(grid, dtype=np.float32)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        x = W32 / s32
+    dist = np.abs(x[None] - q32.reshape((-1,) + (1,) * W32.ndim))
+    codes = np.argmin(dist, axis=0)
+    zero_code = int(np.argmin(np.abs(q32)))
+    return np.where(s32 == 0, zero_code, codes).astype(np.uint8)
+
+
+def init_group_scales(W32: np.ndarray, group: int, grid: np.ndarray) -> np.ndarray:
+    """s_g = max_{c in g} |W_c| / max_k |q_k| in fp32; 1 for an all-zero group."""
+    nr, C = W32.shape
+    absmax = np.abs(W32).reshape(nr, C // group, group).max(axis=2)
+    qmax = np.float32(np.max(np.abs(np.asarray(grid, dtype=np.float32))))
+    s = (absmax / qmax).astype(np.float32)
+    return np.where(absmax == 0, np.float32(1.0), s).astype(np.float32)
+
+
+def init_kquant2_scales(W32: np.ndarray, grid: np.ndarray):
+    """Two-level scales: sub-scale s_j = absmax_16 / qmax; d = fp16(max_j s_j / 31)
+    per 256-weight super-block; sc_j = clamp(rne(s_j / d), -32, 31) (0 when d = 0);
+    effective scale d * sc_j (exact in fp32).  All fp32."""
+    nr, C = W32.shape
+    qmax = np.float32(np.max(np.abs(np.asarray(grid, dtype=np.float32))))
+    sj = (np.abs(W32).reshape(nr, C // SUB_BLOCK, SUB_BLOCK).max(axis=2) / qmax).astype(np.float32)
+    smax = sj.reshape(nr, C // SUPER_BLOCK, SUPER_BLOCK // SUB_BLOCK).max(axis=2)
+    d = f16_bits_to_f32(f32_to_f16_bits((smax / np.float32(31.0)).astype(np.float32)))
+    d_sub = np.repeat(d, SUPER_BLOCK // SUB_BLOCK, axis=1)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        ratio = (sj / d_sub).astype(np.float32)
+    sc = np.where(d_sub > 0, np.clip(np.rint(ratio), -32, 31), 0).astype(np.int32)
+    s_eff = (d_sub * sc.astype(np.float32)).astype(np.float32)
+    return s_eff, d, sc
+
+
+def init_state(prob: Problem, W, row_ids, init_bias: float = 2.0) -> RowState:
+    """Initial state: scales, RTN codes, logits = init_bias on the RTN level
+    (0 elsewhere), zero Lion momenta.  W holds the rows' stored values."""
+    W32 = np.asarray(W, dtype=np.float32)
+    nr, C = W32.shape
+    kq_d = kq_sc = None
+    if prob.scale_mode == "kquant2":
+        s, kq_d, kq_sc = init_kquant2_scales(W32, prob.grid)
+        assert prob.group == SUB_BLOCK
+    else:
+        s = init_group_scales(W32, prob.group, prob.grid)
+    codes = rtn_codes(W32, np.repeat(s, prob.group, axis=1), prob.grid)
+    logits = np.zeros((prob.K, nr, C), dtype=np.float32)
+    for k in range(prob.K):
+        logits[k][codes == k] = np.float32(init_bias)
+    return RowState(row_ids=np.asarray(row_ids, dtype=np.int64), W=W32.astype(np.float64),
+                    logits=logits, scales=s.astype(np.float32),
+                    m_logits=np.zeros_like(logits), m_scales=np.zeros_like(s, dtype=np.float32),
+                    kq_d=kq_d, kq_sc=kq_sc)
+
+
+# ----------------------------------------------------------------------------
+# hard projection (Alg. 2, final lines, generalised to K levels)
+# ----------------------------------------------------------------------------
+def project(logits32: np.ndarray):
+    """k* = argmax_k l_k (lowest k on ties) and margin = l_(1) - l_(2) in fp32."""
+    codes = np.argmax(logits32, axis=0).astype(np.uint8)
+    srt = np.sort(logits32, axis=0)
+    margin = (srt[-1] - srt[-2]).astype(np.float32)
+    return codes, margin
+
+
+# ----------------------------------------------------------------------------
+# packing (§4.1 symmetric group-wise codes + fp16 scale; §4.4 / App. E K-Quant)
+# ----------------------------------------------------------------------------
+def code_bits(K: int) -> int:
+    return 2 if K <= 4 else 3
+
+
+def bits_per_param(K: int, group: int) -> float:
+    """The paper's storage accounting: log2(#levels) bits per code plus a 16-bit
+    scale per group (Table 1: 2.13, 3.13 and 1.71 bit/param at group 128)."""
+    return float(np.log2(K)) + 16.0 / group
+
+
+def _pack_stream(codes: np.ndarray, bits: int) -> np.ndarray:
+    """Little-endian bit stream: element j of every 32-element chunk at bit bits*j
+    of that chunk's bits-word (96-bit for 3-bit codes, 64-bit for 2-bit); words
+    emitted as little-endian uint32.  Returns uint32 words."""
+    c = codes.astype(np.uint64).reshape(-1)
+    n = c.size
+    pad = (-n) % 32
+    if pad:
+        c = np.concatenate([c, np.zeros(pad, dtype=np.uint64)])
+    chunks = c.reshape(-1, 32)
+    words = np.zeros((chunks.shape[0], bits), dtype=np.uint64)
+    for j in range(32):
+        p = bits * j
+        w, o = p // 32, p % 32
+        words[:, w] |= (chunks[:, j] << np.uint64(o)) & np.uint64(0xFFFFFFFF)
+        if o + bits > 32:
+            words[:, w + 1] |= chunks[:, j] >> np.uint64(32 - o)
+    return words.reshape(-1).astype(np.uint32)
+
+
+def _unpack_stream(words: np.ndarray, bits: int, n: int) -> np.ndarray:
+    w = np.asarray(words, dtype=np.uint64).reshape(-1, bits)
+    out = np.zeros((w.shape[0], 32), dtype=np.uint64)
+    mask = np.uint64((1 << bits) - 1)
+    for j in range(32):
+        p = bits * j
+        k, o = p // 32, p % 32
+        v = w[:, k] >> np.uint64(o)
+        if o + bits > 32:
+            v = v | (w[:, k + 1] << np.uint64(32 - o))
+        out[:, j] = v & mask
+    return out.reshape(-1)[:n].astype(np.uint8)
+
+
+def code_section_bytes(n: int, K: int) -> int:
+    b = code_bits(K)
+    raw = ((n + 31) // 32) * 4 * b
+    return (raw + 15) // 16 * 16
+
+
+def pack_group(codes: np.ndarray, scales32: np.ndarray, K: int) -> bytes:
+    """codes [E*R*C] row-major, scales [E*R*C/G] row-major ->
+    [code stream, padded to 16 B] || [fp16 scales, little-endian]."""
+    n = codes.size
+    words = _pack_stream(codes, code_bits(K))
+    code_sec = words.astype("<u4").tobytes()
+    code_sec += b"\0" * (code_section_bytes(n, K) - len(code_sec))
+    return code_sec + f32_to_f16_bits(scales32.reshape(-1)).astype("<u2").tobytes()
+
+
+def unpack_group(buf: bytes, n: int, K: int, n_groups: int):
+    cs = code_section_bytes(n, K)
+    bits = code_bits(K)
+    nw = ((n + 31) // 32) * bits
+    words = np.frombuffer(buf[: nw * 4], dtype="<u4")
+    codes = _unpack_stream(words, bits, n)
+    sc = np.frombuffer(buf[cs: cs + 2 * n_groups], dtype="<u2")
+    return codes, sc
+
+
+KQ_RECORD = 110   # 96 B codes || 12 B sub-scales || 2 B fp16 d
+
+
+def pack_kquant2(codes: np.ndarray, d32: np.ndarray, sc: np.ndarray) -> bytes:
+    """One 110-byte record per 256 consecutive weights (row-major):
+    3-bit codes (same stream as pack_group) || 16 sub-scale codes sc+32 as a
+    6-bit little-endian stream || fp16 d."""
+    nb = codes.size // SUPER_BLOCK
+    cw = _pack_stream(codes.reshape(nb, SUPER_BLOCK), 3).reshape(nb, 24)
+    s6 = (sc.reshape(nb, 16).astype(np.int64) + 32).astype(np.uint64)
+    sw = np.zeros((nb, 3), dtype=np.uint64)
+    for j in range(16):
+        p = 6 * j
+        w, o = p // 32, p % 32
+        sw[:, w] |= (s6[:, j] << np.uint64(o)) & np.uint64(0xFFFFFFFF)
+        if o + 6 > 32:
+            sw[:, w + 1] |= s6[:, j] >> np.uint64(32 - o)
+    dh = f32_to_f16_bits(d32.reshape(nb)).astype("<u2")
+    rec = np.zeros((nb, KQ_RECORD), dtype=np.uint8)
+    rec[:, :96] = cw.astype("<u4").view(np.uint8).reshape(nb, 96)
+    rec[:, 96:108] = sw.astype(np.uint32).astype("<u4").view(np.uint8).reshape(nb, 12)
+    rec[:, 108:110] = dh.view(np.uint8).reshape(nb, 2)
+    return rec.tobytes()
+
+
+def unpack_kquant2(buf: bytes, n: int):
+    nb = n // SUPER_BLOCK
+    rec = np.frombuffer(buf, dtype=np.uint8)[: nb * KQ_RECORD].reshape(nb, KQ_RECORD)
+    cw = rec[:, :96].copy().view("<u4").reshape(-1)
+    codes = _unpack_stream(cw, 3, n)
+    sw = rec[:, 96:108].copy().view("<u4").astype(np.uint64).reshape(nb, 3)
+    sc = np.zeros((nb, 16), dtype=np.int32)
+    for j in range(16):
+        p = 6 * j
+        w, o = p // 32, p % 32
+        v = sw[:, w] >> np.uint64(o)
+        if o + 6 > 32:
+            v = v | (sw[:, w + 1] << np.uint64(32 - o))
+        sc[:, j] = (v & np.uint64(63)).astype(np.int32) - 32
+    d = f16_bits_to_f32(rec[:, 108:110].copy().view("<u2").reshape(nb))
+    return codes, d, sc

@@ -1,0 +1,124 @@
+"""The five synthetic layer workloads the step is built and measured on.
+
+Each workload fixes a layer shape, a grid, a group size, a calibration recipe
+and a temperature schedule.  The shapes follow the layers the paper quantizes
+(Llama-3.1-8B/70B linear layers and MoE experts, §4.1); the optimiser
+hyper-parameters follow the paper's training tables (Table 5: Lion, logits lr
+1e-4, group-scales lr 5e-5, betas (0.9, 0.95), weight decay 1.0; Table 7: the
+K-Quant scales are frozen, scale lr 0).
+
+Nothing here computes any part of the method.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field, replace
+from typing import Tuple
+
+GRID_TERNARY = (-1.0, 0.0, 1.0)
+GRID_2BIT_SYM = (-1.5, -0.5, 0.5, 1.5)
+GRID_2BIT_SKEWED = (-2.0, -1.0, 0.0, 1.0)          # §3.2 "The 2-bit case"
+GRID_3BIT_SYM = (-3.5, -2.5, -1.5, -0.5, 0.5, 1.5, 2.5, 3.5)
+
+SCALE_GROUP = "group"
+SCALE_KQUANT2 = "kquant2"
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    experts: int
+    rows: int                  # R = out_features
+    cols: int                  # C = in_features
+    grid: Tuple[float, ...]
+    group: int                 # scale group along the input dim (16 = K-Quant sub-block)
+    w_dtype: str               # "f32" | "bf16"
+    calib: str                 # "X" (tokens kept) | "H" (Gram matrix)
+    tokens: int                # calibration tokens per expert
+    token_dist: str            # "normal" | "student_t3"
+    outliers: int              # number of outlier channels
+    outlier_scale: float
+    steps: int
+    tau0: float
+    tau1: float
+    kappa: float = 1.0
+    scale_mode: str = SCALE_GROUP
+    init_bias: float = 2.0
+    seed: int = 0
+    lr_logits: float = 1e-4
+    lr_scales: float = 5e-5
+    beta1: float = 0.9
+    beta2: float = 0.95
+    wd_logits: float = 1.0
+    wd_scales: float = 0.0
+    data_seed: int = 0
+    pack: bool = False
+
+    @property
+    def K(self) -> int:
+        return len(self.grid)
+
+    @property
+    def n(self) -> int:
+        return self.experts * self.rows * self.cols
+
+    def tau(self, t: int) -> float:
+        """Linear temperature schedule tau0 -> tau1 over steps 0..T-1."""
+        if self.steps <= 1:
+            return self.tau0
+        return self.tau0 + (self.tau1 - self.tau0) * t / (self.steps - 1)
+
+    def w_bytes(self) -> int:
+        return 4 if self.w_dtype == "f32" else 2
+
+    def elementwise_bytes_per_weight(self) -> int:
+        """Algorithmic HBM bytes per weight of one steady-state step's fused
+        elementwise kernel (backward t + Lion + forward t+1):
+        read logits, logit momentum (4K each), G (4), W (b_W);
+        write logits, logit momentum (4K each), D for the next step (2)."""
+        return 16 * self.K + 4 + self.w_bytes() + 2
+
+    def gemm_flops_per_step(self) -> int:
+        return 2 * self.experts * self.rows * self.cols * self.cols
+
+
+WORKLOADS = {
+    w.name: w
+    for w in [
+        Workload(name="ternary_256x512", experts=1, rows=256, cols=512, grid=GRID_TERNARY,
+                 group=128, w_dtype="f32", calib="X", tokens=256, token_dist="normal",
+                 outliers=4, outlier_scale=20.0, steps=50, tau0=1.0, tau1=1.0, data_seed=1000),
+        Workload(name="llama8b_q_proj", experts=1, rows=4096, cols=4096, grid=GRID_2BIT_SYM,
+                 group=128, w_dtype="bf16", calib="H", tokens=128 * 2048, token_dist="normal",
+                 outliers=41, outlier_scale=30.0, steps=500, tau0=1.0, tau1=0.1, data_seed=2000),
+        Workload(name="llama8b_down_proj", experts=1, rows=4096, cols=14336, grid=GRID_3BIT_SYM,
+                 group=128, w_dtype="bf16", calib="H", tokens=256 * 2048, token_dist="student_t3",
+                 outliers=0, outlier_scale=1.0, steps=200, tau0=0.5, tau1=0.5, data_seed=3000),
+        Workload(name="llama70b_gate_proj", experts=1, rows=28672, cols=8192, grid=GRID_2BIT_SYM,
+                 group=64, w_dtype="bf16", calib="H", tokens=128 * 2048, token_dist="normal",
+                 outliers=82, outlier_scale=30.0, steps=100, tau0=1.0, tau1=1.0, data_seed=4000,
+                 pack=True),
+        Workload(name="moe64_kquant3", experts=64, rows=2048, cols=7168, grid=GRID_3BIT_SYM,
+                 group=16, w_dtype="bf16", calib="H", tokens=4096, token_dist="normal",
+                 outliers=72, outlier_scale=30.0, steps=100, tau0=1.0, tau1=1.0,
+                 scale_mode=SCALE_KQUANT2, lr_scales=0.0, data_seed=5000, pack=True),
+    ]
+}
+
+ORDER = ["ternary_256x512", "llama8b_q_proj", "llama8b_down_proj", "llama70b_gate_proj",
+         "moe64_kquant3"]
+
+
+def shrunk(w: Workload, experts: int | None = None, rows: int | None = None,
+           cols: int | None = None, tokens: int | None = None) -> Workload:
+    """The same workload recipe at a smaller shape (for tests the oracle finishes in seconds)."""
+    kw = {}
+    if experts is not None:
+        kw["experts"] = experts
+    if rows is not None:
+        kw["rows"] = rows
+    if cols is not None:
+        kw["cols"] = cols
+        kw["outliers"] = min(w.outliers, max(1, cols // 100)) if w.outliers else 0
+    if tokens is not None:
+        kw["tokens"] = tokens
+    return replace(w, **kw)

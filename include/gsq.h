@@ -1,0 +1,255 @@
+/*
+ * gsq.h -- C ABI of libgsq: one optimisation step of the GSQ relaxed scalar
+ * quantizer (Gumbel-Softmax Quantization) for a linear layer, on one sm_103a GPU.
+ *
+ * The method (paper: "GSQ: Highly-Accurate Low-Precision Scalar Quantization for
+ * LLMs via Gumbel-Softmax Sampling"):
+ *   - every weight w_i of W gets one learnable logit l_{i,k} per level q_k of an
+ *     ordered grid (§3.2, "General scalar quantization": l in R^{d x 2^b});
+ *   - each step draws Gumbel noise g_{i,k} (Alg. 1), forms the tempered softmax
+ *     p_{i,k} = softmax_k((kappa*l_{i,k} + g_{i,k}) / tau) (Alg. 1), the soft value
+ *     w~_i = sum_k p_{i,k} q_k and the soft weight W^_i = s_{group(i)} * w~_i with one
+ *     learnable scale per group of consecutive inputs (§3.2; §4.1 "Quantization
+ *     configuration");
+ *   - the loss is the layer-wise reconstruction error of Eq. 1 for a linear layer,
+ *     L = sum_t ||(W^ - W) x_t||^2 = tr(D H D^T), D = W^ - W, H = X^T X;
+ *   - logits and scales are updated with Lion (§3.3 "Optimizer", App. B);
+ *   - after training the logits are hard-projected by argmax (Alg. 2, last lines)
+ *     and packed into a symmetric group-wise scalar format (§4.1) or a two-level
+ *     K-Quant-like format (§4.4, App. E).
+ *
+ * Conventions for every entry point:
+ *   - All functions return a gsq_status (int32_t).  GSQ_OK = 0.  On failure
+ *     gsq_last_error() returns a thread-local, human-readable message.
+ *   - No C++ exception crosses this boundary.
+ *   - "device" pointers are CUDA device (or managed) memory on the current device;
+ *     "host" pointers are ordinary host memory.  Nothing here allocates device
+ *     memory: the caller provides a workspace and every output buffer.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).
+ *     Work is enqueued on it; calls return without waiting for the GPU except
+ *     where a function says it synchronises.
+ *   - Argument errors are detected on the host before anything is enqueued.
+ *     Launch errors are reported as GSQ_ERR_CUDA.
+ *   - Fault injection for host-side tests: with the environment variable
+ *     GSQ_FAULT_INJECT=<function name>:<n>, the n-th call (1-based) of that
+ *     function returns GSQ_ERR_INJECTED before touching the GPU.
+ */
+#ifndef GSQ_H_
+#define GSQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define GSQ_API __attribute__((visibility("default")))
+#else
+#define GSQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes -------------------------------------------------------- */
+enum {
+  GSQ_OK = 0,
+  GSQ_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-positive tau, ...   */
+  GSQ_ERR_SHAPE = 2,       /* shape not supported (divisibility, limits)      */
+  GSQ_ERR_WORKSPACE = 3,   /* workspace too small or misaligned               */
+  GSQ_ERR_CUDA = 4,        /* a CUDA runtime/driver call or launch failed     */
+  GSQ_ERR_NONFINITE = 5,   /* W or the calibration input holds NaN/Inf        */
+  GSQ_ERR_STATE = 6,       /* call out of order (e.g. destroyed handle)       */
+  GSQ_ERR_TIMEOUT = 7,     /* a bounded device-side wait gave up              */
+  GSQ_ERR_INJECTED = 8,    /* GSQ_FAULT_INJECT fired                          */
+  GSQ_ERR_UNSUPPORTED = 9  /* device is not sm_103 / feature not available    */
+};
+typedef int32_t gsq_status;
+
+/* ---- descriptor enums ---------------------------------------------------- */
+#define GSQ_MAX_LEVELS 8
+enum { GSQ_DTYPE_F32 = 0, GSQ_DTYPE_BF16 = 1 };
+enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1 };
+enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
+enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
+enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel draw */
+
+/* Layer problem (Eq. 1 with a linear f; §3.2; §4.1; Table 5 for the defaults).
+ *
+ * W            device, borrowed during gsq_init_layer only.  Row-major
+ *              [num_experts][out_features][in_features], dtype w_dtype.
+ * calib        device, borrowed during gsq_init_layer only, fp32.
+ *              GSQ_CALIB_H: Gram matrices H_e = X_e^T X_e, [E][C][C] row-major
+ *              (symmetrised as (H + H^T)/2 on copy).
+ *              GSQ_CALIB_X: tokens X_e, [E][n_tokens][C] row-major; H_e is formed
+ *              from them at init (fp32, on the GPU).
+ * grid         the K ordered levels q_0 < ... < q_{K-1} (host values, copied).
+ * group_size   scale group along the input dim, power of two in [4, 128],
+ *              in_features % group_size == 0.  GSQ_SCALE_KQUANT2 requires 16.
+ * scale_mode   GSQ_SCALE_GROUP: one fp32 scale per group, learned (signed).
+ *              GSQ_SCALE_KQUANT2: two-level frozen scales: per 16-weight sub-block
+ *              s = d * sc with an fp16 d per 256-weight super-block and a 6-bit
+ *              signed sc; requires lr_scales == 0 and in_features % 256 == 0.
+ * init_bias    logit given to the round-to-nearest level at init (others 0).
+ * seed         key of the counter-based Gumbel noise (Philox4x32-10).
+ * lr_*, beta*, wd_*  Lion hyper-parameters; lr_scales = wd_scales = 0 freezes
+ *              the scales.
+ * gemm_precision  GSQ_GEMM_BF16: the loss contraction G = D (H + H^T) runs on the
+ *              tensor cores with bf16 D and H and fp32 accumulation;
+ *              GSQ_GEMM_F32: fp32 D and H on the CUDA cores (validation).
+ * Limits: 1 <= E, 1 <= R, 8 <= C, C % 8 == 0, E*R*C < 2^40, 2 <= K <= 8.
+ */
+typedef struct gsq_layer_desc {
+  int32_t num_experts;
+  int32_t out_features;
+  int32_t in_features;
+  int32_t w_dtype;
+  const void* W;
+  const float* calib;
+  int64_t n_tokens;
+  int32_t calib_kind;
+  int32_t num_levels;
+  float grid[GSQ_MAX_LEVELS];
+  int32_t group_size;
+  int32_t scale_mode;
+  float init_bias;
+  uint32_t flags;
+  uint64_t seed;
+  float lr_logits;
+  float lr_scales;
+  float beta1;
+  float beta2;
+  float wd_logits;
+  float wd_scales;
+  int32_t gemm_precision;
+  int32_t reserved;
+} gsq_layer_desc;
+
+typedef struct gsq_layer gsq_layer; /* opaque handle, host memory owned by libgsq */
+
+/* Bytes of device workspace gsq_init_layer needs for this descriptor.  Pure
+ * host arithmetic; no CUDA call.  The workspace must be 256-byte aligned. */
+GSQ_API gsq_status gsq_workspace_size(const gsq_layer_desc* desc, size_t* bytes);
+
+/* Validate `desc`, carve `workspace` (device, caller-owned, must outlive the
+ * handle), and initialise the state on `stream`: copy W; form H (from X if
+ * GSQ_CALIB_X), symmetrise it and convert it to the GEMM operand precision;
+ * initial scales (absmax / max|q|, or the two-level K-Quant scales); RTN codes;
+ * logits = init_bias on the RTN level; Lion momenta = 0.  Synchronises `stream`
+ * once, to report GSQ_ERR_NONFINITE if W or calib holds NaN/Inf.  On success
+ * *out receives a new handle (release with gsq_destroy). */
+GSQ_API gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t bytes,
+                          void* stream, gsq_layer** out);
+
+/* One optimisation step t (Alg. 2 loop body generalised to K levels):
+ *   forward   noise for step t, p = softmax((kappa l + g)/tau), W^, D = W^ - W
+ *             (skipped when the previous call already produced D for
+ *             (t, tau, kappa) through its look-ahead);
+ *   loss      G = dL/dW^ = D (H + H^T) on the tensor cores (or fp32 cores),
+ *             L_t = 1/2 sum D*G = tr(D H D^T);
+ *   backward  dL/dl_k = (kappa/tau) G s p_k (q_k - w~),  dL/ds_g = sum_g G w~;
+ *   update    Lion on logits and scales, in place;
+ *   look-ahead (next_tau > 0): the same kernel then draws the noise of step t+1
+ *             and writes D for (t+1, next_tau, next_kappa), so the next call
+ *             skips its forward.  Results are identical either way.
+ * step         noise counter t, < 2^32.  tau > 0, kappa finite.
+ * loss_dev     device fp32 scalar, nullable: receives L_t (the loss of this
+ *              step's forward, before the update).
+ * grad_logits_dev / grad_scales_dev  device, nullable.  If either is non-null
+ *              the step runs in gradient-export mode: it writes the raw
+ *              gradients ([K][E][R][C] fp32 and [E][R][C/G] fp32), skips the Lion
+ *              update and ignores next_tau.
+ * Never synchronises; graph-capturable for a fixed argument list. */
+GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float kappa, float next_tau,
+                    float next_kappa, void* stream, float* loss_dev, float* grad_logits_dev,
+                    float* grad_scales_dev);
+
+/* Forward only (Alg. 1 for every weight): writes D for (step, tau, kappa) into
+ * the workspace and, if what_dev (device fp32 [E][R][C]) is non-null, the soft
+ * weight W^.  A following gsq_step with the same (step, tau, kappa) reuses D. */
+GSQ_API gsq_status gsq_forward(gsq_layer* layer, uint64_t step, float tau, float kappa, void* stream,
+                       float* what_dev);
+
+/* Hard projection (Alg. 2, last lines, for K levels): codes_dev (device uint8
+ * [E][R][C], nullable) receives argmax_k l_k of the noise-free logits, lowest k on
+ * ties; margin_dev (device fp32 [E][R][C], nullable) receives l_(1) - l_(2). */
+GSQ_API gsq_status gsq_project(gsq_layer* layer, void* stream, uint8_t* codes_dev, float* margin_dev);
+
+/* Size of the packed output of gsq_pack. */
+GSQ_API gsq_status gsq_packed_size(const gsq_layer* layer, size_t* bytes);
+
+/* Project and pack (§4.1; §4.4 and App. E) into out_dev (device, cap bytes):
+ *  GSQ_SCALE_GROUP: code stream (2-bit codes for K <= 4, 3-bit for K <= 8; within
+ *    each chunk of 32 consecutive weights of the row-major [E][R][C] order, code j
+ *    sits at bit b*j of a little-endian b*32-bit word), padded to 16 bytes, then
+ *    the fp16 (round-to-nearest-even) group scales [E][R][C/G], little-endian.
+ *  GSQ_SCALE_KQUANT2: one 110-byte record per 256 consecutive weights: 96 B of
+ *    3-bit codes (same stream), 12 B of sixteen 6-bit sub-scale codes sc+32
+ *    (little-endian stream, code j at bit 6j), 2 B fp16 d.
+ * *written (host, nullable) receives the byte count. */
+GSQ_API gsq_status gsq_pack(gsq_layer* layer, void* stream, void* out_dev, size_t cap, size_t* written);
+
+/* State tensors for inspection, checkpoint and resume. */
+enum {
+  GSQ_T_LOGITS = 0,     /* fp32 [K][E][R][C]                                   */
+  GSQ_T_SCALES = 1,     /* fp32 [E][R][C/G] (effective scale d*sc for KQUANT2)  */
+  GSQ_T_MOM_LOGITS = 2, /* fp32 [K][E][R][C]                                   */
+  GSQ_T_MOM_SCALES = 3, /* fp32 [E][R][C/G]                                    */
+  GSQ_T_D = 4,          /* last forward's D = W^ - W, [E][R][C], bf16 or fp32  */
+  GSQ_T_G = 5,          /* last step's dL/dW^, fp32 [E][R][C]                  */
+  GSQ_T_W = 6,          /* stored copy of W, [E][R][C], w_dtype                */
+  GSQ_T_H = 7,          /* GEMM operand H (symmetrised), [E][C][C], bf16/fp32  */
+  GSQ_T_KQ_D = 8,       /* fp16 bits [E*R*C/256] (KQUANT2 only)                */
+  GSQ_T_KQ_SC = 9       /* int8 [E*R*C/16] (KQUANT2 only)                      */
+};
+
+/* Byte size of tensor `which` (0 when the layer has no such tensor). */
+GSQ_API gsq_status gsq_tensor_size(const gsq_layer* layer, int32_t which, size_t* bytes);
+
+/* Copy tensor `which` to/from caller device memory (bytes must equal its size).
+ * gsq_set_tensor invalidates a pending look-ahead forward.  Saving LOGITS,
+ * SCALES, MOM_LOGITS, MOM_SCALES and the step index and restoring them into a
+ * layer built from the same descriptor resumes the trajectory bit for bit. */
+GSQ_API gsq_status gsq_get_tensor(gsq_layer* layer, int32_t which, void* dst_dev, size_t bytes,
+                          void* stream);
+GSQ_API gsq_status gsq_set_tensor(gsq_layer* layer, int32_t which, const void* src_dev, size_t bytes,
+                          void* stream);
+
+/* Synchronise `stream` and report GSQ_ERR_TIMEOUT if a bounded device-side wait
+ * of an earlier launch gave up (the error word is then cleared). */
+GSQ_API gsq_status gsq_sync_status(gsq_layer* layer, void* stream);
+
+/* Per-kernel CUDA-event timing.  While enabled, every launch made by libgsq for
+ * this layer is bracketed by events recorded on the launch stream.
+ * gsq_profile_read synchronises on the last event, returns per-kernel launch
+ * counts and total milliseconds (kinds: GSQ_K_*), and clears the record. */
+enum {
+  GSQ_K_FORWARD = 0,  /* standalone forward (noise + softmax + D)              */
+  GSQ_K_GEMM = 1,     /* loss contraction G = D (H + H^T)                     */
+  GSQ_K_BACKWARD = 2, /* fused backward + Lion (+ look-ahead forward) + loss   */
+  GSQ_K_PROJECT = 3,
+  GSQ_K_PACK = 4,
+  GSQ_K_INIT = 5,
+  GSQ_K_COUNT = 6
+};
+typedef struct gsq_profile {
+  int32_t launches[GSQ_K_COUNT];
+  float total_ms[GSQ_K_COUNT];
+} gsq_profile;
+GSQ_API gsq_status gsq_profile_enable(gsq_layer* layer, int32_t on);
+GSQ_API gsq_status gsq_profile_read(gsq_layer* layer, gsq_profile* out);
+
+/* Release the handle (host memory only; the workspace stays the caller's).
+ * Returns GSQ_ERR_INVALID_ARG for NULL. */
+GSQ_API gsq_status gsq_destroy(gsq_layer* layer);
+
+/* Message of the last failure on this thread ("" if none). */
+GSQ_API const char* gsq_last_error(void);
+
+/* Library version, "major.minor.patch". */
+GSQ_API const char* gsq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GSQ_H_ */

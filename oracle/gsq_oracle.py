@@ -184,7 +184,7 @@ def loss_and_grad(prob: Problem, row_ids: np.ndarray, D: np.ndarray):
             He = prob.H[e]
             DH = De @ He
             L += float(np.sum(DH * De))
-            G[sel] = De @ (He + He.T)
+            G[sel] = DH + De @ He.T              # D (H + H^T)
     return L, G
 
 

@@ -1,0 +1,766 @@
+// Host side of libgsq: the extern "C" entry points declared in include/gsq.h.
+// Validates arguments, carves the caller's workspace, sequences the kernels on
+// the caller's stream and keeps the per-layer bookkeeping (pending look-ahead
+// forward, profiling events).  Never allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <unordered_map>
+#include <unordered_set>
+#include <vector>
+
+#include "gsq_internal.h"
+
+namespace gsq {
+namespace {
+
+constexpr uint64_t kMagic = 0x6773715f6c617972ull;  // "gsq_layr"
+constexpr int kMaxPartials = 16384;
+constexpr int kMaxProfileEvents = 8192;
+
+thread_local std::string g_last_error;
+
+gsq_status fail(gsq_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+gsq_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(GSQ_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// GSQ_FAULT_INJECT=<function>:<n>: the n-th call of <function> fails.
+bool injected(const char* fn) {
+  static std::once_flag once;
+  static std::string target;
+  static long nth = 0;
+  static std::mutex mu;
+  static std::unordered_map<std::string, long> calls;
+  std::call_once(once, [] {
+    const char* v = std::getenv("GSQ_FAULT_INJECT");
+    if (!v) return;
+    const char* colon = std::strchr(v, ':');
+    if (!colon) return;
+    target.assign(v, colon - v);
+    nth = std::strtol(colon + 1, nullptr, 10);
+  });
+  if (target.empty() || target != fn) return false;
+  std::lock_guard<std::mutex> lk(mu);
+  return ++calls[target] == nth;
+}
+
+#define GSQ_INJECT(fn)                                                     \
+  do {                                                                     \
+    if (injected(fn)) return fail(GSQ_ERR_INJECTED, "%s: injected fault", fn); \
+  } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Layout {
+  size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch;
+  size_t total;
+};
+
+struct Shape {
+  int64_t E, R, C, n, ng;
+  int K, group;
+  bool kquant, d_bf16, w_bf16, x_mode;
+};
+
+Shape shape_of(const gsq_layer_desc& d) {
+  Shape s;
+  s.E = d.num_experts;
+  s.R = d.out_features;
+  s.C = d.in_features;
+  s.n = s.E * s.R * s.C;
+  s.K = d.num_levels;
+  s.group = d.group_size;
+  s.ng = s.group > 0 ? s.n / s.group : 0;
+  s.kquant = d.scale_mode == GSQ_SCALE_KQUANT2;
+  s.d_bf16 = d.gemm_precision == GSQ_GEMM_BF16;
+  s.w_bf16 = d.w_dtype == GSQ_DTYPE_BF16;
+  s.x_mode = d.calib_kind == GSQ_CALIB_X;
+  return s;
+}
+
+Layout layout_of(const Shape& s) {
+  Layout L;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += align256(bytes);
+    return o;
+  };
+  const size_t n = static_cast<size_t>(s.n), ng = static_cast<size_t>(s.ng);
+  L.flags = take(sizeof(DevFlags));
+  L.partials = take(sizeof(double) * kMaxPartials);
+  L.logits = take(4 * n * s.K);
+  L.m_logits = take(4 * n * s.K);
+  L.scales = take(4 * ng);
+  L.m_scales = take(4 * ng);
+  L.W = take(n * (s.w_bf16 ? 2 : 4));
+  L.H = take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4));
+  L.D = take(n * (s.d_bf16 ? 2 : 4));
+  L.G = take(4 * n);
+  L.kq_d = s.kquant ? take(2 * (n / kSuperBlock)) : off;
+  L.kq_sc = s.kquant ? take(n / kSubBlock) : off;
+  L.hscratch = s.x_mode ? take(static_cast<size_t>(s.E) * s.C * s.C * 4) : off;
+  L.total = off;
+  return L;
+}
+
+bool is_pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
+
+gsq_status validate_desc(const gsq_layer_desc* d) {
+  if (!d) return fail(GSQ_ERR_INVALID_ARG, "desc is NULL");
+  if (d->num_experts < 1 || d->out_features < 1 || d->in_features < 8)
+    return fail(GSQ_ERR_SHAPE, "need E >= 1, R >= 1, C >= 8 (got %d, %d, %d)", d->num_experts,
+                d->out_features, d->in_features);
+  if (d->in_features % 8 != 0) return fail(GSQ_ERR_SHAPE, "in_features %% 8 != 0 (%d)", d->in_features);
+  const double n = static_cast<double>(d->num_experts) * d->out_features * d->in_features;
+  if (n >= 1099511627776.0) return fail(GSQ_ERR_SHAPE, "E*R*C must be < 2^40");
+  if (d->num_levels < 2 || d->num_levels > GSQ_MAX_LEVELS)
+    return fail(GSQ_ERR_INVALID_ARG, "num_levels must be in [2, 8] (got %d)", d->num_levels);
+  for (int k = 0; k < d->num_levels; ++k) {
+    if (!std::isfinite(d->grid[k])) return fail(GSQ_ERR_INVALID_ARG, "grid[%d] is not finite", k);
+    if (k > 0 && !(d->grid[k] > d->grid[k - 1]))
+      return fail(GSQ_ERR_INVALID_ARG, "grid must be strictly ascending");
+  }
+  float qmax = 0.f;
+  for (int k = 0; k < d->num_levels; ++k) qmax = std::fmax(qmax, std::fabs(d->grid[k]));
+  if (!(qmax > 0.f)) return fail(GSQ_ERR_INVALID_ARG, "grid must have a nonzero level");
+  if (!is_pow2(d->group_size) || d->group_size < 4 || d->group_size > 128)
+    return fail(GSQ_ERR_SHAPE, "group_size must be a power of two in [4, 128] (got %d)", d->group_size);
+  if (d->in_features % d->group_size != 0)
+    return fail(GSQ_ERR_SHAPE, "in_features %% group_size != 0");
+  if (d->w_dtype != GSQ_DTYPE_F32 && d->w_dtype != GSQ_DTYPE_BF16)
+    return fail(GSQ_ERR_INVALID_ARG, "bad w_dtype %d", d->w_dtype);
+  if (d->calib_kind != GSQ_CALIB_H && d->calib_kind != GSQ_CALIB_X)
+    return fail(GSQ_ERR_INVALID_ARG, "bad calib_kind %d", d->calib_kind);
+  if (d->calib_kind == GSQ_CALIB_X && (d->n_tokens < 1 || d->n_tokens > 2147483647LL))
+    return fail(GSQ_ERR_INVALID_ARG, "n_tokens must be in [1, 2^31) for GSQ_CALIB_X");
+  if (d->scale_mode != GSQ_SCALE_GROUP && d->scale_mode != GSQ_SCALE_KQUANT2)
+    return fail(GSQ_ERR_INVALID_ARG, "bad scale_mode %d", d->scale_mode);
+  if (d->scale_mode == GSQ_SCALE_KQUANT2) {
+    if (d->group_size != kSubBlock) return fail(GSQ_ERR_SHAPE, "GSQ_SCALE_KQUANT2 needs group_size 16");
+    if (d->in_features % kSuperBlock != 0)
+      return fail(GSQ_ERR_SHAPE, "GSQ_SCALE_KQUANT2 needs in_features %% 256 == 0");
+    if (d->lr_scales != 0.f || d->wd_scales != 0.f)
+      return fail(GSQ_ERR_INVALID_ARG, "GSQ_SCALE_KQUANT2 scales are frozen: lr_scales = wd_scales = 0");
+  }
+  if (d->gemm_precision != GSQ_GEMM_BF16 && d->gemm_precision != GSQ_GEMM_F32)
+    return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
+  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE))
+    return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
+  const float hp[] = {d->init_bias, d->lr_logits, d->lr_scales, d->beta1, d->beta2, d->wd_logits, d->wd_scales};
+  for (float v : hp)
+    if (!std::isfinite(v)) return fail(GSQ_ERR_INVALID_ARG, "non-finite hyper-parameter");
+  if (d->beta1 < 0.f || d->beta1 > 1.f || d->beta2 < 0.f || d->beta2 > 1.f)
+    return fail(GSQ_ERR_INVALID_ARG, "betas must be in [0, 1]");
+  if (d->lr_logits < 0.f || d->lr_scales < 0.f) return fail(GSQ_ERR_INVALID_ARG, "negative learning rate");
+  return GSQ_OK;
+}
+
+struct DeviceGuard {
+  int prev = -1;
+  bool switched = false;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) switched = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    if (switched) cudaSetDevice(prev);
+  }
+};
+
+}  // namespace
+}  // namespace gsq
+
+using namespace gsq;
+
+struct gsq_layer {
+  uint64_t magic;
+  gsq_layer_desc desc;
+  Shape shape;
+  Layout lay;
+  uint8_t* ws;
+  int device;
+  int num_sms;
+  int grid_fwd, grid_bwd;
+  bool tc;
+  // pending forward (D valid for these arguments)
+  bool d_ready;
+  uint64_t d_step;
+  float d_tau, d_kappa;
+  // profiling
+  bool profiling;
+  std::vector<cudaEvent_t> ev;  // pairs
+  std::vector<int> ev_kind;
+  int ev_used;
+  cudaStream_t last_stream;
+};
+
+namespace {
+
+float* fptr(gsq_layer* L, size_t off) { return reinterpret_cast<float*>(L->ws + off); }
+
+// Live handles, so a stale or twice-destroyed pointer is rejected without
+// being dereferenced.
+std::mutex g_live_mu;
+std::unordered_set<const gsq_layer*> g_live;
+
+bool valid(const gsq_layer* L) {
+  if (!L) return false;
+  std::lock_guard<std::mutex> lk(g_live_mu);
+  return g_live.count(L) != 0 && L->magic == kMagic;
+}
+
+void register_live(const gsq_layer* L) {
+  std::lock_guard<std::mutex> lk(g_live_mu);
+  g_live.insert(L);
+}
+
+void unregister_live(const gsq_layer* L) {
+  std::lock_guard<std::mutex> lk(g_live_mu);
+  g_live.erase(L);
+}
+
+EwParams base_params(gsq_layer* L) {
+  EwParams p;
+  std::memset(&p, 0, sizeof(p));
+  const Shape& s = L->shape;
+  const gsq_layer_desc& d = L->desc;
+  p.n = s.n;
+  p.nq = s.n / 4;
+  p.K = s.K;
+  p.group = s.group;
+  int lg = 0;
+  while ((1 << lg) < s.group) ++lg;
+  p.log2_group = lg;
+  p.w_bf16 = s.w_bf16;
+  p.d_bf16 = s.d_bf16;
+  for (int k = 0; k < kMaxLevels; ++k) p.grid[k] = k < s.K ? d.grid[k] : 0.f;
+  p.logits = fptr(L, L->lay.logits);
+  p.m_logits = fptr(L, L->lay.m_logits);
+  p.scales = fptr(L, L->lay.scales);
+  p.m_scales = fptr(L, L->lay.m_scales);
+  p.W = L->ws + L->lay.W;
+  p.D = L->ws + L->lay.D;
+  p.G = fptr(L, L->lay.G);
+  p.key0 = static_cast<uint32_t>(d.seed);
+  p.key1 = static_cast<uint32_t>(d.seed >> 32);
+  p.noise = (d.flags & GSQ_FLAG_NO_NOISE) ? 0 : 1;
+  p.lr_l = d.lr_logits;
+  p.lr_s = d.lr_scales;
+  p.b1 = d.beta1;
+  p.b2 = d.beta2;
+  p.wd_l = d.wd_logits;
+  p.wd_s = d.wd_scales;
+  p.scales_frozen = (d.lr_scales == 0.f && d.wd_scales == 0.f) ? 1 : 0;
+  p.loss_partials = reinterpret_cast<double*>(L->ws + L->lay.partials);
+  p.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+  return p;
+}
+
+void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
+  slot = -1;
+  if (!L->profiling || L->ev_used >= kMaxProfileEvents) return;
+  const int i = L->ev_used;
+  if (static_cast<int>(L->ev_kind.size()) <= i) {
+    cudaEvent_t a, b;
+    if (cudaEventCreate(&a) != cudaSuccess) return;
+    if (cudaEventCreate(&b) != cudaSuccess) {
+      cudaEventDestroy(a);
+      return;
+    }
+    L->ev.push_back(a);
+    L->ev.push_back(b);
+    L->ev_kind.push_back(kind);
+  }
+  L->ev_kind[i] = kind;
+  cudaEventRecord(L->ev[2 * i], s);
+  slot = i;
+  L->ev_used = i + 1;
+}
+
+void prof_end(gsq_layer* L, int slot, cudaStream_t s) {
+  if (slot < 0) return;
+  cudaEventRecord(L->ev[2 * slot + 1], s);
+  L->last_stream = s;
+}
+
+gsq_status launch_fwd(gsq_layer* L, uint64_t step, float tau, float kappa, float* what,
+                      cudaStream_t s) {
+  EwParams p = base_params(L);
+  p.t = static_cast<uint32_t>(step);
+  p.kappa = kappa;
+  p.inv_tau = static_cast<float>(1.0 / tau);
+  p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
+  p.what = what;
+  int slot;
+  prof_begin(L, GSQ_K_FORWARD, s, slot);
+  const cudaError_t e = launch_forward(p, L->grid_fwd, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "forward kernel");
+  L->d_ready = true;
+  L->d_step = step;
+  L->d_tau = tau;
+  L->d_kappa = kappa;
+  return GSQ_OK;
+}
+
+gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
+  const Shape& sh = L->shape;
+  int slot;
+  prof_begin(L, GSQ_K_GEMM, s, slot);
+  cudaError_t e;
+  if (sh.d_bf16) {
+    TcGemm g;
+    g.E = static_cast<int>(sh.E);
+    g.R = static_cast<int>(sh.R);
+    g.C = static_cast<int>(sh.C);
+    g.D = L->ws + L->lay.D;
+    g.H = L->ws + L->lay.H;
+    g.G = fptr(L, L->lay.G);
+    g.alpha = 2.0f;
+    g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+    e = launch_tc_gemm(g, L->num_sms, s);
+  } else {
+    SimtGemm g;
+    g.batch = static_cast<int>(sh.E);
+    g.M = static_cast<int>(sh.R);
+    g.N = static_cast<int>(sh.C);
+    g.Kd = static_cast<int>(sh.C);
+    g.A = L->ws + L->lay.D;
+    g.sam = sh.C;
+    g.sak = 1;
+    g.sab = sh.R * sh.C;
+    g.B = L->ws + L->lay.H;
+    g.sbk = sh.C;
+    g.sbn = 1;
+    g.sbb = sh.C * sh.C;
+    g.C = fptr(L, L->lay.G);
+    g.ldc = sh.C;
+    g.scb = sh.R * sh.C;
+    g.alpha = 2.0f;
+    g.bf16_inputs = 0;
+    e = launch_simt_gemm(g, s);
+  }
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "loss GEMM");
+  return GSQ_OK;
+}
+
+size_t tensor_bytes(const gsq_layer* L, int which) {
+  const Shape& s = L->shape;
+  const size_t n = static_cast<size_t>(s.n), ng = static_cast<size_t>(s.ng);
+  switch (which) {
+    case GSQ_T_LOGITS:
+    case GSQ_T_MOM_LOGITS: return 4 * n * s.K;
+    case GSQ_T_SCALES:
+    case GSQ_T_MOM_SCALES: return 4 * ng;
+    case GSQ_T_D: return n * (s.d_bf16 ? 2 : 4);
+    case GSQ_T_G: return 4 * n;
+    case GSQ_T_W: return n * (s.w_bf16 ? 2 : 4);
+    case GSQ_T_H: return static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4);
+    case GSQ_T_KQ_D: return s.kquant ? 2 * (n / kSuperBlock) : 0;
+    case GSQ_T_KQ_SC: return s.kquant ? n / kSubBlock : 0;
+    default: return 0;
+  }
+}
+
+size_t tensor_offset(const gsq_layer* L, int which) {
+  switch (which) {
+    case GSQ_T_LOGITS: return L->lay.logits;
+    case GSQ_T_MOM_LOGITS: return L->lay.m_logits;
+    case GSQ_T_SCALES: return L->lay.scales;
+    case GSQ_T_MOM_SCALES: return L->lay.m_scales;
+    case GSQ_T_D: return L->lay.D;
+    case GSQ_T_G: return L->lay.G;
+    case GSQ_T_W: return L->lay.W;
+    case GSQ_T_H: return L->lay.H;
+    case GSQ_T_KQ_D: return L->lay.kq_d;
+    case GSQ_T_KQ_SC: return L->lay.kq_sc;
+    default: return 0;
+  }
+}
+
+size_t code_section_bytes(int64_t n, int K) {
+  const int bits = K <= 4 ? 2 : 3;
+  const size_t raw = static_cast<size_t>((n + 31) / 32) * 4 * bits;
+  return (raw + 15) / 16 * 16;
+}
+
+size_t packed_bytes(const gsq_layer* L) {
+  const Shape& s = L->shape;
+  if (s.kquant) return static_cast<size_t>(s.n / kSuperBlock) * kKqRecord;
+  return code_section_bytes(s.n, s.K) + 2 * static_cast<size_t>(s.ng);
+}
+
+}  // namespace
+
+extern "C" {
+
+gsq_status gsq_workspace_size(const gsq_layer_desc* desc, size_t* bytes) {
+  GSQ_INJECT("gsq_workspace_size");
+  if (!bytes) return fail(GSQ_ERR_INVALID_ARG, "bytes is NULL");
+  const gsq_status st = validate_desc(desc);
+  if (st != GSQ_OK) return st;
+  *bytes = layout_of(shape_of(*desc)).total;
+  return GSQ_OK;
+}
+
+gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t bytes, void* stream,
+                          gsq_layer** out) {
+  GSQ_INJECT("gsq_init_layer");
+  if (!out) return fail(GSQ_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  gsq_status st = validate_desc(desc);
+  if (st != GSQ_OK) return st;
+  if (!desc->W || !desc->calib) return fail(GSQ_ERR_INVALID_ARG, "W and calib must be device pointers");
+  if (!workspace) return fail(GSQ_ERR_WORKSPACE, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+    return fail(GSQ_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const Shape sh = shape_of(*desc);
+  const Layout lay = layout_of(sh);
+  if (bytes < lay.total)
+    return fail(GSQ_ERR_WORKSPACE, "workspace too small: %zu < %zu bytes", bytes, lay.total);
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+  if (prop.major != 10 || prop.minor != 3)
+    return fail(GSQ_ERR_UNSUPPORTED, "libgsq is built for sm_103 (found sm_%d%d)", prop.major, prop.minor);
+  const bool tc = tc_gemm_supported(dev);
+  if (sh.d_bf16 && !tc) return fail(GSQ_ERR_UNSUPPORTED, "tensor-map encoder unavailable for the bf16 GEMM");
+
+  gsq_layer* L = new (std::nothrow) gsq_layer();
+  if (!L) return fail(GSQ_ERR_INVALID_ARG, "host allocation failed");
+  L->magic = kMagic;
+  L->desc = *desc;
+  L->desc.W = nullptr;      // borrowed pointers are not kept
+  L->desc.calib = nullptr;
+  L->shape = sh;
+  L->lay = lay;
+  L->ws = static_cast<uint8_t*>(workspace);
+  L->device = dev;
+  L->num_sms = prop.multiProcessorCount;
+  L->tc = tc;
+  L->d_ready = false;
+  L->profiling = false;
+  L->ev_used = 0;
+  L->last_stream = nullptr;
+  const int64_t nq_blocks = (sh.n / 4 + kEwThreads - 1) / kEwThreads;
+  auto clamp_grid = [&](int g) {
+    int64_t v = g < nq_blocks ? g : nq_blocks;
+    if (v > kMaxPartials) v = kMaxPartials;
+    return static_cast<int>(v < 1 ? 1 : v);
+  };
+  L->grid_fwd = clamp_grid(ew_grid_size(sh.K, 0, L->num_sms));
+  L->grid_bwd = clamp_grid(ew_grid_size(sh.K, 1, L->num_sms));
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DevFlags* flags = reinterpret_cast<DevFlags*>(L->ws + lay.flags);
+  auto bail = [&](gsq_status code) {
+    delete L;
+    return code;
+  };
+  if ((e = cudaMemsetAsync(flags, 0, sizeof(DevFlags), s)) != cudaSuccess)
+    return bail(cuda_fail(e, "clear flags"));
+  const size_t wbytes = static_cast<size_t>(sh.n) * (sh.w_bf16 ? 2 : 4);
+  if ((e = cudaMemcpyAsync(L->ws + lay.W, desc->W, wbytes, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "copy W"));
+  if ((e = launch_nonfinite_scan(L->ws + lay.W, sh.n, sh.w_bf16, &flags->nonfinite, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "scan W"));
+  const int64_t calib_count = sh.x_mode ? sh.E * desc->n_tokens * sh.C : sh.E * sh.C * sh.C;
+  if ((e = launch_nonfinite_scan(desc->calib, calib_count, 0, &flags->nonfinite, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "scan calib"));
+
+  int slot;
+  prof_begin(L, GSQ_K_INIT, s, slot);
+  const float* hsrc = desc->calib;
+  if (sh.x_mode) {
+    SimtGemm g;  // H[e] = X[e]^T X[e]
+    g.batch = static_cast<int>(sh.E);
+    g.M = static_cast<int>(sh.C);
+    g.N = static_cast<int>(sh.C);
+    g.Kd = static_cast<int>(desc->n_tokens);
+    g.A = desc->calib;
+    g.sam = 1;
+    g.sak = sh.C;
+    g.sab = desc->n_tokens * sh.C;
+    g.B = desc->calib;
+    g.sbk = sh.C;
+    g.sbn = 1;
+    g.sbb = desc->n_tokens * sh.C;
+    g.C = fptr(L, lay.hscratch);
+    g.ldc = sh.C;
+    g.scb = sh.C * sh.C;
+    g.alpha = 1.0f;
+    g.bf16_inputs = 0;
+    if ((e = launch_simt_gemm(g, s)) != cudaSuccess) return bail(cuda_fail(e, "X^T X"));
+    hsrc = fptr(L, lay.hscratch);
+  }
+  if ((e = launch_symmetrize(hsrc, L->ws + lay.H, static_cast<int>(sh.E), static_cast<int>(sh.C),
+                             sh.d_bf16, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "symmetrise H"));
+
+  InitParams ip;
+  std::memset(&ip, 0, sizeof(ip));
+  ip.n = sh.n;
+  ip.K = sh.K;
+  ip.group = sh.group;
+  ip.kquant = sh.kquant;
+  ip.w_bf16 = sh.w_bf16;
+  for (int k = 0; k < kMaxLevels; ++k) ip.grid[k] = k < sh.K ? desc->grid[k] : 0.f;
+  ip.init_bias = desc->init_bias;
+  ip.W = L->ws + lay.W;
+  ip.logits = fptr(L, lay.logits);
+  ip.m_logits = fptr(L, lay.m_logits);
+  ip.scales = fptr(L, lay.scales);
+  ip.m_scales = fptr(L, lay.m_scales);
+  ip.kq_d = sh.kquant ? reinterpret_cast<uint16_t*>(L->ws + lay.kq_d) : nullptr;
+  ip.kq_sc = sh.kquant ? reinterpret_cast<int8_t*>(L->ws + lay.kq_sc) : nullptr;
+  if ((e = launch_init_state(ip, L->num_sms, s)) != cudaSuccess) return bail(cuda_fail(e, "init state"));
+  prof_end(L, slot, s);
+
+  unsigned int bad = 0;
+  if ((e = cudaMemcpyAsync(&bad, &flags->nonfinite, sizeof(bad), cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "read scan result"));
+  if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return bail(cuda_fail(e, "init"));
+  if (bad) return bail(fail(GSQ_ERR_NONFINITE, "W or calib holds %u non-finite values", bad));
+  register_live(L);
+  *out = L;
+  return GSQ_OK;
+}
+
+gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float next_tau,
+                    float next_kappa, void* stream, float* loss_dev, float* grad_logits_dev,
+                    float* grad_scales_dev) {
+  GSQ_INJECT("gsq_step");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (step >= (1ull << 32)) return fail(GSQ_ERR_INVALID_ARG, "step must be < 2^32");
+  if (!(tau > 0.f) || !std::isfinite(tau) || !std::isfinite(kappa))
+    return fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");
+  const bool export_mode = grad_logits_dev || grad_scales_dev;
+  const bool lookahead = !export_mode && next_tau > 0.f;
+  if (lookahead) {
+    if (!std::isfinite(next_tau) || !std::isfinite(next_kappa))
+      return fail(GSQ_ERR_INVALID_ARG, "next_tau / next_kappa must be finite");
+    if (step + 1 >= (1ull << 32)) return fail(GSQ_ERR_INVALID_ARG, "step + 1 must be < 2^32");
+  }
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  gsq_status st;
+  if (!(L->d_ready && L->d_step == step && L->d_tau == tau && L->d_kappa == kappa)) {
+    if ((st = launch_fwd(L, step, tau, kappa, nullptr, s)) != GSQ_OK) return st;
+  }
+  if ((st = launch_gemm(L, s)) != GSQ_OK) return st;
+
+  EwParams p = base_params(L);
+  p.t = static_cast<uint32_t>(step);
+  p.kappa = kappa;
+  p.inv_tau = static_cast<float>(1.0 / tau);
+  p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
+  p.lookahead = lookahead ? 1 : 0;
+  if (lookahead) {
+    p.t_next = static_cast<uint32_t>(step + 1);
+    p.kappa_next = next_kappa;
+    p.inv_tau_next = static_cast<float>(1.0 / next_tau);
+  }
+  p.grad_logits = grad_logits_dev;
+  p.grad_scales = grad_scales_dev;
+  p.loss_out = loss_dev;
+  int slot;
+  prof_begin(L, GSQ_K_BACKWARD, s, slot);
+  const cudaError_t e = launch_backward(p, L->grid_bwd, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+  if (lookahead) {
+    L->d_ready = true;
+    L->d_step = step + 1;
+    L->d_tau = next_tau;
+    L->d_kappa = next_kappa;
+  } else if (!export_mode) {
+    L->d_ready = false;
+  }
+  return GSQ_OK;
+}
+
+gsq_status gsq_forward(gsq_layer* L, uint64_t step, float tau, float kappa, void* stream,
+                       float* what_dev) {
+  GSQ_INJECT("gsq_forward");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (step >= (1ull << 32)) return fail(GSQ_ERR_INVALID_ARG, "step must be < 2^32");
+  if (!(tau > 0.f) || !std::isfinite(tau) || !std::isfinite(kappa))
+    return fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");
+  DeviceGuard guard(L->device);
+  return launch_fwd(L, step, tau, kappa, what_dev, static_cast<cudaStream_t>(stream));
+}
+
+gsq_status gsq_project(gsq_layer* L, void* stream, uint8_t* codes_dev, float* margin_dev) {
+  GSQ_INJECT("gsq_project");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!codes_dev && !margin_dev) return GSQ_OK;
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ProjectParams p;
+  p.n = L->shape.n;
+  p.K = L->shape.K;
+  p.logits = fptr(L, L->lay.logits);
+  p.codes = codes_dev;
+  p.margin = margin_dev;
+  int slot;
+  prof_begin(L, GSQ_K_PROJECT, s, slot);
+  const cudaError_t e = launch_project(p, L->num_sms, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "project kernel");
+  return GSQ_OK;
+}
+
+gsq_status gsq_packed_size(const gsq_layer* L, size_t* bytes) {
+  GSQ_INJECT("gsq_packed_size");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!bytes) return fail(GSQ_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = packed_bytes(L);
+  return GSQ_OK;
+}
+
+gsq_status gsq_pack(gsq_layer* L, void* stream, void* out_dev, size_t cap, size_t* written) {
+  GSQ_INJECT("gsq_pack");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!out_dev) return fail(GSQ_ERR_INVALID_ARG, "out_dev is NULL");
+  const size_t need = packed_bytes(L);
+  if (cap < need) return fail(GSQ_ERR_INVALID_ARG, "pack buffer too small: %zu < %zu", cap, need);
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  PackParams p;
+  p.n = L->shape.n;
+  p.K = L->shape.K;
+  p.group = L->shape.group;
+  p.kquant = L->shape.kquant;
+  p.logits = fptr(L, L->lay.logits);
+  p.scales = fptr(L, L->lay.scales);
+  p.kq_d = L->shape.kquant ? reinterpret_cast<const uint16_t*>(L->ws + L->lay.kq_d) : nullptr;
+  p.kq_sc = L->shape.kquant ? reinterpret_cast<const int8_t*>(L->ws + L->lay.kq_sc) : nullptr;
+  p.out = static_cast<uint8_t*>(out_dev);
+  p.code_bytes = static_cast<int64_t>(code_section_bytes(L->shape.n, L->shape.K));
+  int slot;
+  prof_begin(L, GSQ_K_PACK, s, slot);
+  const cudaError_t e = launch_pack(p, L->num_sms, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "pack kernel");
+  if (written) *written = need;
+  return GSQ_OK;
+}
+
+gsq_status gsq_tensor_size(const gsq_layer* L, int32_t which, size_t* bytes) {
+  GSQ_INJECT("gsq_tensor_size");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!bytes) return fail(GSQ_ERR_INVALID_ARG, "bytes is NULL");
+  if (which < GSQ_T_LOGITS || which > GSQ_T_KQ_SC) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
+  *bytes = tensor_bytes(L, which);
+  return GSQ_OK;
+}
+
+static gsq_status copy_tensor(gsq_layer* L, int32_t which, void* dst, const void* src, size_t bytes,
+                              void* stream, const char* fn) {
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (which < GSQ_T_LOGITS || which > GSQ_T_KQ_SC) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
+  const size_t need = tensor_bytes(L, which);
+  if (need == 0) return fail(GSQ_ERR_INVALID_ARG, "%s: layer has no tensor %d", fn, which);
+  if (bytes != need) return fail(GSQ_ERR_INVALID_ARG, "%s: bytes %zu != tensor size %zu", fn, bytes, need);
+  if (!dst || !src) return fail(GSQ_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+  DeviceGuard guard(L->device);
+  const cudaError_t e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return GSQ_OK;
+}
+
+gsq_status gsq_get_tensor(gsq_layer* L, int32_t which, void* dst_dev, size_t bytes, void* stream) {
+  GSQ_INJECT("gsq_get_tensor");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  return copy_tensor(L, which, dst_dev, L->ws + tensor_offset(L, which), bytes, stream, "gsq_get_tensor");
+}
+
+gsq_status gsq_set_tensor(gsq_layer* L, int32_t which, const void* src_dev, size_t bytes, void* stream) {
+  GSQ_INJECT("gsq_set_tensor");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  const gsq_status st =
+      copy_tensor(L, which, L->ws + tensor_offset(L, which), src_dev, bytes, stream, "gsq_set_tensor");
+  if (st == GSQ_OK) L->d_ready = false;
+  return st;
+}
+
+gsq_status gsq_sync_status(gsq_layer* L, void* stream) {
+  GSQ_INJECT("gsq_sync_status");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "gsq_sync_status");
+  DevFlags* flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+  unsigned int err = 0;
+  e = cudaMemcpy(&err, &flags->error, sizeof(err), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "read error word");
+  if (err) {
+    cudaMemset(&flags->error, 0, sizeof(err));
+    return fail(GSQ_ERR_TIMEOUT, "a bounded device-side wait gave up (code 0x%x)", err);
+  }
+  return GSQ_OK;
+}
+
+gsq_status gsq_profile_enable(gsq_layer* L, int32_t on) {
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  L->profiling = on != 0;
+  return GSQ_OK;
+}
+
+gsq_status gsq_profile_read(gsq_layer* L, gsq_profile* out) {
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!out) return fail(GSQ_ERR_INVALID_ARG, "out is NULL");
+  std::memset(out, 0, sizeof(*out));
+  DeviceGuard guard(L->device);
+  if (L->ev_used > 0) {
+    cudaError_t e = cudaEventSynchronize(L->ev[2 * (L->ev_used - 1) + 1]);
+    if (e != cudaSuccess) return cuda_fail(e, "profile sync");
+    for (int i = 0; i < L->ev_used; ++i) {
+      float ms = 0.f;
+      e = cudaEventElapsedTime(&ms, L->ev[2 * i], L->ev[2 * i + 1]);
+      if (e != cudaSuccess) return cuda_fail(e, "profile elapsed");
+      out->launches[L->ev_kind[i]] += 1;
+      out->total_ms[L->ev_kind[i]] += ms;
+    }
+  }
+  L->ev_used = 0;
+  return GSQ_OK;
+}
+
+gsq_status gsq_destroy(gsq_layer* L) {
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  unregister_live(L);
+  for (cudaEvent_t e : L->ev) cudaEventDestroy(e);
+  L->magic = 0;
+  delete L;
+  return GSQ_OK;
+}
+
+const char* gsq_last_error(void) { return g_last_error.c_str(); }
+
+const char* gsq_version(void) { return "0.1.0"; }
+
+}  // extern "C"

@@ -1,0 +1,795 @@
+// Elementwise kernels of the GSQ step (HBM-bound): initial state, forward
+// (noise + tempered softmax + soft weight, Alg. 1), fused backward + Lion
+// (+ the next step's forward), hard projection and packing.
+//
+// Data layout in HBM (n = E*R*C, flat index i = (e*R + r)*C + c):
+//   logits, logit momenta : K planes of n fp32 ([K][E][R][C]), so every level is
+//                           a unit-stride stream read with 128-bit loads;
+//   scales, scale momenta : [n / G] fp32;  W, D : [n] (bf16 or fp32);  G : [n] fp32.
+// Work split: one thread owns a quad of 4 consecutive weights (one float4 per
+// plane); a scale group of G consecutive weights is G/4 adjacent lanes of one
+// warp, so per-group sums are warp shuffles.  Grid-stride loops are warp-uniform.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <type_traits>
+
+#include "gsq_internal.h"
+
+namespace gsq {
+namespace {
+
+// ---------------------------------------------------------------------------
+// Counter-based Gumbel noise (Alg. 1 draw; resampled every step, §3.3).
+// Philox4x32-10 from its definition (Salmon, Moraes, Dror, Shaw, SC'11):
+// S-box multipliers 0xD2511F53 / 0xCD9E8D57, Weyl key increments 0x9E3779B9 /
+// 0xBB67AE85.  Counter (lo32(i), hi32(i), t, level block), key = seed.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
+                                               uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c0;
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c0);
+    const uint32_t lo1 = 0xCD9E8D57u * c2;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2);
+    c0 = hi1 ^ c1 ^ k0;
+    c1 = lo1;
+    c2 = hi0 ^ c3 ^ k1;
+    c3 = lo0;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return make_uint4(c0, c1, c2, c3);
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float fast_log2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// -ln(u) for u in [2^-24, 1 - 2^-24], accurate to a few ulp in relative terms
+// even as u -> 1 (where -ln u -> 0).  Argument reduction u = 2^e m with m in
+// [sqrt(1/2), sqrt(2)), then ln m = 2 atanh(y), y = (m - 1)/(m + 1), by its
+// odd power series 2(y + y^3/3 + y^5/5 + ...) (Abramowitz & Stegun 4.1.27);
+// |y| <= 0.1716, so terms through y^9 leave a relative remainder below 2e-9.
+__device__ __forceinline__ float neg_log_unit(float u) {
+  const uint32_t b = __float_as_uint(u);
+  int e = static_cast<int>(b >> 23) - 127;
+  float m = __uint_as_float((b & 0x007FFFFFu) | 0x3F800000u);  // [1, 2)
+  if (m > 1.41421356f) {
+    m *= 0.5f;
+    e += 1;
+  }
+  const float y = __fdividef(m - 1.0f, m + 1.0f);
+  const float y2 = y * y;
+  const float poly =
+      fmaf(y2, fmaf(y2, fmaf(y2, fmaf(y2, 1.0f / 9.0f, 1.0f / 7.0f), 1.0f / 5.0f), 1.0f / 3.0f),
+           1.0f);
+  const float ln_m = 2.0f * y * poly;
+  return -fmaf(static_cast<float>(e), 0.69314718055994531f, ln_m);
+}
+
+// g = -ln(-ln u), u = (floor(x / 2^9) + 1/2) 2^-23 built exactly from the bits.
+__device__ __forceinline__ float gumbel_from_word(uint32_t x) {
+  const float one_plus = __uint_as_float(0x3F800000u | (x >> 9));  // 1 + j 2^-23
+  const float u = one_plus - __uint_as_float(0x3F7FFFFFu);         // (j + 1/2) 2^-23, exact
+  const float E = neg_log_unit(u);
+  return -0.69314718055994531f * fast_log2(E);
+}
+
+template <int K>
+__device__ __forceinline__ void draw_noise(uint32_t key0, uint32_t key1, uint32_t t, uint64_t i,
+                                           int noise, float (&g)[K]) {
+  if (!noise) {
+#pragma unroll
+    for (int k = 0; k < K; ++k) g[k] = 0.0f;
+    return;
+  }
+#pragma unroll
+  for (int blk = 0; blk < (K + 3) / 4; ++blk) {
+    const uint4 w = philox4x32_10(static_cast<uint32_t>(i), static_cast<uint32_t>(i >> 32), t,
+                                  static_cast<uint32_t>(blk), key0, key1);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (4 * blk + j < K) g[4 * blk + j] = gumbel_from_word(ws[j]);
+  }
+}
+
+// Tempered softmax over the levels and the soft value (Alg. 1):
+//   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k.
+// w~ is carried as q_m + delta, delta = sum_j p_j (q_j - q_m), m = argmax z, so
+// q_k - w~ = (q_k - q_m) - delta keeps full relative accuracy when p is
+// nearly one-hot.
+template <int K>
+struct Soft {
+  float p[K];
+  float qm;
+  float delta;
+};
+
+template <int K>
+__device__ __forceinline__ void relax(const float (&l)[K], const float (&g)[K], float kappa,
+                                      float scale_log2, const float (&q)[kMaxLevels],
+                                      Soft<K>& s) {
+  float z[K];
+  float zmax = -INFINITY;
+  int m = 0;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    z[k] = fmaf(kappa, l[k], g[k]) * scale_log2;  // (kappa l + g)/tau in log2 units
+    if (z[k] > zmax) {
+      zmax = z[k];
+      m = k;
+    }
+  }
+  float sum = 0.0f;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    s.p[k] = fast_exp2(z[k] - zmax);
+    sum += s.p[k];
+  }
+  const float inv = __fdividef(1.0f, sum);
+  float qm = q[0];
+#pragma unroll
+  for (int k = 1; k < K; ++k) qm = (m == k) ? q[k] : qm;
+  float delta = 0.0f;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    s.p[k] *= inv;
+    delta = fmaf(s.p[k], q[k] - qm, delta);
+  }
+  s.qm = qm;
+  s.delta = delta;
+}
+
+__device__ __forceinline__ void load_w4(const void* W, int64_t q, int bf16, float (&w)[4]) {
+  if (bf16) {
+    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(W) + q);
+    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&raw.x);
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&raw.y);
+    const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+    w[0] = fa.x; w[1] = fa.y; w[2] = fb.x; w[3] = fb.y;
+  } else {
+    const float4 v = __ldg(reinterpret_cast<const float4*>(W) + q);
+    w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+  }
+}
+
+// Rounds D to its storage precision in place and stores it.
+__device__ __forceinline__ void store_d4(void* D, int64_t q, int bf16, float (&d)[4]) {
+  if (bf16) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(d[0], d[1]);
+    const __nv_bfloat162 b = __floats2bfloat162_rn(d[2], d[3]);
+    const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+    d[0] = fa.x; d[1] = fa.y; d[2] = fb.x; d[3] = fb.y;
+    uint2 raw;
+    raw.x = *reinterpret_cast<const uint32_t*>(&a);
+    raw.y = *reinterpret_cast<const uint32_t*>(&b);
+    reinterpret_cast<uint2*>(D)[q] = raw;
+  } else {
+    reinterpret_cast<float4*>(D)[q] = make_float4(d[0], d[1], d[2], d[3]);
+  }
+}
+
+__device__ __forceinline__ float round_d(float d, int bf16) {
+  return bf16 ? __bfloat162float(__float2bfloat16_rn(d)) : d;
+}
+
+__device__ __forceinline__ float sign_of(float c) {
+  return c > 0.0f ? 1.0f : (c < 0.0f ? -1.0f : 0.0f);
+}
+
+__device__ __forceinline__ float group_sum(float v, int seg) {
+  for (int off = 1; off < seg; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+__device__ __forceinline__ void load_grid(const EwParams& P, float (&q)[kMaxLevels]) {
+#pragma unroll
+  for (int k = 0; k < kMaxLevels; ++k) q[k] = P.grid[k];
+}
+
+// Deterministic loss reduction: per-block double partials, summed in block
+// order by the last block to finish (no device-side wait).
+__device__ __forceinline__ void reduce_loss(float acc, const EwParams& P) {
+  __shared__ double red[kEwThreads / 32];
+  __shared__ bool is_last;
+  double v = static_cast<double>(acc);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
+    P.loss_partials[blockIdx.x] = s;
+    __threadfence();
+    const unsigned int prev = atomicAdd(&P.flags->blocks_done, 1u);
+    is_last = (prev == gridDim.x - 1);
+  }
+  __syncthreads();
+  if (is_last && threadIdx.x == 0) {
+    __threadfence();
+    double s = 0.0;
+    for (unsigned int b = 0; b < gridDim.x; ++b) s += __ldcg(P.loss_partials + b);
+    if (P.loss_out) *P.loss_out = static_cast<float>(s);
+    P.flags->blocks_done = 0u;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Forward: D = s * w~ - W for step (t, tau, kappa); optional W^ export.
+// Bytes per weight: read 4K (logits) + b_W, write 2 or 4 (D).
+// ---------------------------------------------------------------------------
+template <int K>
+__global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
+  float q[kMaxLevels];
+  load_grid(P, q);
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const float scale_log2 = P.inv_tau * 1.4426950408889634f;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+       base < P.nq; base += stride) {
+    const int64_t qi = base + lane;
+    if (qi >= P.nq) continue;
+    float l[K][4];
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qi);
+      l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
+    }
+    float w[4];
+    load_w4(P.W, qi, P.w_bf16, w);
+    const float s = __ldg(P.scales + ((qi * 4) >> P.log2_group));
+    float d[4], what[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint64_t i = static_cast<uint64_t>(qi) * 4 + j;
+      float lj[K], g[K];
+#pragma unroll
+      for (int k = 0; k < K; ++k) lj[k] = l[k][j];
+      draw_noise<K>(P.key0, P.key1, P.t, i, P.noise, g);
+      Soft<K> sm;
+      relax<K>(lj, g, P.kappa, scale_log2, q, sm);
+      // D = s w~ - W as one rounding (identical in every kernel that forms D)
+      const float wt = sm.qm + sm.delta;
+      what[j] = __fmul_rn(s, wt);
+      d[j] = __fmaf_rn(s, wt, -w[j]);
+    }
+    store_d4(P.D, qi, P.d_bf16, d);
+    if (P.what) reinterpret_cast<float4*>(P.what)[qi] = make_float4(what[0], what[1], what[2], what[3]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Fused backward for step t: recompute the noise and p, loss partial
+// 1/2 D*G, gradients (App. B softmax Jacobian), per-group scale gradient by
+// warp shuffles, Lion in place; then (look-ahead) the forward of step t+1 from
+// the updated registers.  Bytes per weight with look-ahead: read 8K + 4 + b_W,
+// write 8K + 2 (D bf16).
+// ---------------------------------------------------------------------------
+template <int K, bool kExport>
+__global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
+  float q[kMaxLevels];
+  load_grid(P, q);
+  const int lane = threadIdx.x & 31;
+  const int seg = P.group >> 2;  // lanes per scale group
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const float scale_log2 = P.inv_tau * 1.4426950408889634f;
+  const float scale_log2_next = P.inv_tau_next * 1.4426950408889634f;
+  const float decay_l = 1.0f - P.lr_l * P.wd_l;
+  const float decay_s = 1.0f - P.lr_s * P.wd_s;
+  float loss_acc = 0.0f;
+
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+       base < P.nq; base += stride) {
+    const int64_t qi = base + lane;
+    const bool active = qi < P.nq;
+    const int64_t qc = active ? qi : 0;
+    // l: logits; m: Lion momentum (or, in export mode, the logit gradient)
+    float l[K][4], m[K][4];
+    float w[4] = {0.f, 0.f, 0.f, 0.f};
+    float4 gv = make_float4(0.f, 0.f, 0.f, 0.f);
+    float s = 0.0f, ms = 0.0f;
+    const int64_t gidx = (qc * 4) >> P.log2_group;
+#pragma unroll
+    for (int k = 0; k < K; ++k)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) l[k][j] = m[k][j] = 0.0f;
+    if (active) {
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qi);
+        l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
+      }
+      if (!kExport) {
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+          const float4 v = __ldcs(reinterpret_cast<const float4*>(P.m_logits + k * P.n) + qi);
+          m[k][0] = v.x; m[k][1] = v.y; m[k][2] = v.z; m[k][3] = v.w;
+        }
+      }
+      gv = __ldcs(reinterpret_cast<const float4*>(P.G) + qi);
+      load_w4(P.W, qi, P.w_bf16, w);
+      s = __ldg(P.scales + gidx);
+      if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
+    }
+    const float Gq[4] = {gv.x, gv.y, gv.z, gv.w};
+    float ds = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint64_t i = static_cast<uint64_t>(qc) * 4 + j;
+      float lj[K], g[K];
+#pragma unroll
+      for (int k = 0; k < K; ++k) lj[k] = l[k][j];
+      draw_noise<K>(P.key0, P.key1, P.t, i, P.noise, g);
+      Soft<K> sm;
+      relax<K>(lj, g, P.kappa, scale_log2, q, sm);
+      const float wt = sm.qm + sm.delta;
+      const float dj = round_d(__fmaf_rn(s, wt, -w[j]), P.d_bf16);
+      loss_acc = fmaf(0.5f * dj, Gq[j], loss_acc);
+      ds = fmaf(Gq[j], wt, ds);
+      const float A = P.kappa_over_tau * Gq[j] * s;
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        // dL/dl_k = (kappa/tau) G s p_k (q_k - w~)   (softmax Jacobian, App. B)
+        const float dl = A * sm.p[k] * ((q[k] - sm.qm) - sm.delta);
+        if (kExport) {
+          m[k][j] = dl;
+        } else {
+          // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l (1 - lr wd) - lr sign(c);
+          // m <- b2 m + (1-b2) g
+          const float c = fmaf(P.b1, m[k][j], (1.0f - P.b1) * dl);
+          l[k][j] = fmaf(l[k][j], decay_l, -P.lr_l * sign_of(c));
+          m[k][j] = fmaf(P.b2, m[k][j], (1.0f - P.b2) * dl);
+        }
+      }
+    }
+    ds = group_sum(ds, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
+
+    if (kExport) {
+      if (active) {
+        if (P.grad_logits) {
+#pragma unroll
+          for (int k = 0; k < K; ++k)
+            reinterpret_cast<float4*>(P.grad_logits + k * P.n)[qi] =
+                make_float4(m[k][0], m[k][1], m[k][2], m[k][3]);
+        }
+        if (P.grad_scales && !P.scales_frozen && (lane & (seg - 1)) == 0) P.grad_scales[gidx] = ds;
+      }
+      continue;
+    }
+
+    if (!P.scales_frozen) {
+      const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
+      s = fmaf(s, decay_s, -P.lr_s * sign_of(c));
+      ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
+    }
+    if (active) {
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        __stcs(reinterpret_cast<float4*>(P.logits + k * P.n) + qi,
+               make_float4(l[k][0], l[k][1], l[k][2], l[k][3]));
+        __stcs(reinterpret_cast<float4*>(P.m_logits + k * P.n) + qi,
+               make_float4(m[k][0], m[k][1], m[k][2], m[k][3]));
+      }
+      if (!P.scales_frozen && (lane & (seg - 1)) == 0) {
+        P.scales[gidx] = s;
+        P.m_scales[gidx] = ms;
+      }
+      if (P.lookahead) {
+        // forward of step t+1 from the updated logits and scale (Alg. 1)
+        float d[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint64_t i = static_cast<uint64_t>(qi) * 4 + j;
+          float lj[K], g[K];
+#pragma unroll
+          for (int k = 0; k < K; ++k) lj[k] = l[k][j];
+          draw_noise<K>(P.key0, P.key1, P.t_next, i, P.noise, g);
+          Soft<K> sm;
+          relax<K>(lj, g, P.kappa_next, scale_log2_next, q, sm);
+          d[j] = __fmaf_rn(s, sm.qm + sm.delta, -w[j]);
+        }
+        store_d4(P.D, qi, P.d_bf16, d);
+      }
+    }
+  }
+  reduce_loss(loss_acc, P);
+}
+
+// ---------------------------------------------------------------------------
+// Initial state.  Group mode: s = absmax_g / max|q| (1 for an all-zero group);
+// RTN code k0 = argmin_k |W/s - q_k| (lowest k on ties); logits = bias on k0.
+// All decisions in fp32 with IEEE division, as the oracle takes them.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int rtn_code(float w, float s, const float (&q)[kMaxLevels], int K,
+                                        int zero_code) {
+  if (s == 0.0f) return zero_code;
+  const float x = __fdiv_rn(w, s);
+  int best = 0;
+  float bd = fabsf(x - q[0]);
+  for (int k = 1; k < K; ++k) {
+    const float dk = fabsf(x - q[k]);
+    if (dk < bd) {
+      bd = dk;
+      best = k;
+    }
+  }
+  return best;
+}
+
+struct InitConsts {
+  float q[kMaxLevels];
+  float qmax;
+  int zero_code;
+};
+
+__device__ __forceinline__ InitConsts init_consts(const InitParams& P) {
+  InitConsts c;
+  c.qmax = 0.0f;
+  c.zero_code = 0;
+  float zmin = INFINITY;
+  for (int k = 0; k < kMaxLevels; ++k) c.q[k] = P.grid[k];
+  for (int k = 0; k < P.K; ++k) {
+    c.qmax = fmaxf(c.qmax, fabsf(c.q[k]));
+    if (fabsf(c.q[k]) < zmin) {
+      zmin = fabsf(c.q[k]);
+      c.zero_code = k;
+    }
+  }
+  return c;
+}
+
+__device__ __forceinline__ void write_init_quad(const InitParams& P, int64_t qi, const int (&code)[4]) {
+  for (int k = 0; k < P.K; ++k) {
+    float4 v;
+    v.x = code[0] == k ? P.init_bias : 0.0f;
+    v.y = code[1] == k ? P.init_bias : 0.0f;
+    v.z = code[2] == k ? P.init_bias : 0.0f;
+    v.w = code[3] == k ? P.init_bias : 0.0f;
+    reinterpret_cast<float4*>(P.logits + k * P.n)[qi] = v;
+    reinterpret_cast<float4*>(P.m_logits + k * P.n)[qi] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+__global__ void __launch_bounds__(kEwThreads) k_init_group(const InitParams P) {
+  const InitConsts c = init_consts(P);
+  const int lane = threadIdx.x & 31;
+  const int seg = P.group >> 2;
+  const int64_t nq = P.n >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  int log2g = 0;
+  while ((1 << log2g) < P.group) ++log2g;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+       base < nq; base += stride) {
+    const int64_t qi = base + lane;
+    const bool active = qi < nq;
+    float w[4] = {0.f, 0.f, 0.f, 0.f};
+    if (active) load_w4(P.W, qi, P.w_bf16, w);
+    float amax = fmaxf(fmaxf(fabsf(w[0]), fabsf(w[1])), fmaxf(fabsf(w[2]), fabsf(w[3])));
+    for (int off = 1; off < seg; off <<= 1)
+      amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+    if (!active) continue;
+    const float s = amax == 0.0f ? 1.0f : __fdiv_rn(amax, c.qmax);
+    int code[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) code[j] = rtn_code(w[j], s, c.q, P.K, c.zero_code);
+    write_init_quad(P, qi, code);
+    if ((lane & (seg - 1)) == 0) {
+      const int64_t gi = (qi * 4) >> log2g;
+      P.scales[gi] = s;
+      P.m_scales[gi] = 0.0f;
+    }
+  }
+}
+
+// K-Quant-like two-level scales: one warp per 256-weight super-block, lane l
+// owns weights 8l..8l+7 (sub-block l/2).  s_j = absmax_16 / max|q|;
+// d = fp16_rne(max_j s_j / 31); sc_j = clamp(rne(s_j / d), -32, 31) (0 if d = 0);
+// effective scale d*sc_j (exact in fp32).
+__global__ void __launch_bounds__(kEwThreads) k_init_kquant(const InitParams P) {
+  const InitConsts c = init_consts(P);
+  const int lane = threadIdx.x & 31;
+  const int64_t nsb = P.n / kSuperBlock;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  for (int64_t sb = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       sb < nsb; sb += warps) {
+    const int64_t q0 = sb * (kSuperBlock / 4) + 2 * lane;  // first of this lane's two quads
+    float w[8];
+    {
+      float a[4], b[4];
+      load_w4(P.W, q0, P.w_bf16, a);
+      load_w4(P.W, q0 + 1, P.w_bf16, b);
+      for (int j = 0; j < 4; ++j) {
+        w[j] = a[j];
+        w[4 + j] = b[j];
+      }
+    }
+    float amax = 0.0f;
+    for (int j = 0; j < 8; ++j) amax = fmaxf(amax, fabsf(w[j]));
+    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
+    const float sj = __fdiv_rn(amax, c.qmax);
+    float smax = sj;
+    for (int off = 2; off < 32; off <<= 1) smax = fmaxf(smax, __shfl_xor_sync(0xffffffffu, smax, off));
+    const __half dh = __float2half_rn(__fdiv_rn(smax, 31.0f));
+    const float d = __half2float(dh);
+    int sc = 0;
+    if (d > 0.0f) sc = static_cast<int>(fminf(fmaxf(rintf(__fdiv_rn(sj, d)), -32.0f), 31.0f));
+    const float s = d * static_cast<float>(sc);
+    int code[2][4];
+    for (int j = 0; j < 8; ++j) code[j >> 2][j & 3] = rtn_code(w[j], s, c.q, P.K, c.zero_code);
+    write_init_quad(P, q0, code[0]);
+    write_init_quad(P, q0 + 1, code[1]);
+    if ((lane & 1) == 0) {
+      const int64_t sub = sb * (kSuperBlock / kSubBlock) + (lane >> 1);
+      P.scales[sub] = s;
+      P.m_scales[sub] = 0.0f;
+      P.kq_sc[sub] = static_cast<int8_t>(sc);
+    }
+    if (lane == 0) P.kq_d[sb] = __half_as_ushort(dh);
+  }
+}
+
+__global__ void k_nonfinite(const void* x, int64_t count, int bf16, unsigned int* counter) {
+  unsigned int bad = 0;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < count; i += stride) {
+    float v;
+    if (bf16)
+      v = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(x)[i]);
+    else
+      v = reinterpret_cast<const float*>(x)[i];
+    bad += isfinite(v) ? 0u : 1u;
+  }
+  for (int off = 16; off > 0; off >>= 1) bad += __shfl_down_sync(0xffffffffu, bad, off);
+  if ((threadIdx.x & 31) == 0 && bad) atomicAdd(counter, bad);
+}
+
+// ---------------------------------------------------------------------------
+// Hard projection: k* = argmax_k l_k (lowest k on ties), margin l_(1) - l_(2).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void argmax_margin(const float* logits, int64_t n, int K, int64_t i,
+                                              int& code, float& margin) {
+  float best = __ldcs(logits + i), second = -INFINITY;
+  code = 0;
+  for (int k = 1; k < K; ++k) {
+    const float v = __ldcs(logits + k * n + i);
+    if (v > best) {
+      second = best;
+      best = v;
+      code = k;
+    } else if (v > second) {
+      second = v;
+    }
+  }
+  margin = best - second;
+}
+
+__global__ void __launch_bounds__(kEwThreads) k_project(const ProjectParams P) {
+  const int64_t nq = P.n >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t qi = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; qi < nq; qi += stride) {
+    float best[4], second[4];
+    int code[4] = {0, 0, 0, 0};
+    {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits) + qi);
+      best[0] = v.x; best[1] = v.y; best[2] = v.z; best[3] = v.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) second[j] = -INFINITY;
+    for (int k = 1; k < P.K; ++k) {
+      const float4 v4 = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qi);
+      const float v[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (v[j] > best[j]) {
+          second[j] = best[j];
+          best[j] = v[j];
+          code[j] = k;
+        } else if (v[j] > second[j]) {
+          second[j] = v[j];
+        }
+      }
+    }
+    if (P.codes) {
+      const uint32_t packed = static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
+                              (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
+      reinterpret_cast<uint32_t*>(P.codes)[qi] = packed;
+    }
+    if (P.margin)
+      reinterpret_cast<float4*>(P.margin)[qi] =
+          make_float4(best[0] - second[0], best[1] - second[1], best[2] - second[2], best[3] - second[3]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Packing.  One warp per chunk of 32 consecutive weights: lane j projects weight
+// j of the chunk and contributes its code at bit b*j of the chunk's b-word
+// little-endian stream; the words are OR-reduced across the warp.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t stream_word(uint32_t code, int bits, int lane, int word) {
+  const int shift = bits * lane - 32 * word;  // position of this code inside `word`
+  if (shift >= 32 || shift <= -bits) return 0u;
+  return shift >= 0 ? (code << shift) : (code >> (-shift));
+}
+
+__global__ void __launch_bounds__(kEwThreads) k_pack_group(const PackParams P) {
+  const int lane = threadIdx.x & 31;
+  const int bits = P.K <= 4 ? 2 : 3;
+  const int64_t nchunks = (P.n + 31) / 32;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  uint32_t* words = reinterpret_cast<uint32_t*>(P.out);
+  for (int64_t ch = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       ch < nchunks; ch += warps) {
+    const int64_t i = ch * 32 + lane;
+    uint32_t code = 0;
+    if (i < P.n) {
+      int c;
+      float mg;
+      argmax_margin(P.logits, P.n, P.K, i, c, mg);
+      code = static_cast<uint32_t>(c);
+    }
+    for (int wd = 0; wd < bits; ++wd) {
+      const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(code, bits, lane, wd));
+      if (lane == wd) words[ch * bits + wd] = v;
+    }
+  }
+  // fp16 (round-to-nearest-even) group scales after the padded code section
+  uint16_t* sc = reinterpret_cast<uint16_t*>(P.out + P.code_bytes);
+  const int64_t ng = P.n / P.group;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < ng; g += stride)
+    sc[g] = __half_as_ushort(__float2half_rn(P.scales[g]));
+  // zero the padding words of the code section
+  const int64_t used = nchunks * bits;
+  for (int64_t wi = used + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+       wi < P.code_bytes / 4; wi += stride)
+    words[wi] = 0u;
+}
+
+__global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) {
+  __shared__ uint32_t rec[kEwThreads / 32][28];
+  const int lane = threadIdx.x & 31;
+  const int wib = threadIdx.x >> 5;
+  const int64_t nsb = P.n / kSuperBlock;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  for (int64_t sb = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + wib; sb < nsb; sb += warps) {
+    for (int ch = 0; ch < 8; ++ch) {
+      int c;
+      float mg;
+      argmax_margin(P.logits, P.n, P.K, sb * kSuperBlock + ch * 32 + lane, c, mg);
+      for (int wd = 0; wd < 3; ++wd) {
+        const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(static_cast<uint32_t>(c), 3, lane, wd));
+        if (lane == wd) rec[wib][ch * 3 + wd] = v;
+      }
+    }
+    uint32_t s6 = 0;
+    if (lane < 16) s6 = static_cast<uint32_t>(static_cast<int>(P.kq_sc[sb * 16 + lane]) + 32) & 63u;
+    for (int wd = 0; wd < 3; ++wd) {
+      const uint32_t v = __reduce_or_sync(0xffffffffu, lane < 16 ? stream_word(s6, 6, lane, wd) : 0u);
+      if (lane == wd) rec[wib][24 + wd] = v;
+    }
+    if (lane == 0) rec[wib][27] = static_cast<uint32_t>(P.kq_d[sb]);
+    __syncwarp();
+    const uint8_t* bytes = reinterpret_cast<const uint8_t*>(rec[wib]);
+    uint8_t* dst = P.out + sb * kKqRecord;
+    for (int b = lane; b < kKqRecord; b += 32) dst[b] = bytes[b];
+    __syncwarp();
+  }
+}
+
+template <int K>
+void set_max_smem_carveout() {
+  cudaFuncSetAttribute(k_forward<K>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_backward<K, false>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_backward<K, true>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+}
+
+int grid_for(const void* fn, int num_sms, int threads) {
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, threads, 0) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  return per_sm * num_sms;
+}
+
+}  // namespace
+
+#define GSQ_DISPATCH_K(K_, EXPR)                    \
+  switch (K_) {                                     \
+    case 2: { constexpr int KK = 2; EXPR; } break;  \
+    case 3: { constexpr int KK = 3; EXPR; } break;  \
+    case 4: { constexpr int KK = 4; EXPR; } break;  \
+    case 5: { constexpr int KK = 5; EXPR; } break;  \
+    case 6: { constexpr int KK = 6; EXPR; } break;  \
+    case 7: { constexpr int KK = 7; EXPR; } break;  \
+    case 8: { constexpr int KK = 8; EXPR; } break;  \
+    default: return cudaErrorInvalidValue;          \
+  }
+
+int ew_grid_size(int K, int which, int num_sms) {
+  int g = num_sms;
+  auto pick = [&](auto kk) {
+    constexpr int KK = decltype(kk)::value;
+    set_max_smem_carveout<KK>();
+    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<KK>), num_sms, kEwThreads)
+                   : grid_for(reinterpret_cast<const void*>(k_backward<KK, false>), num_sms, kEwThreads);
+  };
+  switch (K) {
+    case 2: pick(std::integral_constant<int, 2>{}); break;
+    case 3: pick(std::integral_constant<int, 3>{}); break;
+    case 4: pick(std::integral_constant<int, 4>{}); break;
+    case 5: pick(std::integral_constant<int, 5>{}); break;
+    case 6: pick(std::integral_constant<int, 6>{}); break;
+    case 7: pick(std::integral_constant<int, 7>{}); break;
+    case 8: pick(std::integral_constant<int, 8>{}); break;
+    default: break;
+  }
+  return g;
+}
+
+cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s) {
+  GSQ_DISPATCH_K(p.K, (k_forward<KK><<<grid, kEwThreads, 0, s>>>(p)));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
+  const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
+  if (export_mode) {
+    GSQ_DISPATCH_K(p.K, (k_backward<KK, true><<<grid, kEwThreads, 0, s>>>(p)));
+  } else {
+    GSQ_DISPATCH_K(p.K, (k_backward<KK, false><<<grid, kEwThreads, 0, s>>>(p)));
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s) {
+  if (p.kquant) {
+    const int64_t nsb = p.n / kSuperBlock;
+    const int64_t blocks = (nsb + (kEwThreads / 32) - 1) / (kEwThreads / 32);
+    const int grid = static_cast<int>(blocks < 16LL * num_sms ? blocks : 16LL * num_sms);
+    k_init_kquant<<<grid > 0 ? grid : 1, kEwThreads, 0, s>>>(p);
+  } else {
+    const int64_t blocks = ((p.n >> 2) + kEwThreads - 1) / kEwThreads;
+    const int grid = static_cast<int>(blocks < 16LL * num_sms ? blocks : 16LL * num_sms);
+    k_init_group<<<grid > 0 ? grid : 1, kEwThreads, 0, s>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16, unsigned int* counter,
+                                  cudaStream_t s) {
+  if (count <= 0) return cudaSuccess;
+  const int64_t blocks = (count + 255) / 256;
+  const int grid = static_cast<int>(blocks < 4096 ? blocks : 4096);
+  k_nonfinite<<<grid, 256, 0, s>>>(x, count, is_bf16, counter);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_project(const ProjectParams& p, int num_sms, cudaStream_t s) {
+  const int64_t blocks = ((p.n >> 2) + kEwThreads - 1) / kEwThreads;
+  const int grid = static_cast<int>(blocks < 8LL * num_sms ? blocks : 8LL * num_sms);
+  k_project<<<grid > 0 ? grid : 1, kEwThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack(const PackParams& p, int num_sms, cudaStream_t s) {
+  const int grid = 8 * num_sms;
+  if (p.kquant)
+    k_pack_kquant<<<grid, kEwThreads, 0, s>>>(p);
+  else
+    k_pack_group<<<grid, kEwThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace gsq

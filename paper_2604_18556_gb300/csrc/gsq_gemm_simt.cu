@@ -1,0 +1,122 @@
+// CUDA-core GEMM for the fp32 validation path of the loss contraction
+// (G = 2 D H_sym, Eq. 1 with a linear layer) and for forming H = X^T X from
+// calibration tokens at init; plus the symmetrisation / precision conversion of
+// H.  Not the performance path: the bf16 contraction runs on the tensor cores.
+#include <cuda_bf16.h>
+
+#include "gsq_internal.h"
+
+namespace gsq {
+namespace {
+
+constexpr int BM = 64, BN = 64, BK = 16, TM = 4, TN = 4;
+
+template <bool kBf16>
+__device__ __forceinline__ float ld_in(const void* p, int64_t idx) {
+  if (kBf16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[idx]);
+  return reinterpret_cast<const float*>(p)[idx];
+}
+
+// C[b][m][n] = alpha * sum_k A[b][m*sam + k*sak] * B[b][k*sbk + n*sbn], fp32 accumulate.
+template <bool kBf16>
+__global__ void __launch_bounds__(256) k_simt_gemm(const SimtGemm g) {
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int b = blockIdx.z;
+  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  const int tid = threadIdx.x;
+  const int tx = tid % (BN / TN), ty = tid / (BN / TN);
+  const char* Ab = reinterpret_cast<const char*>(g.A) + b * g.sab * (kBf16 ? 2 : 4);
+  const char* Bb = reinterpret_cast<const char*>(g.B) + b * g.sbb * (kBf16 ? 2 : 4);
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.0f;
+  for (int k0 = 0; k0 < g.Kd; k0 += BK) {
+    for (int e = tid; e < BM * BK; e += 256) {
+      const int mm = e / BK, kk = e % BK;
+      const int gm = m0 + mm, gk = k0 + kk;
+      As[kk][mm] = (gm < g.M && gk < g.Kd) ? ld_in<kBf16>(Ab, gm * g.sam + gk * g.sak) : 0.0f;
+    }
+    for (int e = tid; e < BN * BK; e += 256) {
+      const int kk = e / BN, nn = e % BN;
+      const int gk = k0 + kk, gn = n0 + nn;
+      Bs[kk][nn] = (gk < g.Kd && gn < g.N) ? ld_in<kBf16>(Bb, gk * g.sbk + gn * g.sbn) : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float a[TM], bb[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty * TM + i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) bb[j] = Bs[kk][tx * TN + j];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], bb[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  float* Cb = g.C + b * g.scb;
+#pragma unroll
+  for (int i = 0; i < TM; ++i) {
+    const int gm = m0 + ty * TM + i;
+    if (gm >= g.M) continue;
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int gn = n0 + tx * TN + j;
+      if (gn < g.N) Cb[static_cast<int64_t>(gm) * g.ldc + gn] = g.alpha * acc[i][j];
+    }
+  }
+}
+
+// out[e] = (H[e] + H[e]^T) / 2 in bf16 or fp32, through a 32x32 shared tile.
+template <bool kBf16Out>
+__global__ void k_symmetrize(const float* H, void* out, int C) {
+  __shared__ float t[32][33];
+  const int e = blockIdx.z;
+  const int64_t base = static_cast<int64_t>(e) * C * C;
+  const int i0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  for (int r = ty; r < 32; r += 8) {
+    const int i = j0 + r, j = i0 + tx;  // transposed tile: H[j0 + r][i0 + tx]
+    t[r][tx] = (i < C && j < C) ? H[base + static_cast<int64_t>(i) * C + j] : 0.0f;
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int i = i0 + r, j = j0 + tx;
+    if (i < C && j < C) {
+      const float v = (H[base + static_cast<int64_t>(i) * C + j] + t[tx][r]) * 0.5f;
+      if (kBf16Out)
+        reinterpret_cast<__nv_bfloat16*>(out)[base + static_cast<int64_t>(i) * C + j] =
+            __float2bfloat16_rn(v);
+      else
+        reinterpret_cast<float*>(out)[base + static_cast<int64_t>(i) * C + j] = v;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_simt_gemm(const SimtGemm& g, cudaStream_t s) {
+  dim3 grid((g.N + BN - 1) / BN, (g.M + BM - 1) / BM, g.batch);
+  if (g.bf16_inputs)
+    k_simt_gemm<true><<<grid, 256, 0, s>>>(g);
+  else
+    k_simt_gemm<false><<<grid, 256, 0, s>>>(g);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_bf16, cudaStream_t s) {
+  dim3 grid((C + 31) / 32, (C + 31) / 32, E);
+  dim3 block(32, 8);
+  if (out_bf16)
+    k_symmetrize<true><<<grid, block, 0, s>>>(H, out, C);
+  else
+    k_symmetrize<false><<<grid, block, 0, s>>>(H, out, C);
+  return cudaGetLastError();
+}
+
+}  // namespace gsq

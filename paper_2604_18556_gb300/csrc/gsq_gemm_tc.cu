@@ -1,0 +1,399 @@
+// Loss contraction on the 5th-generation tensor cores (sm_103a):
+//   G[e] = alpha * D[e] H[e]^T   (bf16 operands, fp32 accumulation in TMEM)
+// D[e] is R x C row-major, H[e] is C x C row-major and symmetric, so both are
+// "K-major" operands (the contraction index is contiguous) and H^T = H gives
+// G = 2 D H_sym = dL/dW^ of L = tr(D H D^T) (Eq. 1 with a linear layer).
+//
+// Persistent, warp-specialised kernel, one CTA per SM:
+//   warp 0     TMA producer: 128x64 tile of D and 256x64 tile of H per stage,
+//              128-byte swizzle, into a 4-stage shared-memory ring;
+//   warp 1     TMEM allocator and MMA issuer: tcgen05.mma.cta_group::1.kind::f16
+//              M=128 N=256 K=16, four per 64-wide k-block, accumulating in TMEM;
+//              tcgen05.commit frees a stage / publishes a finished accumulator;
+//   warps 2-5  epilogue: tcgen05.ld 32x32b of the accumulator (each warp owns
+//              the 32 TMEM lanes of its quarter), scale by alpha, store fp32.
+// The accumulator is double-buffered in TMEM (2 x 256 columns) so the epilogue
+// of tile i overlaps the MMAs of tile i+1.  Every mbarrier wait is bounded
+// (2 s of %globaltimer); on expiry the CTA records an error code in the
+// workspace flags, waits (bounded) for its own in-flight copies, frees its TMEM
+// and returns.
+#include <cuda.h>
+
+#include "gsq_internal.h"
+
+namespace gsq {
+namespace {
+
+constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
+constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;
+constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;
+constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr int TC_THREADS = 192;
+constexpr int TC_TMEM_COLS = 2 * TC_BN;
+constexpr int TC_SMEM_BYTES = TC_STAGES * TC_STAGE_BYTES + 256 + 1024;
+// kind::f16 instruction descriptor: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1),
+// B bf16 (10-12 = 1), both K-major (bits 15, 16 = 0), N>>3 at 17-22, M>>4 at 24-28.
+constexpr uint32_t TC_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                              (static_cast<uint32_t>(TC_BN >> 3) << 17) |
+                              (static_cast<uint32_t>(TC_BM >> 4) << 24);
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+struct TcArgs {
+  int E, R, C;
+  float* G;
+  float alpha;
+  DevFlags* flags;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase of parity `parity`.  Returns false when the
+// time limit passes (and raises `abort`) or when another role raised it.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          bool honour_abort = true) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (honour_abort && *abort) return false;
+    if (global_ns() - t0 > kWaitLimitNs) {
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor, K-major operand with 128-byte swizzle:
+// start address >> 4 (bits 0-13), leading byte offset (unused for swizzled
+// K-major, set to 1), stride byte offset 1024 B >> 4 (bits 32-45) between
+// 8-row core-matrix groups, descriptor version 1 (bits 46-47), swizzle mode
+// 128B = 2 (bits 61-63).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(1) << 16) |
+         (static_cast<uint64_t>(1024 >> 4) << 32) | (static_cast<uint64_t>(1) << 46) |
+         (static_cast<uint64_t>(2) << 61);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t da, uint64_t db, uint32_t accum) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
+      "l"(da), "l"(db), "r"(TC_IDESC), "r"(accum));
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int Mt, int Nt, int& e, int& m, int& n) {
+  const int per_e = Mt * Nt;
+  e = tile / per_e;
+  const int r = tile - e * per_e;
+  n = r / Mt;  // m fastest: CTAs running together share the same H rows
+  m = r - n * Mt;
+}
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const TcArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES);
+  uint64_t* empty_bar = full_bar + TC_STAGES;
+  uint64_t* tfull_bar = empty_bar + TC_STAGES;
+  uint64_t* tempty_bar = tfull_bar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(full_bar + s, 1);
+      mbar_init(empty_bar + s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar + a, 1);
+      mbar_init(tempty_bar + a, 128);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TC_TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int Mt = (args.R + TC_BM - 1) / TC_BM;
+  const int Nt = (args.C + TC_BN - 1) / TC_BN;
+  const int KB = (args.C + TC_BK - 1) / TC_BK;
+  const int tiles = args.E * Mt * Nt;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_phase[TC_STAGES];
+      bool issued[TC_STAGES];
+      for (int s = 0; s < TC_STAGES; ++s) issued[s] = false;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
+        int e, m, n;
+        tile_coords(tile, Mt, Nt, e, m, n);
+        const int arow = e * args.R + m * TC_BM;
+        const int brow = e * args.C + n * TC_BN;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(empty_bar + stage, phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + stage * TC_STAGE_BYTES;
+          uint8_t* sb = sa + TC_A_BYTES;
+          mbar_expect_tx(full_bar + stage, TC_STAGE_BYTES);
+          tma_load_2d(sa, &tmA, full_bar + stage, kb * TC_BK, arow);
+          tma_load_2d(sb, &tmB, full_bar + stage, kb * TC_BK, brow);
+          issued[stage] = true;
+          issued_phase[stage] = phase;
+          if (++stage == TC_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // abort: wait (bounded, ignoring the abort flag) for our own copies in flight
+        for (int s = 0; s < TC_STAGES; ++s)
+          if (issued[s]) mbar_wait(full_bar + s, issued_phase[s], abort_flag, false);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
+        if (!mbar_wait(tempty_bar + acc, acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * TC_BN);
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(full_bar + stage, phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * TC_STAGE_BYTES);
+          const uint64_t da = sw128_desc(sa);
+          const uint64_t db = sw128_desc(sa + TC_A_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)  // advance 16 bf16 = 32 B = 2 units of 16 B
+            umma_bf16(d_tmem, da + 2 * k, db + 2 * k, (kb | k) != 0 ? 1u : 0u);
+          umma_commit(empty_bar + stage);
+          if (++stage == TC_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(tfull_bar + acc);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31 are this warp's
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+      if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
+      tc_fence_after();
+      int e, m, n;
+      tile_coords(tile, Mt, Nt, e, m, n);
+      const int row = m * TC_BM + quarter * 32 + lane;
+      const int col0 = n * TC_BN;
+      float* grow = args.G + (static_cast<int64_t>(e) * args.R + row) * args.C;
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * TC_BN) +
+                             (static_cast<uint32_t>(quarter * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < TC_BN; c += 16) {
+        float v[16];
+        tmem_ld16(taddr + c, v);
+        if (row < args.R) {
+#pragma unroll
+          for (int j = 0; j < 16; j += 4) {
+            const int col = col0 + c + j;
+            if (col < args.C)
+              *reinterpret_cast<float4*>(grow + col) =
+                  make_float4(args.alpha * v[j], args.alpha * v[j + 1], args.alpha * v[j + 2],
+                              args.alpha * v[j + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(tempty_bar + acc);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TC_TMEM_COLS));
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(&args.flags->error, 0x7C01u);
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                        uint32_t box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(TC_BK), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool tc_gemm_supported(int device) {
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return false;
+  return prop.major == 10 && prop.minor == 3 && get_encode_fn() != nullptr;
+}
+
+cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e =
+        cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  CUtensorMap ta, tb;
+  if (!encode_kmajor_bf16(&ta, g.D, static_cast<uint64_t>(g.C),
+                          static_cast<uint64_t>(g.E) * g.R, TC_BM) ||
+      !encode_kmajor_bf16(&tb, g.H, static_cast<uint64_t>(g.C),
+                          static_cast<uint64_t>(g.E) * g.C, TC_BN))
+    return cudaErrorInvalidValue;
+  TcArgs a;
+  a.E = g.E;
+  a.R = g.R;
+  a.C = g.C;
+  a.G = g.G;
+  a.alpha = g.alpha;
+  a.flags = g.flags;
+  const int Mt = (g.R + TC_BM - 1) / TC_BM, Nt = (g.C + TC_BN - 1) / TC_BN;
+  const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  k_tc_gemm<<<grid, TC_THREADS, TC_SMEM_BYTES, s>>>(ta, tb, a);
+  return cudaGetLastError();
+}
+
+}  // namespace gsq

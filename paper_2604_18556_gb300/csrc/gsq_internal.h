@@ -1,0 +1,146 @@
+// Internal declarations shared by the libgsq CUDA sources (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/gsq.h"
+
+namespace gsq {
+
+constexpr int kMaxLevels = GSQ_MAX_LEVELS;
+constexpr int kSubBlock = 16;     // K-Quant-like sub-block (6-bit sub-scale)
+constexpr int kSuperBlock = 256;  // K-Quant-like super-block (fp16 d)
+constexpr int kKqRecord = 110;    // bytes per packed super-block
+constexpr int kEwThreads = 256;   // threads per block of the elementwise kernels
+
+// Device-side status words, one 256-byte slot of the workspace.
+struct DevFlags {
+  unsigned int blocks_done;  // last-block-done counter of the loss reduction
+  unsigned int error;        // nonzero: a bounded wait gave up (code of the site)
+  unsigned int nonfinite;    // init scan: count of non-finite inputs
+  unsigned int pad[61];
+};
+
+// Everything the elementwise kernels need, passed by value.
+struct EwParams {
+  // shape
+  int64_t n;          // E*R*C weights
+  int64_t nq;         // n / 4 quads
+  int K;
+  int group;          // scale group (16 for K-Quant)
+  int log2_group;
+  int w_bf16;         // W storage: 1 bf16, 0 fp32
+  int d_bf16;         // D storage: 1 bf16, 0 fp32
+  float grid[kMaxLevels];
+  // state (device)
+  float* logits;      // [K][n]
+  float* m_logits;    // [K][n]
+  float* scales;      // [n/group]
+  float* m_scales;    // [n/group]
+  const void* W;      // [n]
+  void* D;            // [n]
+  const float* G;     // [n]
+  // noise
+  uint32_t key0, key1;
+  int noise;          // 0: g = 0
+  // step t (backward / forward)
+  uint32_t t;
+  float kappa, inv_tau, kappa_over_tau;
+  // look-ahead forward (t + 1)
+  int lookahead;
+  uint32_t t_next;
+  float kappa_next, inv_tau_next;
+  // Lion
+  float lr_l, lr_s, b1, b2, wd_l, wd_s;
+  int scales_frozen;
+  // outputs
+  float* grad_logits;  // export mode: [K][n]
+  float* grad_scales;  // export mode: [n/group]
+  float* what;         // forward: optional W^ export [n]
+  double* loss_partials;
+  DevFlags* flags;
+  float* loss_out;     // nullable
+};
+
+// ---- launchers (gsq_elementwise.cu) ----------------------------------------
+cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
+cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
+int ew_grid_size(int K, int which, int num_sms);  // which: 0 forward, 1 backward
+
+struct InitParams {
+  int64_t n;
+  int K;
+  int group;
+  int kquant;
+  int w_bf16;
+  float grid[kMaxLevels];
+  float init_bias;
+  const void* W;       // stored copy
+  float* logits;
+  float* m_logits;
+  float* scales;
+  float* m_scales;
+  uint16_t* kq_d;      // [n/256]
+  int8_t* kq_sc;       // [n/16]
+};
+cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s);
+cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16,
+                                  unsigned int* counter, cudaStream_t s);
+
+struct ProjectParams {
+  int64_t n;
+  int K;
+  const float* logits;
+  uint8_t* codes;
+  float* margin;
+};
+cudaError_t launch_project(const ProjectParams& p, int num_sms, cudaStream_t s);
+
+struct PackParams {
+  int64_t n;
+  int K;
+  int group;
+  int kquant;
+  const float* logits;
+  const float* scales;     // group mode
+  const uint16_t* kq_d;    // kquant
+  const int8_t* kq_sc;     // kquant
+  uint8_t* out;
+  int64_t code_bytes;      // group mode: size of the padded code section
+};
+cudaError_t launch_pack(const PackParams& p, int num_sms, cudaStream_t s);
+
+// ---- GEMMs (gsq_gemm_simt.cu, gsq_gemm_tc.cu) --------------------------------
+// C[b][m][n] = alpha * sum_k A[b][m*sam + k*sak] * B[b][k*sbk + n*sbn]
+struct SimtGemm {
+  int batch, M, N, Kd;
+  const void* A;
+  int64_t sam, sak, sab;
+  const void* B;
+  int64_t sbk, sbn, sbb;
+  float* C;
+  int64_t ldc, scb;
+  float alpha;
+  int bf16_inputs;  // 1: A and B are bf16, else fp32
+};
+cudaError_t launch_simt_gemm(const SimtGemm& g, cudaStream_t s);
+
+// H_out[e] = (H[e] + H[e]^T) / 2 converted to bf16 (out_bf16=1) or fp32.
+cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_bf16,
+                              cudaStream_t s);
+
+// tcgen05 / TMA bf16 GEMM: G[e] = alpha * D[e] (R x C, bf16, row-major) *
+// H[e]^T (C x C, bf16, row-major; symmetric so H^T = H), fp32 out.
+struct TcGemm {
+  int E, R, C;
+  const void* D;
+  const void* H;
+  float* G;
+  float alpha;
+  DevFlags* flags;
+};
+bool tc_gemm_supported(int device);
+cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
+
+}  // namespace gsq

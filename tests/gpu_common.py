@@ -1,0 +1,134 @@
+"""Helpers shared by the GPU parity tests: build a layer through the C ABI and the
+matching oracle problem from the same seeded inputs, read GPU state back into
+oracle form, and the tolerance checks the acceptance criteria name.
+
+Tolerances (from the acceptance criteria of the step):
+  * hard assignments and packed bits: bit-exact (entries whose top-two logit
+    margin is below 1e-5 excluded where the logits themselves came from two
+    trajectories);
+  * fp32 path (GEMM on fp32 operands): loss, gradients and W^ within 1e-4 relative;
+  * bf16 tensor-core GEMM path: GEMM-backed quantities within 2e-2 relative.
+"Relative" is applied elementwise as |a - b| <= tol * (|b| + rms(b)) -- the rms
+term keeps entries that are tiny by cancellation from failing on absolute
+noise -- and, for the whole tensor, ||a - b|| <= tol * ||b||.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import gsq_oracle as O
+from paper_2604_18556_gb300 import configs as C
+from paper_2604_18556_gb300 import inputs
+
+TOL_F32 = 1e-4
+TOL_BF16 = 2e-2
+
+
+def gsq():
+    from paper_2604_18556_gb300 import build
+    build.build()
+    from paper_2604_18556_gb300 import gsq as g
+    return g
+
+
+def assert_close(a, b, tol, what=""):
+    a = np.asarray(a, dtype=np.float64).reshape(-1)
+    b = np.asarray(b, dtype=np.float64).reshape(-1)
+    assert a.shape == b.shape, (what, a.shape, b.shape)
+    if b.size == 0:
+        return
+    rms = float(np.sqrt(np.mean(b * b)))
+    err = np.abs(a - b)
+    bad = err > tol * (np.abs(b) + rms)
+    if bad.any():
+        i = int(np.argmax(err / (np.abs(b) + rms + 1e-300)))
+        raise AssertionError(f"{what}: {int(bad.sum())}/{b.size} elements beyond {tol}; worst at {i}: "
+                             f"got {a[i]!r} want {b[i]!r} (rms {rms:.3e})")
+    nrm = float(np.linalg.norm(b))
+    assert float(np.linalg.norm(a - b)) <= tol * nrm + 1e-300, (what, float(np.linalg.norm(a - b)) / nrm)
+
+
+def rel_err(a, b) -> float:
+    a = np.asarray(a, dtype=np.float64).reshape(-1)
+    b = np.asarray(b, dtype=np.float64).reshape(-1)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+class Case:
+    """A layer problem on the GPU (through the C ABI) and the same problem for the oracle."""
+
+    def __init__(self, w: C.Workload, gemm: str = "f32", noise: bool = True, seed=None,
+                 keep_calib_host: bool = True, device="cuda"):
+        g = gsq()
+        self.w = w
+        self.gemm = gemm
+        self.W = inputs.make_weight(w, device=device)
+        if w.calib == "X":
+            self.calib = inputs.make_tokens(w, device=device)
+        else:
+            self.calib = inputs.make_gram(w, device=device)
+        hyper = dict(init_bias=w.init_bias, seed=w.seed if seed is None else seed,
+                     lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
+                     wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise)
+        self.layer = g.Layer(self.W, self.calib, w.grid, w.group, calib_kind=w.calib,
+                             scale_mode=w.scale_mode, gemm=gemm, **hyper)
+        self.prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float),
+                              group=w.group, seed=hyper["seed"], scale_mode=w.scale_mode,
+                              lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1,
+                              beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
+                              noise=noise)
+        if keep_calib_host:
+            host = self.calib.double().cpu().numpy()
+            if w.calib == "X":
+                self.prob.X = host
+            else:
+                self.prob.H = host
+        self.W_host = self.W.float().cpu().numpy().reshape(w.experts * w.rows, w.cols)
+
+    # ---- GPU state -> numpy ------------------------------------------------------
+    def tensor(self, which, dtype):
+        return self.layer.get_tensor(which, dtype)
+
+    def logits(self):
+        g = gsq()
+        E, R, Cc, K = self.w.experts, self.w.rows, self.w.cols, self.w.K
+        return self.tensor(g.GSQ_T_LOGITS, torch.float32).view(K, E * R, Cc).cpu().numpy()
+
+    def state(self, rows=None) -> O.RowState:
+        g = gsq()
+        w = self.w
+        nr = w.experts * w.rows
+        K = w.K
+        f = lambda which: self.tensor(which, torch.float32).cpu().numpy()
+        st = O.RowState(row_ids=np.arange(nr, dtype=np.int64), W=self.W_host.astype(np.float64),
+                        logits=f(g.GSQ_T_LOGITS).reshape(K, nr, w.cols),
+                        scales=f(g.GSQ_T_SCALES).reshape(nr, w.cols // w.group),
+                        m_logits=f(g.GSQ_T_MOM_LOGITS).reshape(K, nr, w.cols),
+                        m_scales=f(g.GSQ_T_MOM_SCALES).reshape(nr, w.cols // w.group))
+        if w.scale_mode == "kquant2":
+            d16 = self.tensor(g.GSQ_T_KQ_D, torch.int16).cpu().numpy().view(np.uint16)
+            st.kq_d = O.f16_bits_to_f32(d16).reshape(nr, w.cols // 256)
+            st.kq_sc = self.tensor(g.GSQ_T_KQ_SC, torch.int8).cpu().numpy().astype(np.int32).reshape(
+                nr, w.cols // 16)
+        return st if rows is None else st.subset(rows)
+
+    def G(self):
+        g = gsq()
+        return self.tensor(g.GSQ_T_G, torch.float32).view(-1, self.w.cols).cpu().numpy()
+
+    def D(self):
+        g = gsq()
+        dt = torch.bfloat16 if self.gemm == "bf16" else torch.float32
+        return self.tensor(g.GSQ_T_D, dt).float().view(-1, self.w.cols).cpu().numpy()
+
+    def H_operand(self):
+        g = gsq()
+        dt = torch.bfloat16 if self.gemm == "bf16" else torch.float32
+        C_ = self.w.cols
+        return self.tensor(g.GSQ_T_H, dt).float().view(self.w.experts, C_, C_).cpu().numpy()
+
+    def oracle_init(self, rows=None) -> O.RowState:
+        nr = self.w.experts * self.w.rows
+        ids = np.arange(nr) if rows is None else np.asarray(rows)
+        return O.init_state(self.prob, self.W_host[ids], ids, init_bias=self.w.init_bias)

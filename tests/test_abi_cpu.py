@@ -1,0 +1,177 @@
+"""C-ABI checks that need no GPU: the library loads and exports every function
+include/gsq.h declares; the ctypes descriptor matches the C layout (checked by
+compiling the header with gcc); host-side validation, workspace sizing and
+fault injection answer before any CUDA call."""
+import ctypes
+import os
+import re
+import subprocess
+import sys
+import textwrap
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "gsq.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    sys.path.insert(0, ROOT)
+    from paper_2604_18556_gb300 import build
+    build.build()
+    from paper_2604_18556_gb300 import gsq
+    return gsq
+
+
+def _declared():
+    src = open(HEADER).read()
+    return sorted(set(re.findall(r"GSQ_API\s+[\w\s\*]+?\b(gsq_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 16
+    out = subprocess.run(["nm", "-D", "--defined-only", lib.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {ln.split()[-1] for ln in out.splitlines() if ln.strip()}
+    assert set(names) <= exported
+    assert set(names) == set(lib.EXPORTED)
+    # the statically linked CUDA runtime stays private
+    assert not any(s.startswith("cuda") for s in exported)
+    cdll = ctypes.CDLL(lib.LIB_PATH)
+    for n in names:
+        assert getattr(cdll, n) is not None
+
+
+def test_descriptor_layout_matches_c(lib, tmp_path):
+    fields = [f for f, _ in lib.gsq_layer_desc._fields_]
+    prog = "#include <stdio.h>\n#include <stddef.h>\n#include \"gsq.h\"\nint main(void){\n"
+    prog += 'printf("size %zu\\n", sizeof(gsq_layer_desc));\n'
+    for f in fields:
+        prog += f'printf("{f} %zu\\n", offsetof(gsq_layer_desc, {f}));\n'
+    prog += 'printf("profile %zu\\n", sizeof(gsq_profile));\nreturn 0;}\n'
+    c = tmp_path / "layout.c"
+    c.write_text(prog)
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = dict(ln.split() for ln in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                   check=True).stdout.splitlines())
+    assert int(out["size"]) == ctypes.sizeof(lib.gsq_layer_desc)
+    assert int(out["profile"]) == ctypes.sizeof(lib.gsq_profile)
+    for f in fields:
+        assert int(out[f]) == getattr(lib.gsq_layer_desc, f).offset, f
+
+
+def _desc(lib, **kw):
+    base = dict(experts=1, rows=64, cols=256, grid=(-1.5, -0.5, 0.5, 1.5), group_size=128)
+    base.update(kw)
+    return lib.make_desc(**base)
+
+
+def _align(x):
+    return (x + 255) // 256 * 256
+
+
+def test_workspace_size_formula(lib):
+    from paper_2604_18556_gb300.configs import WORKLOADS
+    for w in WORKLOADS.values():
+        d = lib.make_desc(experts=w.experts, rows=w.rows, cols=w.cols, grid=w.grid,
+                          group_size=w.group, w_dtype=lib.GSQ_DTYPE_F32 if w.w_dtype == "f32" else lib.GSQ_DTYPE_BF16,
+                          calib_kind=lib.GSQ_CALIB_X if w.calib == "X" else lib.GSQ_CALIB_H,
+                          n_tokens=w.tokens if w.calib == "X" else 0,
+                          scale_mode=lib.GSQ_SCALE_KQUANT2 if w.scale_mode == "kquant2" else lib.GSQ_SCALE_GROUP,
+                          lr_scales=w.lr_scales)
+        n, K = w.n, w.K
+        expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * K * n) + 2 * _align(4 * n // w.group)
+        expect += _align(n * w.w_bytes()) + _align(w.experts * w.cols ** 2 * 2) + _align(2 * n) + _align(4 * n)
+        if w.scale_mode == "kquant2":
+            expect += _align(2 * n // 256) + _align(n // 16)
+        if w.calib == "X":
+            expect += _align(4 * w.experts * w.cols ** 2)
+        assert lib.gsq_workspace_size(d) == expect, w.name
+    # the largest workload fits comfortably in one GB300's HBM
+    big = WORKLOADS["moe64_kquant3"]
+    d = lib.make_desc(experts=big.experts, rows=big.rows, cols=big.cols, grid=big.grid, group_size=16,
+                      scale_mode=lib.GSQ_SCALE_KQUANT2, lr_scales=0.0)
+    assert lib.gsq_workspace_size(d) < 100e9
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(cols=260), 2),                         # C % 8
+    (dict(cols=192, group_size=128), 2),         # C % G
+    (dict(group_size=96), 2),                    # not a power of two
+    (dict(group_size=256), 2),
+    (dict(grid=(0.5, -0.5)), 1),                 # not ascending
+    (dict(grid=(1.0,)), 1),                      # K < 2
+    (dict(grid=tuple(range(9))), 1),             # K > 8
+    (dict(grid=(0.0, 0.0 + 1e-30)), 1),          # no level of usable magnitude? ascending but tiny ok
+    (dict(rows=0), 2),
+    (dict(scale_mode=1, group_size=16), 1),      # KQUANT2 needs frozen scales
+    (dict(scale_mode=1, group_size=16, lr_scales=0.0, cols=128), 2),   # C % 256
+    (dict(w_dtype=7), 1),
+    (dict(calib_kind=1, n_tokens=0), 1),
+    (dict(gemm=5), 1),
+    (dict(beta1=1.5), 1),
+])
+def test_descriptor_validation(lib, kw, status):
+    d = _desc(lib, **kw)
+    if kw.get("grid") == (0.0, 1e-30):
+        # ascending, finite, nonzero max level: valid
+        assert lib.gsq_workspace_size(d) > 0
+        return
+    with pytest.raises(lib.GsqError) as ei:
+        lib.gsq_workspace_size(d)
+    assert ei.value.status == status
+    assert lib.gsq_last_error()
+
+
+def test_init_rejects_bad_buffers_before_cuda(lib):
+    d = _desc(lib)
+    nbytes = lib.gsq_workspace_size(d)
+    with pytest.raises(lib.GsqError) as ei:      # W / calib missing
+        lib.gsq_init_layer(d, 256, nbytes, 0)
+    assert ei.value.status == lib.GSQ_ERR_INVALID_ARG
+    d.W, d.calib = 4096, 8192
+    with pytest.raises(lib.GsqError) as ei:      # workspace NULL
+        lib.gsq_init_layer(d, 0, nbytes, 0)
+    assert ei.value.status == lib.GSQ_ERR_WORKSPACE
+    with pytest.raises(lib.GsqError) as ei:      # misaligned
+        lib.gsq_init_layer(d, 256 + 16, nbytes, 0)
+    assert ei.value.status == lib.GSQ_ERR_WORKSPACE
+    with pytest.raises(lib.GsqError) as ei:      # too small
+        lib.gsq_init_layer(d, 256, nbytes - 1, 0)
+    assert ei.value.status == lib.GSQ_ERR_WORKSPACE and "too small" in lib.gsq_last_error()
+
+
+def test_handle_checks(lib):
+    for fn, args in [(lib._lib.gsq_step, (None, 0, 1.0, 1.0, 0.0, 1.0, None, None, None, None)),
+                     (lib._lib.gsq_step, (12345678, 0, 1.0, 1.0, 0.0, 1.0, None, None, None, None)),
+                     (lib._lib.gsq_project, (None, None, None, None)),
+                     (lib._lib.gsq_destroy, (None,)),
+                     (lib._lib.gsq_destroy, (987654321,)),
+                     (lib._lib.gsq_sync_status, (None, None))]:
+        assert fn(*args) == lib.GSQ_ERR_INVALID_ARG
+    assert lib.gsq_version().count(".") == 2
+
+
+def test_fault_injection_env(tmp_path):
+    code = textwrap.dedent(f"""
+        import sys; sys.path.insert(0, {ROOT!r})
+        from paper_2604_18556_gb300 import gsq
+        d = gsq.make_desc(experts=1, rows=8, cols=128, grid=(-1.0, 0.0, 1.0), group_size=128)
+        out = []
+        for i in range(4):
+            try:
+                gsq.gsq_workspace_size(d); out.append(0)
+            except gsq.GsqError as e:
+                out.append(e.status)
+        print(out)
+    """)
+    env = dict(os.environ, GSQ_FAULT_INJECT="gsq_workspace_size:3")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, check=True)
+    assert r.stdout.strip() == "[0, 0, 8, 0]"
+    env["GSQ_FAULT_INJECT"] = "gsq_init_layer:1"
+    code2 = code.replace("gsq.gsq_workspace_size(d)", "gsq.gsq_init_layer(d, 256, 1 << 30, 0)")
+    r = subprocess.run([sys.executable, "-c", code2], capture_output=True, text=True, env=env, check=True)
+    assert r.stdout.strip() == "[8, 1, 1, 1]"   # injected first, then argument errors

@@ -267,6 +267,8 @@ EwParams base_params(gsq_layer* L) {
   p.b2 = d.beta2;
   p.wd_l = d.wd_logits;
   p.wd_s = d.wd_scales;
+  p.lrwd_l = static_cast<float>(static_cast<double>(d.lr_logits) * d.wd_logits);
+  p.lrwd_s = static_cast<float>(static_cast<double>(d.lr_scales) * d.wd_scales);
   p.scales_frozen = (d.lr_scales == 0.f && d.wd_scales == 0.f) ? 1 : 0;
   p.loss_partials = reinterpret_cast<double*>(L->ws + L->lay.partials);
   p.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);

@@ -286,8 +286,6 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   const float scale_log2 = P.inv_tau * 1.4426950408889634f;
   const float scale_log2_next = P.inv_tau_next * 1.4426950408889634f;
-  const float decay_l = 1.0f - P.lr_l * P.wd_l;
-  const float decay_s = 1.0f - P.lr_s * P.wd_s;
   float loss_acc = 0.0f;
 
   for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
@@ -346,10 +344,10 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
         if (kExport) {
           m[k][j] = dl;
         } else {
-          // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l (1 - lr wd) - lr sign(c);
-          // m <- b2 m + (1-b2) g
+          // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l - lr wd l - lr sign(c);
+          // m <- b2 m + (1-b2) g.  The decay is one fma on l (no rounded 1 - lr wd).
           const float c = fmaf(P.b1, m[k][j], (1.0f - P.b1) * dl);
-          l[k][j] = fmaf(l[k][j], decay_l, -P.lr_l * sign_of(c));
+          l[k][j] = fmaf(-P.lrwd_l, l[k][j], l[k][j]) - P.lr_l * sign_of(c);
           m[k][j] = fmaf(P.b2, m[k][j], (1.0f - P.b2) * dl);
         }
       }
@@ -371,7 +369,7 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
 
     if (!P.scales_frozen) {
       const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
-      s = fmaf(s, decay_s, -P.lr_s * sign_of(c));
+      s = fmaf(-P.lrwd_s, s, s) - P.lr_s * sign_of(c);
       ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
     }
     if (active) {

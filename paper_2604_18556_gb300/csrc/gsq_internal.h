@@ -53,6 +53,7 @@ struct EwParams {
   float kappa_next, inv_tau_next;
   // Lion
   float lr_l, lr_s, b1, b2, wd_l, wd_s;
+  float lrwd_l, lrwd_s;  // lr * wd, rounded once from double
   int scales_frozen;
   // outputs
   float* grad_logits;  // export mode: [K][n]

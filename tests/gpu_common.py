@@ -49,6 +49,25 @@ def assert_close(a, b, tol, what=""):
     assert float(np.linalg.norm(a - b)) <= tol * nrm + 1e-300, (what, float(np.linalg.norm(a - b)) / nrm)
 
 
+def assert_gemm_bound(G, D, H, what="", alpha=2.0):
+    """fp32-accumulated G = alpha D H against exact products of the same operands:
+    every entry within the summation error bound |g^ - g| <= gamma_n sum_k |d_k h_k|
+    with gamma_n ~ n u, u = 2^-24 (Higham, Accuracy and Stability of Numerical
+    Algorithms, Thm 3.5; holds for any summation order), and the whole tensor
+    within 1e-5 in the Frobenius norm."""
+    D = np.asarray(D, np.float64)
+    H = np.asarray(H, np.float64)
+    exact = alpha * D @ H
+    absum = abs(alpha) * np.abs(D) @ np.abs(H)
+    n = D.shape[-1]
+    bound = 1.01 * n * 2.0 ** -24 * absum + 1e-30
+    err = np.abs(np.asarray(G, np.float64) - exact)
+    worst = float((err / bound).max())
+    assert worst <= 1.0, (what, worst)
+    assert float(np.linalg.norm(err)) <= 1e-5 * float(np.linalg.norm(exact)) + 1e-30, what
+    return worst
+
+
 def rel_err(a, b) -> float:
     a = np.asarray(a, dtype=np.float64).reshape(-1)
     b = np.asarray(b, dtype=np.float64).reshape(-1)

@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_common import TOL_BF16, TOL_F32, Case, assert_close, gsq, rel_err
+from gpu_common import TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound, gsq
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -72,30 +72,45 @@ def test_step_loss_and_gradients(name, gemm):
         assert_close(gs.cpu().numpy(), ref.d_scales, tol, "dL/dscales")
     if gemm == "bf16":
         # the tensor-core GEMM against exact products of its own bf16 operands
-        D, H = case.D(), case.H_operand()
+        D, H, G = case.D(), case.H_operand(), case.G()
         rows = np.arange(w.experts * w.rows)
-        Gx = np.empty_like(D, dtype=np.float64)
         for e in range(w.experts):
             sel = rows // w.rows == e
-            Gx[sel] = 2.0 * D[sel].astype(np.float64) @ H[e].astype(np.float64)
-        assert_close(case.G(), Gx, 1e-5, "tcgen05 GEMM vs its operands")
+            assert_gemm_bound(G[sel], D[sel], H[e], f"tcgen05 GEMM vs its operands, expert {e}")
         assert_close(loss.cpu().numpy(), [0.5 * np.sum(D * case.G())], 1e-5, "loss = 1/2 sum D*G")
 
 
-def _check_lion(gpu, orc, c_orc, lr, flip_frac, what):
+def _check_lion(gpu, orc, theta_in, c_orc, lr, flip_frac, what):
     """Lion results agree to rounding except where the sign of the momentum mix
     c is decided by a difference below the path's tolerance; such flips move a
     parameter by at most 2 lr."""
     gpu = np.asarray(gpu, np.float64).reshape(-1)
     orc = np.asarray(orc, np.float64).reshape(-1)
+    theta_in = np.asarray(theta_in, np.float64).reshape(-1)
     c = np.abs(np.asarray(c_orc, np.float64).reshape(-1))
     diff = np.abs(gpu - orc)
-    same = diff <= 4 * np.spacing(np.abs(orc).astype(np.float32)).astype(np.float64) + 1e-12
+    # rounding is relative to the operands (theta, lr), not to a result that may
+    # cancel to ~0 (theta = lr, sign(c) = +1)
+    mag = np.maximum(np.maximum(np.abs(orc), np.abs(theta_in)), lr)
+    same = diff <= 4 * np.spacing(mag.astype(np.float32)).astype(np.float64)
     flip = ~same
     assert np.all(diff[flip] <= 2.0 * lr * 1.001 + 1e-7), what
     thresh = flip_frac * np.sqrt(np.mean(c * c))
     assert np.all(c[flip] <= thresh), (what, int(flip.sum()), float(c[flip].max()), thresh)
     return int(flip.sum())
+
+
+def _check_momentum(gpu, orc, grad, b2, tol, what):
+    """m' = b2 m + (1 - b2) g with the same m on both sides: the difference is
+    (1 - b2) times the gradient difference, so the gradient's tolerance carries
+    over (|dg| <= tol (|g| + rms g)), plus fp32 rounding of m'."""
+    gpu = np.asarray(gpu, np.float64).reshape(-1)
+    orc = np.asarray(orc, np.float64).reshape(-1)
+    g = np.asarray(grad, np.float64).reshape(-1)
+    bound = (1 - b2) * tol * (np.abs(g) + np.sqrt(np.mean(g * g))) + \
+        2 * np.spacing(np.abs(orc).astype(np.float32)).astype(np.float64)
+    bad = np.abs(gpu - orc) > bound
+    assert not bad.any(), (what, int(bad.sum()))
 
 
 @pytest.mark.parametrize("gemm", ["f32", "bf16"])
@@ -119,12 +134,14 @@ def test_step_update(name, gemm):
         assert_close(loss.cpu().numpy(), [res.loss], tol, f"loss t={t}")
         m0 = st_gpu_before.m_logits.astype(np.float64)
         c_l = w.beta1 * m0 + (1 - w.beta1) * res.d_logits
-        _check_lion(gpu.logits, st_sync.logits, c_l, w.lr_logits, 2 * tol, "logits")
-        assert_close(gpu.m_logits, st_sync.m_logits, tol, "logit momentum")
+        _check_lion(gpu.logits, st_sync.logits, st_gpu_before.logits, c_l, w.lr_logits, 2 * tol,
+                    "logits")
+        _check_momentum(gpu.m_logits, st_sync.m_logits, res.d_logits, w.beta2, tol, "logit momentum")
         if res.d_scales is not None:
             c_s = w.beta1 * st_gpu_before.m_scales.astype(np.float64) + (1 - w.beta1) * res.d_scales
-            _check_lion(gpu.scales, st_sync.scales, c_s, w.lr_scales, 2 * tol, "scales")
-            assert_close(gpu.m_scales, st_sync.m_scales, tol, "scale momentum")
+            _check_lion(gpu.scales, st_sync.scales, st_gpu_before.scales, c_s, w.lr_scales,
+                        2 * tol, "scales")
+            _check_momentum(gpu.m_scales, st_sync.m_scales, res.d_scales, w.beta2, tol, "scale momentum")
         else:
             assert np.array_equal(gpu.scales, st_gpu_before.scales)
         losses.append(float(loss.item()))
@@ -220,8 +237,12 @@ def test_trajectory_ternary_full_run():
         assert_close(loss.cpu().numpy(), [res.loss], TOL_F32, f"loss t={t}")
     gpu = case.state()
     diff = np.abs(gpu.logits.astype(np.float64) - st.logits)
-    flips = int((diff > 1e-6).sum())
+    # a Lion sign flip moves a logit by 2 lr; fp32 rounding drift over 50 steps
+    # stays orders of magnitude below lr / 2
+    flips = int((diff > 0.5 * w.lr_logits).sum())
     assert flips <= 1e-4 * diff.size, flips
+    drift = diff[diff <= 0.5 * w.lr_logits]
+    assert drift.max() <= 1e-5, drift.max()
     assert diff.max() <= 2 * w.lr_logits * w.steps
     oc, om = O.project(st.logits)
     gc, _ = O.project(gpu.logits)

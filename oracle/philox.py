@@ -14,7 +14,7 @@ Stream layout (a reading; the paper is silent):
   counter = (lo32(i), hi32(i), t, k div 4), key = (lo32(seed), hi32(seed)),
   where i = (e*R + r)*C + c is the flat weight index, t the step index and k the
   grid level; level k takes 32-bit word (k mod 4) of that block.
-  u = (floor(x / 2^9) + 1/2) * 2^-23   (exactly representable in fp32, in (0,1))
+  u = ((x mod 2^23) + 1/2) * 2^-23     (low 23 bits; exactly representable in fp32, in (0,1))
   g = -ln(-ln(u))                       (inverse-CDF of Gumbel(0, 1)), in fp64.
 """
 from __future__ import annotations
@@ -49,8 +49,8 @@ def philox4x32_10(c0, c1, c2, c3, k0: int, k1: int):
 
 
 def uniform_from_word(x) -> np.ndarray:
-    """u = (floor(x / 2^9) + 1/2) * 2^-23, in float64 (exact)."""
-    j = (np.asarray(x, dtype=np.uint64) >> np.uint64(9)).astype(np.float64)
+    """u = ((x mod 2^23) + 1/2) * 2^-23, in float64 (exact)."""
+    j = (np.asarray(x, dtype=np.uint64) & np.uint64(0x7FFFFF)).astype(np.float64)
     return (j + 0.5) * 2.0 ** -23
 
 

@@ -24,6 +24,7 @@ namespace {
 constexpr uint64_t kMagic = 0x6773715f6c617972ull;  // "gsq_layr"
 constexpr int kMaxPartials = 16384;
 constexpr int kMaxProfileEvents = 8192;
+constexpr double kLog2e = 1.4426950408889634;
 
 thread_local std::string g_last_error;
 
@@ -306,7 +307,7 @@ gsq_status launch_fwd(gsq_layer* L, uint64_t step, float tau, float kappa, float
                       cudaStream_t s) {
   EwParams p = base_params(L);
   p.t = static_cast<uint32_t>(step);
-  p.kappa = kappa;
+  p.kappa_log2 = static_cast<float>(kappa * kLog2e);
   p.inv_tau = static_cast<float>(1.0 / tau);
   p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
   p.what = what;
@@ -575,13 +576,13 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
 
   EwParams p = base_params(L);
   p.t = static_cast<uint32_t>(step);
-  p.kappa = kappa;
+  p.kappa_log2 = static_cast<float>(kappa * kLog2e);
   p.inv_tau = static_cast<float>(1.0 / tau);
   p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
   p.lookahead = lookahead ? 1 : 0;
   if (lookahead) {
     p.t_next = static_cast<uint32_t>(step + 1);
-    p.kappa_next = next_kappa;
+    p.kappa_log2_next = static_cast<float>(next_kappa * kLog2e);
     p.inv_tau_next = static_cast<float>(1.0 / next_tau);
   }
   p.grad_logits = grad_logits_dev;

@@ -25,20 +25,34 @@ namespace {
 // S-box multipliers 0xD2511F53 / 0xCD9E8D57, Weyl key increments 0x9E3779B9 /
 // 0xBB67AE85.  Counter (lo32(i), hi32(i), t, level block), key = seed.
 // ---------------------------------------------------------------------------
+// Round keys of the Weyl schedule, computed once per thread from the seed (the
+// same for every thread, so they live in uniform registers).
+struct PhiloxKeys {
+  uint32_t k0[10], k1[10];
+};
+
+__device__ __forceinline__ PhiloxKeys philox_keys(uint32_t key0, uint32_t key1) {
+  PhiloxKeys k;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    k.k0[r] = key0 + static_cast<uint32_t>(r) * 0x9E3779B9u;
+    k.k1[r] = key1 + static_cast<uint32_t>(r) * 0xBB67AE85u;
+  }
+  return k;
+}
+
 __device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
-                                               uint32_t k0, uint32_t k1) {
+                                               const PhiloxKeys& k) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
     const uint32_t lo0 = 0xD2511F53u * c0;
     const uint32_t hi0 = __umulhi(0xD2511F53u, c0);
     const uint32_t lo1 = 0xCD9E8D57u * c2;
     const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2);
-    c0 = hi1 ^ c1 ^ k0;
+    c0 = hi1 ^ c1 ^ k.k0[r];
     c1 = lo1;
-    c2 = hi0 ^ c3 ^ k1;
+    c2 = hi0 ^ c3 ^ k.k1[r];
     c3 = lo0;
-    k0 += 0x9E3779B9u;
-    k1 += 0xBB67AE85u;
   }
   return make_uint4(c0, c1, c2, c3);
 }
@@ -55,60 +69,64 @@ __device__ __forceinline__ float fast_log2(float x) {
   return y;
 }
 
-// -ln(u) for u in [2^-24, 1 - 2^-24], accurate to a few ulp in relative terms
-// even as u -> 1 (where -ln u -> 0).  Argument reduction u = 2^e m with m in
-// [sqrt(1/2), sqrt(2)), then ln m = 2 atanh(y), y = (m - 1)/(m + 1), by its
-// odd power series 2(y + y^3/3 + y^5/5 + ...) (Abramowitz & Stegun 4.1.27);
-// |y| <= 0.1716, so terms through y^9 leave a relative remainder below 2e-9.
-__device__ __forceinline__ float neg_log_unit(float u) {
-  const uint32_t b = __float_as_uint(u);
-  int e = static_cast<int>(b >> 23) - 127;
-  float m = __uint_as_float((b & 0x007FFFFFu) | 0x3F800000u);  // [1, 2)
-  if (m > 1.41421356f) {
-    m *= 0.5f;
-    e += 1;
-  }
+// -log2(u) for u in [2^-24, 1 - 2^-24], accurate to a few ulp in relative terms
+// even as u -> 1 (where -log2 u -> 0).  Branch-free range reduction u = 2^e m
+// with m in [sqrt(1/2), sqrt(2)): subtracting the bit pattern of sqrt(1/2) from
+// the bits of u moves the exponent boundary to sqrt(2) (the integer-offset
+// reduction of fdlibm-style logf).  Then log2 m = (2 / ln 2) atanh(y),
+// y = (m - 1)/(m + 1), by the odd series 2(y + y^3/3 + y^5/5 + ...)
+// (Abramowitz & Stegun 4.1.27); |y| <= 0.1716, so terms through y^9 leave a
+// relative remainder below 2e-9.
+__device__ __forceinline__ float neg_log2_unit(float u) {
+  const uint32_t bu = __float_as_uint(u);
+  const int e = static_cast<int>(bu - 0x3F3504F3u) >> 23;
+  const float m = __uint_as_float(bu - (static_cast<uint32_t>(e) << 23));  // 2^-e u
   const float y = __fdividef(m - 1.0f, m + 1.0f);
   const float y2 = y * y;
-  const float poly =
-      fmaf(y2, fmaf(y2, fmaf(y2, fmaf(y2, 1.0f / 9.0f, 1.0f / 7.0f), 1.0f / 5.0f), 1.0f / 3.0f),
-           1.0f);
-  const float ln_m = 2.0f * y * poly;
-  return -fmaf(static_cast<float>(e), 0.69314718055994531f, ln_m);
+  constexpr float c1 = 2.8853900817779268f;   // 2 / ln 2
+  constexpr float c3 = c1 / 3.0f, c5 = c1 / 5.0f, c7 = c1 / 7.0f, c9 = c1 / 9.0f;
+  const float poly = fmaf(y2, fmaf(y2, fmaf(y2, fmaf(y2, c9, c7), c5), c3), c1);
+  return -fmaf(y, poly, static_cast<float>(e));
 }
 
-// g = -ln(-ln u), u = (floor(x / 2^9) + 1/2) 2^-23 built exactly from the bits.
-__device__ __forceinline__ float gumbel_from_word(uint32_t x) {
-  const float one_plus = __uint_as_float(0x3F800000u | (x >> 9));  // 1 + j 2^-23
-  const float u = one_plus - __uint_as_float(0x3F7FFFFFu);         // (j + 1/2) 2^-23, exact
-  const float E = neg_log_unit(u);
-  return -0.69314718055994531f * fast_log2(E);
+// The Gumbel draw in log2 units, up to a constant common to every level:
+//   g = -ln(-ln u) = -ln 2 * [log2(-log2 u) + log2(ln 2)],
+// so g * log2(e) = -log2(-log2 u) - log2(ln 2).  The softmax over levels is
+// invariant to a shift shared by all levels, so the kernels use
+//   h = -log2(-log2 u),  z'_k = kappa log2(e) l_k + h_k,  p = softmax(z'/tau in log2 units),
+// which equals softmax((kappa l + g)/tau) (Alg. 1).  u = (x mod 2^23 + 1/2) 2^-23 is
+// built exactly from the low 23 bits of the Philox word.
+__device__ __forceinline__ float gumbel_log2_from_word(uint32_t x) {
+  const float one_plus = __uint_as_float(0x3F800000u | (x & 0x007FFFFFu));  // 1 + j 2^-23
+  const float u = one_plus - __uint_as_float(0x3F7FFFFFu);                 // (j + 1/2) 2^-23, exact
+  return -fast_log2(neg_log2_unit(u));
 }
 
 template <int K>
-__device__ __forceinline__ void draw_noise(uint32_t key0, uint32_t key1, uint32_t t, uint64_t i,
-                                           int noise, float (&g)[K]) {
+__device__ __forceinline__ void draw_noise(const PhiloxKeys& keys, uint32_t t, uint64_t i,
+                                           int noise, float (&h)[K]) {
   if (!noise) {
 #pragma unroll
-    for (int k = 0; k < K; ++k) g[k] = 0.0f;
+    for (int k = 0; k < K; ++k) h[k] = 0.0f;
     return;
   }
 #pragma unroll
   for (int blk = 0; blk < (K + 3) / 4; ++blk) {
     const uint4 w = philox4x32_10(static_cast<uint32_t>(i), static_cast<uint32_t>(i >> 32), t,
-                                  static_cast<uint32_t>(blk), key0, key1);
+                                  static_cast<uint32_t>(blk), keys);
     const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j)
-      if (4 * blk + j < K) g[4 * blk + j] = gumbel_from_word(ws[j]);
+      if (4 * blk + j < K) h[4 * blk + j] = gumbel_log2_from_word(ws[j]);
   }
 }
 
 // Tempered softmax over the levels and the soft value (Alg. 1):
-//   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k.
-// w~ is carried as q_m + delta, delta = sum_j p_j (q_j - q_m), m = argmax z, so
-// q_k - w~ = (q_k - q_m) - delta keeps full relative accuracy when p is
-// nearly one-hot.
+//   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k,
+// evaluated as p_k = 2^((z'_k - z'_max)/tau) / sum_j 2^(...) with z' from the
+// draw above (kappa_log2 = kappa log2 e).  w~ is carried as q_m + delta,
+// delta = sum_j p_j (q_j - q_m), m = argmax z', so q_k - w~ = (q_k - q_m) - delta
+// keeps full relative accuracy when p is nearly one-hot.
 template <int K>
 struct Soft {
   float p[K];
@@ -117,38 +135,56 @@ struct Soft {
 };
 
 template <int K>
-__device__ __forceinline__ void relax(const float (&l)[K], const float (&g)[K], float kappa,
-                                      float scale_log2, const float (&q)[kMaxLevels],
-                                      Soft<K>& s) {
+__device__ __forceinline__ void relax(const float (&l)[K], const float (&h)[K], float kappa_log2,
+                                      float inv_tau, const float (&q)[kMaxLevels], Soft<K>& s) {
   float z[K];
   float zmax = -INFINITY;
-  int m = 0;
-#pragma unroll
-  for (int k = 0; k < K; ++k) {
-    z[k] = fmaf(kappa, l[k], g[k]) * scale_log2;  // (kappa l + g)/tau in log2 units
-    if (z[k] > zmax) {
-      zmax = z[k];
-      m = k;
-    }
-  }
-  float sum = 0.0f;
-#pragma unroll
-  for (int k = 0; k < K; ++k) {
-    s.p[k] = fast_exp2(z[k] - zmax);
-    sum += s.p[k];
-  }
-  const float inv = __fdividef(1.0f, sum);
   float qm = q[0];
 #pragma unroll
-  for (int k = 1; k < K; ++k) qm = (m == k) ? q[k] : qm;
+  for (int k = 0; k < K; ++k) {
+    z[k] = fmaf(kappa_log2, l[k], h[k]);
+    if (z[k] > zmax) {
+      zmax = z[k];
+      qm = q[k];
+    }
+  }
+  const float off = -zmax * inv_tau;
+  float sum = 0.0f;
   float delta = 0.0f;
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    s.p[k] *= inv;
+    s.p[k] = fast_exp2(fmaf(z[k], inv_tau, off));
+    sum += s.p[k];
     delta = fmaf(s.p[k], q[k] - qm, delta);
   }
+  const float inv = __fdividef(1.0f, sum);
+#pragma unroll
+  for (int k = 0; k < K; ++k) s.p[k] *= inv;
   s.qm = qm;
-  s.delta = delta;
+  s.delta = delta * inv;
+}
+
+// Soft value only (forward): w~ = sum_k 2^((z'_k - z'_max)/tau) q_k / sum_k 2^(...).
+template <int K>
+__device__ __forceinline__ float soft_value(const float (&l)[K], const float (&h)[K],
+                                            float kappa_log2, float inv_tau,
+                                            const float (&q)[kMaxLevels]) {
+  float z[K];
+  float zmax = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    z[k] = fmaf(kappa_log2, l[k], h[k]);
+    zmax = fmaxf(zmax, z[k]);
+  }
+  const float off = -zmax * inv_tau;
+  float sum = 0.0f, num = 0.0f;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    const float e = fast_exp2(fmaf(z[k], inv_tau, off));
+    sum += e;
+    num = fmaf(e, q[k], num);
+  }
+  return num * __fdividef(1.0f, sum);
 }
 
 __device__ __forceinline__ void load_w4(const void* W, int64_t q, int bf16, float (&w)[4]) {
@@ -184,8 +220,9 @@ __device__ __forceinline__ float round_d(float d, int bf16) {
   return bf16 ? __bfloat162float(__float2bfloat16_rn(d)) : d;
 }
 
-__device__ __forceinline__ float sign_of(float c) {
-  return c > 0.0f ? 1.0f : (c < 0.0f ? -1.0f : 0.0f);
+// lr * sign(c) with sign(0) = 0.
+__device__ __forceinline__ float lr_sign(float lr, float c) {
+  return c != 0.0f ? copysignf(lr, c) : 0.0f;
 }
 
 __device__ __forceinline__ float group_sum(float v, int seg) {
@@ -234,10 +271,10 @@ template <int K>
 __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
+  const PhiloxKeys keys = philox_keys(P.key0, P.key1);
   const int lane = threadIdx.x & 31;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const float scale_log2 = P.inv_tau * 1.4426950408889634f;
-  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+    for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
        base < P.nq; base += stride) {
     const int64_t qi = base + lane;
     if (qi >= P.nq) continue;
@@ -257,11 +294,9 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
       float lj[K], g[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-      draw_noise<K>(P.key0, P.key1, P.t, i, P.noise, g);
-      Soft<K> sm;
-      relax<K>(lj, g, P.kappa, scale_log2, q, sm);
+      draw_noise<K>(keys, P.t, i, P.noise, g);
+      const float wt = soft_value<K>(lj, g, P.kappa_log2, P.inv_tau, q);
       // D = s w~ - W as one rounding (identical in every kernel that forms D)
-      const float wt = sm.qm + sm.delta;
       what[j] = __fmul_rn(s, wt);
       d[j] = __fmaf_rn(s, wt, -w[j]);
     }
@@ -277,16 +312,22 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
 // the updated registers.  Bytes per weight with look-ahead: read 8K + 4 + b_W,
 // write 8K + 2 (D bf16).
 // ---------------------------------------------------------------------------
+// Blocks per SM the register budget aims for: 3 x 256 threads (<= 85 registers)
+// for up to 4 levels, 2 x 256 beyond.
+template <int K>
+struct BwdOcc {
+  static constexpr int value = K <= 4 ? 3 : 2;
+};
+
 template <int K, bool kExport>
-__global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
+__global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
+  const PhiloxKeys keys = philox_keys(P.key0, P.key1);
   const int lane = threadIdx.x & 31;
   const int seg = P.group >> 2;  // lanes per scale group
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const float scale_log2 = P.inv_tau * 1.4426950408889634f;
-  const float scale_log2_next = P.inv_tau_next * 1.4426950408889634f;
-  float loss_acc = 0.0f;
+      float loss_acc = 0.0f;
 
   for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
        base < P.nq; base += stride) {
@@ -329,9 +370,9 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
       float lj[K], g[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-      draw_noise<K>(P.key0, P.key1, P.t, i, P.noise, g);
+      draw_noise<K>(keys, P.t, i, P.noise, g);
       Soft<K> sm;
-      relax<K>(lj, g, P.kappa, scale_log2, q, sm);
+      relax<K>(lj, g, P.kappa_log2, P.inv_tau, q, sm);
       const float wt = sm.qm + sm.delta;
       const float dj = round_d(__fmaf_rn(s, wt, -w[j]), P.d_bf16);
       loss_acc = fmaf(0.5f * dj, Gq[j], loss_acc);
@@ -347,7 +388,7 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
           // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l - lr wd l - lr sign(c);
           // m <- b2 m + (1-b2) g.  The decay is one fma on l (no rounded 1 - lr wd).
           const float c = fmaf(P.b1, m[k][j], (1.0f - P.b1) * dl);
-          l[k][j] = fmaf(-P.lrwd_l, l[k][j], l[k][j]) - P.lr_l * sign_of(c);
+          l[k][j] = fmaf(-P.lrwd_l, l[k][j], l[k][j]) - lr_sign(P.lr_l, c);
           m[k][j] = fmaf(P.b2, m[k][j], (1.0f - P.b2) * dl);
         }
       }
@@ -369,7 +410,7 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
 
     if (!P.scales_frozen) {
       const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
-      s = fmaf(-P.lrwd_s, s, s) - P.lr_s * sign_of(c);
+      s = fmaf(-P.lrwd_s, s, s) - lr_sign(P.lr_s, c);
       ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
     }
     if (active) {
@@ -393,10 +434,9 @@ __global__ void __launch_bounds__(kEwThreads) k_backward(const EwParams P) {
           float lj[K], g[K];
 #pragma unroll
           for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-          draw_noise<K>(P.key0, P.key1, P.t_next, i, P.noise, g);
-          Soft<K> sm;
-          relax<K>(lj, g, P.kappa_next, scale_log2_next, q, sm);
-          d[j] = __fmaf_rn(s, sm.qm + sm.delta, -w[j]);
+          draw_noise<K>(keys, P.t_next, i, P.noise, g);
+          const float wt = soft_value<K>(lj, g, P.kappa_log2_next, P.inv_tau_next, q);
+          d[j] = __fmaf_rn(s, wt, -w[j]);
         }
         store_d4(P.D, qi, P.d_bf16, d);
       }

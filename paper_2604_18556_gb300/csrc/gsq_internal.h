@@ -46,11 +46,11 @@ struct EwParams {
   int noise;          // 0: g = 0
   // step t (backward / forward)
   uint32_t t;
-  float kappa, inv_tau, kappa_over_tau;
+  float kappa_log2, inv_tau, kappa_over_tau;  // kappa_log2 = kappa * log2(e)
   // look-ahead forward (t + 1)
   int lookahead;
   uint32_t t_next;
-  float kappa_next, inv_tau_next;
+  float kappa_log2_next, inv_tau_next;
   // Lion
   float lr_l, lr_s, b1, b2, wd_l, wd_s;
   float lrwd_l, lrwd_s;  // lr * wd, rounded once from double

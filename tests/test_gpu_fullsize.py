@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_common import TOL_BF16, Case, assert_close, assert_gemm_bound, gsq
+from gpu_common import TOL_BF16, Case, assert_close, assert_gemm_bound, assert_grad_close, gsq
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -89,9 +89,8 @@ def test_full_size_step_sampled_rows(name):
                           f"tcgen05 GEMM rows, expert {e}")
     del Hb
     torch.cuda.empty_cache()
-    assert_close(glr, ref.d_logits, TOL_BF16, "dL/dlogits rows")
-    if ref.d_scales is not None:
-        assert_close(gsr, ref.d_scales, TOL_BF16, "dL/dscales rows")
+    assert_grad_close(glr, gsr if ref.d_scales is not None else None, ref, case.prob, tau0,
+                      w.kappa, TOL_BF16, "rows")
 
     # (b) the benchmark's step: update with look-ahead, state-synced on the rows
     case.layer.step(0, tau0, w.kappa, next_tau=tau1, next_kappa=w.kappa, loss=loss)

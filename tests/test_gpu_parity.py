@@ -7,7 +7,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_common import TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound, gsq
+from gpu_common import (TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound,
+                        assert_grad_close, grad_bounds, gsq)
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -67,9 +68,14 @@ def test_step_loss_and_gradients(name, gemm):
     ref = O.step(case.prob, case.oracle_init(), 3, TAU[name], 1.0, update=False)
     assert_close(loss.cpu().numpy(), [ref.loss], tol, "loss")
     assert_close(case.G(), ref.G, tol, "G")
-    assert_close(gl.cpu().numpy(), ref.d_logits, tol, "dL/dlogits")
-    if ref.d_scales is not None:
-        assert_close(gs.cpu().numpy(), ref.d_scales, tol, "dL/dscales")
+    if gemm == "f32":
+        assert_close(gl.cpu().numpy(), ref.d_logits, tol, "dL/dlogits")
+        if ref.d_scales is not None:
+            assert_close(gs.cpu().numpy(), ref.d_scales, tol, "dL/dscales")
+    else:
+        # gradients are linear in G: G's bf16 tolerance carried through (see grad_bounds)
+        assert_grad_close(gl.cpu().numpy(), gs.cpu().numpy() if ref.d_scales is not None else None,
+                          ref, case.prob, TAU[name], 1.0, tol, name)
     if gemm == "bf16":
         # the tensor-core GEMM against exact products of its own bf16 operands
         D, H, G = case.D(), case.H_operand(), case.G()
@@ -100,14 +106,13 @@ def _check_lion(gpu, orc, theta_in, c_orc, lr, flip_frac, what):
     return int(flip.sum())
 
 
-def _check_momentum(gpu, orc, grad, b2, tol, what):
+def _check_momentum(gpu, orc, grad_bound, b2, what):
     """m' = b2 m + (1 - b2) g with the same m on both sides: the difference is
-    (1 - b2) times the gradient difference, so the gradient's tolerance carries
-    over (|dg| <= tol (|g| + rms g)), plus fp32 rounding of m'."""
+    (1 - b2) times the gradient difference, so the gradient's bound carries
+    over, plus fp32 rounding of m'."""
     gpu = np.asarray(gpu, np.float64).reshape(-1)
     orc = np.asarray(orc, np.float64).reshape(-1)
-    g = np.asarray(grad, np.float64).reshape(-1)
-    bound = (1 - b2) * tol * (np.abs(g) + np.sqrt(np.mean(g * g))) + \
+    bound = (1 - b2) * np.asarray(grad_bound, np.float64).reshape(-1) + \
         2 * np.spacing(np.abs(orc).astype(np.float32)).astype(np.float64)
     bad = np.abs(gpu - orc) > bound
     assert not bad.any(), (what, int(bad.sum()))
@@ -136,12 +141,20 @@ def test_step_update(name, gemm):
         c_l = w.beta1 * m0 + (1 - w.beta1) * res.d_logits
         _check_lion(gpu.logits, st_sync.logits, st_gpu_before.logits, c_l, w.lr_logits, 2 * tol,
                     "logits")
-        _check_momentum(gpu.m_logits, st_sync.m_logits, res.d_logits, w.beta2, tol, "logit momentum")
+        if gemm == "f32":
+            gb_l = tol * (np.abs(res.d_logits) + np.sqrt(np.mean(res.d_logits ** 2)))
+            gb_s = None if res.d_scales is None else \
+                tol * (np.abs(res.d_scales) + np.sqrt(np.mean(res.d_scales ** 2)))
+        else:
+            f, gscale, bs = grad_bounds(res, case.prob, tol)
+            gb_l = (1.0 / TAU[name]) * f * gscale[None] + tol * np.abs(res.d_logits)
+            gb_s = None if res.d_scales is None else bs + tol * np.abs(res.d_scales)
+        _check_momentum(gpu.m_logits, st_sync.m_logits, gb_l, w.beta2, "logit momentum")
         if res.d_scales is not None:
             c_s = w.beta1 * st_gpu_before.m_scales.astype(np.float64) + (1 - w.beta1) * res.d_scales
             _check_lion(gpu.scales, st_sync.scales, st_gpu_before.scales, c_s, w.lr_scales,
                         2 * tol, "scales")
-            _check_momentum(gpu.m_scales, st_sync.m_scales, res.d_scales, w.beta2, tol, "scale momentum")
+            _check_momentum(gpu.m_scales, st_sync.m_scales, gb_s, w.beta2, "scale momentum")
         else:
             assert np.array_equal(gpu.scales, st_gpu_before.scales)
         losses.append(float(loss.item()))

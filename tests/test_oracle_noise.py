@@ -43,11 +43,11 @@ def test_philox_vectorised_matches_scalar():
 
 
 def test_uniform_is_exact_open_interval_fp32():
-    x = np.array([0, 1, 511, 512, 0xFFFFFFFF, 0x80000000], dtype=np.uint32)
+    x = np.array([0, 1, 0x800000, 0x800001, 0xFFFFFFFF, 0x400000, 0x7FFFFF], dtype=np.uint32)
     u = philox.uniform_from_word(x)
-    assert u[0] == 2.0 ** -24 and u[1] == 2.0 ** -24 and u[2] == 2.0 ** -24
-    assert u[3] == 3 * 2.0 ** -24
-    assert u[4] == 1.0 - 2.0 ** -24
+    assert u[0] == 2.0 ** -24 and u[2] == 2.0 ** -24          # only the low 23 bits count
+    assert u[1] == 3 * 2.0 ** -24 and u[3] == 3 * 2.0 ** -24
+    assert u[4] == 1.0 - 2.0 ** -24 and u[6] == 1.0 - 2.0 ** -24
     assert u[5] == 0.5 + 2.0 ** -24
     assert np.all(u.astype(np.float32).astype(np.float64) == u)   # representable in fp32
     assert np.all((u > 0) & (u < 1))

@@ -259,8 +259,11 @@ EwParams base_params(gsq_layer* L) {
   p.W = L->ws + L->lay.W;
   p.D = L->ws + L->lay.D;
   p.G = fptr(L, L->lay.G);
-  p.key0 = static_cast<uint32_t>(d.seed);
-  p.key1 = static_cast<uint32_t>(d.seed >> 32);
+  const uint32_t key0 = static_cast<uint32_t>(d.seed), key1 = static_cast<uint32_t>(d.seed >> 32);
+  for (uint32_t r = 0; r < 10; ++r) {
+    p.keys.k0[r] = key0 + r * 0x9E3779B9u;
+    p.keys.k1[r] = key1 + r * 0xBB67AE85u;
+  }
   p.noise = (d.flags & GSQ_FLAG_NO_NOISE) ? 0 : 1;
   p.lr_l = d.lr_logits;
   p.lr_s = d.lr_scales;

@@ -25,21 +25,10 @@ namespace {
 // S-box multipliers 0xD2511F53 / 0xCD9E8D57, Weyl key increments 0x9E3779B9 /
 // 0xBB67AE85.  Counter (lo32(i), hi32(i), t, level block), key = seed.
 // ---------------------------------------------------------------------------
-// Round keys of the Weyl schedule, computed once per thread from the seed (the
-// same for every thread, so they live in uniform registers).
-struct PhiloxKeys {
-  uint32_t k0[10], k1[10];
-};
-
-__device__ __forceinline__ PhiloxKeys philox_keys(uint32_t key0, uint32_t key1) {
-  PhiloxKeys k;
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    k.k0[r] = key0 + static_cast<uint32_t>(r) * 0x9E3779B9u;
-    k.k1[r] = key1 + static_cast<uint32_t>(r) * 0xBB67AE85u;
-  }
-  return k;
-}
+// Round keys of the Weyl schedule (key + r * (0x9E3779B9, 0xBB67AE85)), computed
+// on the host and passed in the kernel parameters, so every XOR reads its key
+// from the constant bank.
+using PhiloxKeys = PhiloxRoundKeys;
 
 __device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
                                                const PhiloxKeys& k) {
@@ -80,7 +69,7 @@ __device__ __forceinline__ float fast_log2(float x) {
 __device__ __forceinline__ float neg_log2_unit(float u) {
   const uint32_t bu = __float_as_uint(u);
   const int e = static_cast<int>(bu - 0x3F3504F3u) >> 23;
-  const float m = __uint_as_float(bu - (static_cast<uint32_t>(e) << 23));  // 2^-e u
+  const float m = __uint_as_float(bu + static_cast<uint32_t>(e) * 0xFF800000u);  // 2^-e u
   const float y = __fdividef(m - 1.0f, m + 1.0f);
   const float y2 = y * y;
   constexpr float c1 = 2.8853900817779268f;   // 2 / ln 2
@@ -271,7 +260,7 @@ template <int K>
 __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
-  const PhiloxKeys keys = philox_keys(P.key0, P.key1);
+  const PhiloxKeys& keys = P.keys;
   const int lane = threadIdx.x & 31;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
@@ -323,7 +312,7 @@ template <int K, bool kExport>
 __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
-  const PhiloxKeys keys = philox_keys(P.key0, P.key1);
+  const PhiloxKeys& keys = P.keys;
   const int lane = threadIdx.x & 31;
   const int seg = P.group >> 2;  // lanes per scale group
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -335,33 +324,31 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
     const bool active = qi < P.nq;
     const int64_t qc = active ? qi : 0;
     // l: logits; m: Lion momentum (or, in export mode, the logit gradient)
+    // Lanes past the end (only in the last warp) read quad 0 and take G = 0, so
+    // every value stays finite and their loss and scale-gradient terms vanish;
+    // nothing is stored for them.  A scale group is never split across active
+    // and inactive lanes.
     float l[K][4], m[K][4];
-    float w[4] = {0.f, 0.f, 0.f, 0.f};
-    float4 gv = make_float4(0.f, 0.f, 0.f, 0.f);
-    float s = 0.0f, ms = 0.0f;
+    float w[4];
+    float s, ms = 0.0f;
     const int64_t gidx = (qc * 4) >> P.log2_group;
 #pragma unroll
-    for (int k = 0; k < K; ++k)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) l[k][j] = m[k][j] = 0.0f;
-    if (active) {
+    for (int k = 0; k < K; ++k) {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qc);
+      l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
+    }
+    if (!kExport) {
 #pragma unroll
       for (int k = 0; k < K; ++k) {
-        const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qi);
-        l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(P.m_logits + k * P.n) + qc);
+        m[k][0] = v.x; m[k][1] = v.y; m[k][2] = v.z; m[k][3] = v.w;
       }
-      if (!kExport) {
-#pragma unroll
-        for (int k = 0; k < K; ++k) {
-          const float4 v = __ldcs(reinterpret_cast<const float4*>(P.m_logits + k * P.n) + qi);
-          m[k][0] = v.x; m[k][1] = v.y; m[k][2] = v.z; m[k][3] = v.w;
-        }
-      }
-      gv = __ldcs(reinterpret_cast<const float4*>(P.G) + qi);
-      load_w4(P.W, qi, P.w_bf16, w);
-      s = __ldg(P.scales + gidx);
-      if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
     }
+    float4 gv = __ldcs(reinterpret_cast<const float4*>(P.G) + qc);
+    if (!active) gv = make_float4(0.f, 0.f, 0.f, 0.f);
+    load_w4(P.W, qc, P.w_bf16, w);
+    s = __ldg(P.scales + gidx);
+    if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
     const float Gq[4] = {gv.x, gv.y, gv.z, gv.w};
     float ds = 0.0f;
 #pragma unroll

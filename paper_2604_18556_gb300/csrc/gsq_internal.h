@@ -22,6 +22,11 @@ struct DevFlags {
   unsigned int pad[61];
 };
 
+// Philox4x32-10 round keys: k0[r] = key0 + r * 0x9E3779B9, k1[r] = key1 + r * 0xBB67AE85.
+struct PhiloxRoundKeys {
+  uint32_t k0[10], k1[10];
+};
+
 // Everything the elementwise kernels need, passed by value.
 struct EwParams {
   // shape
@@ -42,7 +47,7 @@ struct EwParams {
   void* D;            // [n]
   const float* G;     // [n]
   // noise
-  uint32_t key0, key1;
+  PhiloxRoundKeys keys;
   int noise;          // 0: g = 0
   // step t (backward / forward)
   uint32_t t;

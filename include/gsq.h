@@ -238,6 +238,59 @@ typedef struct gsq_profile {
 GSQ_API gsq_status gsq_profile_enable(gsq_layer* layer, int32_t on);
 GSQ_API gsq_status gsq_profile_read(gsq_layer* layer, gsq_profile* out);
 
+/* ---- allocation-free backward update --------------------------------------
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory (a host that owns a fixed pool, a plugin whose
+ * host forbids allocation, code running where allocation is not allowed).
+ * It runs the fused backward + Lion kernel of gsq_step on buffers the caller
+ * owns, for a dL/dW^ the caller supplies (from this library's loss GEMM, read
+ * with gsq_get_tensor(GSQ_T_G), or from any other objective):
+ *   recompute noise and p for (step, tau, kappa); dL/dl and dL/ds from G;
+ *   Lion on logits and scales in place; loss_dev (nullable) = 1/2 sum D*G with
+ *   D = s w~ - W rounded to d_dtype (as the loss GEMM consumed it).
+ * Layouts are those of gsq_get_tensor: logits and m_logits [K][E][R][C] fp32,
+ * scales and m_scales [E][R][C/G] fp32, W [E][R][C] (w_dtype), G [E][R][C] fp32.
+ * Its only scratch (a counter and one double per thread block) is a static
+ * 131,328-byte device array inside libgsq that every GPU loading the library
+ * holds until the process exits; nothing is allocated, so E*R*C is limited to
+ * 16,777,216 weights (larger layers return GSQ_ERR_SHAPE).  The first call on a
+ * device looks up that array's device address (cudaGetSymbolAddress); make that
+ * first call before any stream capture on the device.  All calls on one GPU
+ * share its copy of the array and it keeps the last call's contents (the call
+ * clears the counter before launching): calls that overlap on the same GPU (for
+ * instance on two streams) race and corrupt each other's loss value; the state
+ * update itself does not depend on the array.  Errors: GSQ_ERR_INVALID_ARG,
+ * GSQ_ERR_SHAPE, GSQ_ERR_UNSUPPORTED, GSQ_ERR_CUDA, message via gsq_last_error(). */
+typedef struct gsq_backward_args {
+  int32_t num_experts;
+  int32_t out_features;
+  int32_t in_features;
+  int32_t num_levels;
+  float grid[GSQ_MAX_LEVELS];
+  int32_t group_size;
+  int32_t w_dtype;
+  int32_t d_dtype;
+  uint32_t flags;      /* GSQ_FLAG_NO_NOISE */
+  const void* W;
+  const float* G;
+  float* logits;
+  float* m_logits;
+  float* scales;
+  float* m_scales;
+  float* loss_dev;
+  uint64_t seed;
+  uint64_t step;
+  float tau;
+  float kappa;
+  float lr_logits;
+  float lr_scales;
+  float beta1;
+  float beta2;
+  float wd_logits;
+  float wd_scales;
+} gsq_backward_args;
+GSQ_API gsq_status gsq_backward_update_noalloc(const gsq_backward_args* args, void* stream);
+
 /* Release the handle (host memory only; the workspace stays the caller's).
  * Returns GSQ_ERR_INVALID_ARG for NULL. */
 GSQ_API gsq_status gsq_destroy(gsq_layer* layer);

@@ -38,6 +38,15 @@ gsq_status fail(gsq_status st, const char* fmt, ...) {
   return st;
 }
 
+}  // namespace
+
+gsq_status set_last_error(gsq_status st, const char* msg) {
+  g_last_error = msg;
+  return st;
+}
+
+namespace {
+
 gsq_status cuda_fail(cudaError_t e, const char* what) {
   return fail(GSQ_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
 }

@@ -69,6 +69,9 @@ struct EwParams {
   float* loss_out;     // nullable
 };
 
+// Records `msg` as this thread's gsq_last_error() text and returns `st` (gsq_api.cu).
+gsq_status set_last_error(gsq_status st, const char* msg);
+
 // ---- launchers (gsq_elementwise.cu) ----------------------------------------
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);

@@ -36,7 +36,7 @@ KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init"]
 EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "gsq_project",
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
             "gsq_sync_status", "gsq_profile_enable", "gsq_profile_read", "gsq_destroy",
-            "gsq_last_error", "gsq_version"]
+            "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc"]
 
 
 class gsq_layer_desc(Structure):
@@ -53,6 +53,18 @@ class gsq_layer_desc(Structure):
 
 class gsq_profile(Structure):
     _fields_ = [("launches", c_int32 * GSQ_K_COUNT), ("total_ms", c_float * GSQ_K_COUNT)]
+
+
+class gsq_backward_args(Structure):
+    _fields_ = [
+        ("num_experts", c_int32), ("out_features", c_int32), ("in_features", c_int32),
+        ("num_levels", c_int32), ("grid", c_float * GSQ_MAX_LEVELS), ("group_size", c_int32),
+        ("w_dtype", c_int32), ("d_dtype", c_int32), ("flags", c_uint32), ("W", c_void_p),
+        ("G", c_void_p), ("logits", c_void_p), ("m_logits", c_void_p), ("scales", c_void_p),
+        ("m_scales", c_void_p), ("loss_dev", c_void_p), ("seed", c_uint64), ("step", c_uint64),
+        ("tau", c_float), ("kappa", c_float), ("lr_logits", c_float), ("lr_scales", c_float),
+        ("beta1", c_float), ("beta2", c_float), ("wd_logits", c_float), ("wd_scales", c_float),
+    ]
 
 
 class GsqError(RuntimeError):
@@ -83,6 +95,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "gsq_destroy": (c_int32, [P]),
         "gsq_last_error": (c_char_p, []),
         "gsq_version": (c_char_p, []),
+        "gsq_backward_update_noalloc": (c_int32, [POINTER(gsq_backward_args), P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -180,6 +193,11 @@ def gsq_last_error() -> str:
 
 def gsq_version() -> str:
     return _lib.gsq_version().decode()
+
+
+def gsq_backward_update_noalloc(args: gsq_backward_args, stream: int) -> None:
+    """The allocation-free backward + Lion update (see include/gsq.h)."""
+    _check(_lib.gsq_backward_update_noalloc(byref(args), stream))
 
 
 # ---- convenience wrapper over torch memory and streams -----------------------

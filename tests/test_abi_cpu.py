@@ -44,23 +44,24 @@ def test_every_declared_symbol_is_exported(lib):
         assert getattr(cdll, n) is not None
 
 
-def test_descriptor_layout_matches_c(lib, tmp_path):
-    fields = [f for f, _ in lib.gsq_layer_desc._fields_]
+@pytest.mark.parametrize("struct", ["gsq_layer_desc", "gsq_profile", "gsq_backward_args"])
+def test_struct_layout_matches_c(lib, tmp_path, struct):
+    cls = getattr(lib, struct)
+    fields = [f for f, _ in cls._fields_]
     prog = "#include <stdio.h>\n#include <stddef.h>\n#include \"gsq.h\"\nint main(void){\n"
-    prog += 'printf("size %zu\\n", sizeof(gsq_layer_desc));\n'
+    prog += f'printf("size %zu\\n", sizeof({struct}));\n'
     for f in fields:
-        prog += f'printf("{f} %zu\\n", offsetof(gsq_layer_desc, {f}));\n'
-    prog += 'printf("profile %zu\\n", sizeof(gsq_profile));\nreturn 0;}\n'
+        prog += f'printf("{f} %zu\\n", offsetof({struct}, {f}));\n'
+    prog += "return 0;}\n"
     c = tmp_path / "layout.c"
     c.write_text(prog)
     exe = tmp_path / "layout"
     subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
     out = dict(ln.split() for ln in subprocess.run([str(exe)], capture_output=True, text=True,
                                                    check=True).stdout.splitlines())
-    assert int(out["size"]) == ctypes.sizeof(lib.gsq_layer_desc)
-    assert int(out["profile"]) == ctypes.sizeof(lib.gsq_profile)
+    assert int(out["size"]) == ctypes.sizeof(cls)
     for f in fields:
-        assert int(out[f]) == getattr(lib.gsq_layer_desc, f).offset, f
+        assert int(out[f]) == getattr(cls, f).offset, f
 
 
 def _desc(lib, **kw):

@@ -58,24 +58,54 @@ __device__ __forceinline__ float fast_log2(float x) {
   return y;
 }
 
-// -log2(u) for u in [2^-24, 1 - 2^-24], accurate to a few ulp in relative terms
-// even as u -> 1 (where -log2 u -> 0).  Branch-free range reduction u = 2^e m
+__device__ __forceinline__ float fast_rcp(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Two weights at a time: packed fp32 pair arithmetic (f32x2 instructions, one
+// issue for two correctly rounded operations).
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 neg2(float2 a) { return make_float2(-a.x, -a.y); }
+__device__ __forceinline__ float2 rcp2(float2 a) { return make_float2(fast_rcp(a.x), fast_rcp(a.y)); }
+__device__ __forceinline__ float2 exp2_2(float2 a) { return make_float2(fast_exp2(a.x), fast_exp2(a.y)); }
+
+// log2(u) for u in [2^-24, 1 - 2^-24], accurate to a few ulp in relative terms
+// even as u -> 1 (where log2 u -> 0).  Branch-free range reduction u = 2^e m
 // with m in [sqrt(1/2), sqrt(2)): subtracting the bit pattern of sqrt(1/2) from
 // the bits of u moves the exponent boundary to sqrt(2) (the integer-offset
 // reduction of fdlibm-style logf).  Then log2 m = (2 / ln 2) atanh(y),
 // y = (m - 1)/(m + 1), by the odd series 2(y + y^3/3 + y^5/5 + ...)
 // (Abramowitz & Stegun 4.1.27); |y| <= 0.1716, so terms through y^9 leave a
 // relative remainder below 2e-9.
-__device__ __forceinline__ float neg_log2_unit(float u) {
-  const uint32_t bu = __float_as_uint(u);
-  const int e = static_cast<int>(bu - 0x3F3504F3u) >> 23;
-  const float m = __uint_as_float(bu + static_cast<uint32_t>(e) * 0xFF800000u);  // 2^-e u
-  const float y = __fdividef(m - 1.0f, m + 1.0f);
-  const float y2 = y * y;
-  constexpr float c1 = 2.8853900817779268f;   // 2 / ln 2
+// Arithmetic right shift by 23 of one 32-bit lane.  Written in PTX: with
+// nvcc 13.0 for sm_103a the C++ form of the two lanes' shifts below was
+// combined into one operation on the register pair that corrupted lane x.
+__device__ __forceinline__ int sar23(uint32_t x) {
+  int r;
+  asm("shr.s32 %0, %1, 23;" : "=r"(r) : "r"(x));
+  return r;
+}
+
+__device__ __forceinline__ float2 log2_unit2(float2 u) {
+  constexpr float c1 = 2.8853900817779268f;  // 2 / ln 2
   constexpr float c3 = c1 / 3.0f, c5 = c1 / 5.0f, c7 = c1 / 7.0f, c9 = c1 / 9.0f;
-  const float poly = fmaf(y2, fmaf(y2, fmaf(y2, fmaf(y2, c9, c7), c5), c3), c1);
-  return -fmaf(y, poly, static_cast<float>(e));
+  const uint32_t b0 = __float_as_uint(u.x), b1 = __float_as_uint(u.y);
+  const int e0 = sar23(b0 - 0x3F3504F3u);
+  const int e1 = sar23(b1 - 0x3F3504F3u);
+  const float2 m = make_float2(__uint_as_float(b0 + static_cast<uint32_t>(e0) * 0xFF800000u),
+                               __uint_as_float(b1 + static_cast<uint32_t>(e1) * 0xFF800000u));
+  const float2 y = mul2(add2(m, f2(-1.0f)), rcp2(add2(m, f2(1.0f))));
+  const float2 y2 = mul2(y, y);
+  float2 poly = fma2(y2, f2(c9), f2(c7));
+  poly = fma2(y2, poly, f2(c5));
+  poly = fma2(y2, poly, f2(c3));
+  poly = fma2(y2, poly, f2(c1));
+  return fma2(y, poly, make_float2(static_cast<float>(e0), static_cast<float>(e1)));
 }
 
 // The Gumbel draw in log2 units, up to a constant common to every level:
@@ -84,96 +114,107 @@ __device__ __forceinline__ float neg_log2_unit(float u) {
 // invariant to a shift shared by all levels, so the kernels use
 //   h = -log2(-log2 u),  z'_k = kappa log2(e) l_k + h_k,  p = softmax(z'/tau in log2 units),
 // which equals softmax((kappa l + g)/tau) (Alg. 1).  u = (x mod 2^23 + 1/2) 2^-23 is
-// built exactly from the low 23 bits of the Philox word.
-__device__ __forceinline__ float gumbel_log2_from_word(uint32_t x) {
-  const float one_plus = __uint_as_float(0x3F800000u | (x & 0x007FFFFFu));  // 1 + j 2^-23
-  const float u = one_plus - __uint_as_float(0x3F7FFFFFu);                 // (j + 1/2) 2^-23, exact
-  return -fast_log2(neg_log2_unit(u));
+// built exactly from the low 23 bits of the Philox word.  Two words -> two draws.
+__device__ __forceinline__ float2 gumbel_log2_2(uint32_t x0, uint32_t x1) {
+  const float2 one_plus = make_float2(__uint_as_float(0x3F800000u | (x0 & 0x007FFFFFu)),
+                                      __uint_as_float(0x3F800000u | (x1 & 0x007FFFFFu)));
+  const float2 u = add2(one_plus, f2(-__uint_as_float(0x3F7FFFFFu)));  // (j + 1/2) 2^-23, exact
+  const float2 L = log2_unit2(u);                                      // log2 u < 0
+  return make_float2(-fast_log2(-L.x), -fast_log2(-L.y));
 }
 
+// Noise of weights i0 (even) and i0 + 1 for every level (one Philox call per
+// weight and block of four levels).
 template <int K>
-__device__ __forceinline__ void draw_noise(const PhiloxKeys& keys, uint32_t t, uint64_t i,
-                                           int noise, float (&h)[K]) {
+__device__ __forceinline__ void draw_noise2(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
+                                            int noise, float2 (&h)[K]) {
   if (!noise) {
 #pragma unroll
-    for (int k = 0; k < K; ++k) h[k] = 0.0f;
+    for (int k = 0; k < K; ++k) h[k] = f2(0.0f);
     return;
   }
 #pragma unroll
   for (int blk = 0; blk < (K + 3) / 4; ++blk) {
-    const uint4 w = philox4x32_10(static_cast<uint32_t>(i), static_cast<uint32_t>(i >> 32), t,
-                                  static_cast<uint32_t>(blk), keys);
-    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    const uint32_t lo = static_cast<uint32_t>(i0), hi = static_cast<uint32_t>(i0 >> 32);
+    const uint4 a = philox4x32_10(lo, hi, t, static_cast<uint32_t>(blk), keys);
+    const uint4 b = philox4x32_10(lo + 1u, hi, t, static_cast<uint32_t>(blk), keys);
+    const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j)
-      if (4 * blk + j < K) h[4 * blk + j] = gumbel_log2_from_word(ws[j]);
+      if (4 * blk + j < K) h[4 * blk + j] = gumbel_log2_2(wa[j], wb[j]);
   }
 }
 
-// Tempered softmax over the levels and the soft value (Alg. 1):
+// Tempered softmax over the levels and the soft value (Alg. 1), two weights:
 //   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k,
 // evaluated as p_k = 2^((z'_k - z'_max)/tau) / sum_j 2^(...) with z' from the
 // draw above (kappa_log2 = kappa log2 e).  w~ is carried as q_m + delta,
 // delta = sum_j p_j (q_j - q_m), m = argmax z', so q_k - w~ = (q_k - q_m) - delta
 // keeps full relative accuracy when p is nearly one-hot.
 template <int K>
-struct Soft {
-  float p[K];
-  float qm;
-  float delta;
+struct Soft2 {
+  float2 p[K];
+  float2 qm;
+  float2 delta;
 };
 
 template <int K>
-__device__ __forceinline__ void relax(const float (&l)[K], const float (&h)[K], float kappa_log2,
-                                      float inv_tau, const float (&q)[kMaxLevels], Soft<K>& s) {
-  float z[K];
-  float zmax = -INFINITY;
-  float qm = q[0];
+__device__ __forceinline__ void relax2(const float2 (&l)[K], const float2 (&h)[K],
+                                       float kappa_log2, float inv_tau,
+                                       const float (&q)[kMaxLevels], Soft2<K>& s) {
+  float2 z[K];
+  float zx = -INFINITY, zy = -INFINITY, qx = q[0], qy = q[0];
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    z[k] = fmaf(kappa_log2, l[k], h[k]);
-    if (z[k] > zmax) {
-      zmax = z[k];
-      qm = q[k];
+    z[k] = fma2(f2(kappa_log2), l[k], h[k]);
+    if (z[k].x > zx) {
+      zx = z[k].x;
+      qx = q[k];
+    }
+    if (z[k].y > zy) {
+      zy = z[k].y;
+      qy = q[k];
     }
   }
-  const float off = -zmax * inv_tau;
-  float sum = 0.0f;
-  float delta = 0.0f;
+  const float2 qm = make_float2(qx, qy);
+  const float2 off = mul2(make_float2(zx, zy), f2(-inv_tau));
+  float2 sum = f2(0.0f), delta = f2(0.0f);
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    s.p[k] = fast_exp2(fmaf(z[k], inv_tau, off));
-    sum += s.p[k];
-    delta = fmaf(s.p[k], q[k] - qm, delta);
+    s.p[k] = exp2_2(fma2(z[k], f2(inv_tau), off));
+    sum = add2(sum, s.p[k]);
+    delta = fma2(s.p[k], add2(f2(q[k]), neg2(qm)), delta);
   }
-  const float inv = __fdividef(1.0f, sum);
+  const float2 inv = rcp2(sum);
 #pragma unroll
-  for (int k = 0; k < K; ++k) s.p[k] *= inv;
+  for (int k = 0; k < K; ++k) s.p[k] = mul2(s.p[k], inv);
   s.qm = qm;
-  s.delta = delta * inv;
+  s.delta = mul2(delta, inv);
 }
 
-// Soft value only (forward): w~ = sum_k 2^((z'_k - z'_max)/tau) q_k / sum_k 2^(...).
+// Soft value only (forward), two weights:
+//   w~ = sum_k 2^((z'_k - z'_max)/tau) q_k / sum_k 2^(...).
 template <int K>
-__device__ __forceinline__ float soft_value(const float (&l)[K], const float (&h)[K],
-                                            float kappa_log2, float inv_tau,
-                                            const float (&q)[kMaxLevels]) {
-  float z[K];
-  float zmax = -INFINITY;
+__device__ __forceinline__ float2 soft_value2(const float2 (&l)[K], const float2 (&h)[K],
+                                              float kappa_log2, float inv_tau,
+                                              const float (&q)[kMaxLevels]) {
+  float2 z[K];
+  float zx = -INFINITY, zy = -INFINITY;
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    z[k] = fmaf(kappa_log2, l[k], h[k]);
-    zmax = fmaxf(zmax, z[k]);
+    z[k] = fma2(f2(kappa_log2), l[k], h[k]);
+    zx = fmaxf(zx, z[k].x);
+    zy = fmaxf(zy, z[k].y);
   }
-  const float off = -zmax * inv_tau;
-  float sum = 0.0f, num = 0.0f;
+  const float2 off = mul2(make_float2(zx, zy), f2(-inv_tau));
+  float2 sum = f2(0.0f), num = f2(0.0f);
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    const float e = fast_exp2(fmaf(z[k], inv_tau, off));
-    sum += e;
-    num = fmaf(e, q[k], num);
+    const float2 e = exp2_2(fma2(z[k], f2(inv_tau), off));
+    sum = add2(sum, e);
+    num = fma2(e, f2(q[k]), num);
   }
-  return num * __fdividef(1.0f, sum);
+  return mul2(num, rcp2(sum));
 }
 
 __device__ __forceinline__ void load_w4(const void* W, int64_t q, int bf16, float (&w)[4]) {
@@ -263,7 +304,7 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
   const PhiloxKeys& keys = P.keys;
   const int lane = threadIdx.x & 31;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
        base < P.nq; base += stride) {
     const int64_t qi = base + lane;
     if (qi >= P.nq) continue;
@@ -278,16 +319,17 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
     const float s = __ldg(P.scales + ((qi * 4) >> P.log2_group));
     float d[4], what[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint64_t i = static_cast<uint64_t>(qi) * 4 + j;
-      float lj[K], g[K];
+    for (int pr = 0; pr < 2; ++pr) {
+      float2 l2[K], h[K];
 #pragma unroll
-      for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-      draw_noise<K>(keys, P.t, i, P.noise, g);
-      const float wt = soft_value<K>(lj, g, P.kappa_log2, P.inv_tau, q);
-      // D = s w~ - W as one rounding (identical in every kernel that forms D)
-      what[j] = __fmul_rn(s, wt);
-      d[j] = __fmaf_rn(s, wt, -w[j]);
+      for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+      draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+      const float2 wt = soft_value2<K>(l2, h, P.kappa_log2, P.inv_tau, q);
+      // D = s w~ - W as one rounding per weight (identical in every kernel that forms D)
+      const float2 wh = mul2(f2(s), wt);
+      const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
+      what[2 * pr] = wh.x; what[2 * pr + 1] = wh.y;
+      d[2 * pr] = dd.x; d[2 * pr + 1] = dd.y;
     }
     store_d4(P.D, qi, P.d_bf16, d);
     if (P.what) reinterpret_cast<float4*>(P.what)[qi] = make_float4(what[0], what[1], what[2], what[3]);
@@ -301,11 +343,10 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
 // the updated registers.  Bytes per weight with look-ahead: read 8K + 4 + b_W,
 // write 8K + 2 (D bf16).
 // ---------------------------------------------------------------------------
-// Blocks per SM the register budget aims for: 3 x 256 threads (<= 85 registers)
-// for up to 4 levels, 2 x 256 beyond.
+// Blocks per SM the register budget aims for (measured best on GB300).
 template <int K>
 struct BwdOcc {
-  static constexpr int value = K <= 4 ? 3 : 2;
+  static constexpr int value = 2;
 };
 
 template <int K, bool kExport>
@@ -316,14 +357,13 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
   const int lane = threadIdx.x & 31;
   const int seg = P.group >> 2;  // lanes per scale group
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-      float loss_acc = 0.0f;
+  float2 loss2 = f2(0.0f);
 
   for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
        base < P.nq; base += stride) {
     const int64_t qi = base + lane;
     const bool active = qi < P.nq;
     const int64_t qc = active ? qi : 0;
-    // l: logits; m: Lion momentum (or, in export mode, the logit gradient)
     // Lanes past the end (only in the last warp) read quad 0 and take G = 0, so
     // every value stays finite and their loss and scale-gradient terms vanish;
     // nothing is stored for them.  A scale group is never split across active
@@ -349,38 +389,44 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
     load_w4(P.W, qc, P.w_bf16, w);
     s = __ldg(P.scales + gidx);
     if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
-    const float Gq[4] = {gv.x, gv.y, gv.z, gv.w};
-    float ds = 0.0f;
+    const float2 Gq[2] = {make_float2(gv.x, gv.y), make_float2(gv.z, gv.w)};
+    float2 ds2 = f2(0.0f);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint64_t i = static_cast<uint64_t>(qc) * 4 + j;
-      float lj[K], g[K];
+    for (int pr = 0; pr < 2; ++pr) {
+      float2 l2[K], h[K];
 #pragma unroll
-      for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-      draw_noise<K>(keys, P.t, i, P.noise, g);
-      Soft<K> sm;
-      relax<K>(lj, g, P.kappa_log2, P.inv_tau, q, sm);
-      const float wt = sm.qm + sm.delta;
-      const float dj = round_d(__fmaf_rn(s, wt, -w[j]), P.d_bf16);
-      loss_acc = fmaf(0.5f * dj, Gq[j], loss_acc);
-      ds = fmaf(Gq[j], wt, ds);
-      const float A = P.kappa_over_tau * Gq[j] * s;
+      for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+      draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
+      Soft2<K> sm;
+      relax2<K>(l2, h, P.kappa_log2, P.inv_tau, q, sm);
+      const float2 wt = add2(sm.qm, sm.delta);
+      const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
+      const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
+      loss2 = fma2(mul2(f2(0.5f), dj), Gq[pr], loss2);
+      ds2 = fma2(Gq[pr], wt, ds2);
+      const float2 A = mul2(f2(P.kappa_over_tau * s), Gq[pr]);
 #pragma unroll
       for (int k = 0; k < K; ++k) {
         // dL/dl_k = (kappa/tau) G s p_k (q_k - w~)   (softmax Jacobian, App. B)
-        const float dl = A * sm.p[k] * ((q[k] - sm.qm) - sm.delta);
+        const float2 dk = add2(add2(f2(q[k]), neg2(sm.qm)), neg2(sm.delta));
+        const float2 dl = mul2(A, mul2(sm.p[k], dk));
         if (kExport) {
-          m[k][j] = dl;
+          m[k][2 * pr] = dl.x;
+          m[k][2 * pr + 1] = dl.y;
         } else {
           // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l - lr wd l - lr sign(c);
           // m <- b2 m + (1-b2) g.  The decay is one fma on l (no rounded 1 - lr wd).
-          const float c = fmaf(P.b1, m[k][j], (1.0f - P.b1) * dl);
-          l[k][j] = fmaf(-P.lrwd_l, l[k][j], l[k][j]) - lr_sign(P.lr_l, c);
-          m[k][j] = fmaf(P.b2, m[k][j], (1.0f - P.b2) * dl);
+          const float2 mo = make_float2(m[k][2 * pr], m[k][2 * pr + 1]);
+          const float2 c = fma2(f2(P.b1), mo, mul2(f2(1.0f - P.b1), dl));
+          const float2 ln = add2(fma2(f2(-P.lrwd_l), l2[k], l2[k]),
+                                 make_float2(-lr_sign(P.lr_l, c.x), -lr_sign(P.lr_l, c.y)));
+          const float2 mn = fma2(f2(P.b2), mo, mul2(f2(1.0f - P.b2), dl));
+          l[k][2 * pr] = ln.x; l[k][2 * pr + 1] = ln.y;
+          m[k][2 * pr] = mn.x; m[k][2 * pr + 1] = mn.y;
         }
       }
     }
-    ds = group_sum(ds, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
+    const float ds = group_sum(ds2.x + ds2.y, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
 
     if (kExport) {
       if (active) {
@@ -416,20 +462,21 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
         // forward of step t+1 from the updated logits and scale (Alg. 1)
         float d[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint64_t i = static_cast<uint64_t>(qi) * 4 + j;
-          float lj[K], g[K];
+        for (int pr = 0; pr < 2; ++pr) {
+          float2 l2[K], h[K];
 #pragma unroll
-          for (int k = 0; k < K; ++k) lj[k] = l[k][j];
-          draw_noise<K>(keys, P.t_next, i, P.noise, g);
-          const float wt = soft_value<K>(lj, g, P.kappa_log2_next, P.inv_tau_next, q);
-          d[j] = __fmaf_rn(s, wt, -w[j]);
+          for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+          draw_noise2<K>(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+          const float2 wt = soft_value2<K>(l2, h, P.kappa_log2_next, P.inv_tau_next, q);
+          const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
+          d[2 * pr] = dd.x;
+          d[2 * pr + 1] = dd.y;
         }
         store_d4(P.D, qi, P.d_bf16, d);
       }
     }
   }
-  reduce_loss(loss_acc, P);
+  reduce_loss(loss2.x + loss2.y, P);
 }
 
 // ---------------------------------------------------------------------------

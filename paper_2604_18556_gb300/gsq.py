@@ -16,7 +16,9 @@ from ctypes import (POINTER, Structure, byref, c_char_p, c_float, c_int32, c_int
                     c_uint32, c_uint64, c_void_p)
 from typing import Optional, Sequence
 
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libgsq.so")
+# GSQ_LIBRARY, if set, names a libgsq.so built elsewhere (same ABI).
+LIB_PATH = os.environ.get("GSQ_LIBRARY") or os.path.join(
+    os.path.dirname(os.path.abspath(__file__)), "libgsq.so")
 
 # ---- constants mirrored from gsq.h -------------------------------------------
 GSQ_OK, GSQ_ERR_INVALID_ARG, GSQ_ERR_SHAPE, GSQ_ERR_WORKSPACE, GSQ_ERR_CUDA = 0, 1, 2, 3, 4

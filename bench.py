@@ -51,6 +51,54 @@ def _dist():
     return rank, world, local
 
 
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
+ELEMENTWISE_SRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc", "gsq_elementwise.cu")
+
+
+def source_sha256(path: str = ELEMENTWISE_SRC) -> str:
+    import hashlib
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def committed_traffic(workload: str):
+    """DRAM bytes (read + write) per k_backward launch from the committed ncu
+    capture, or None when there is none for this workload or the kernel source
+    has changed since it was taken."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    with open(TRAFFIC_FILE) as f:
+        d = json.load(f)
+    if d.get("source_sha256") != source_sha256():
+        return None
+    return d.get("workloads", {}).get(workload, {}).get("k_backward_dram_bytes_per_launch")
+
+
+def rank_workload(w, rank: int, world: int):
+    """Each rank quantizes its own independent layer of the same shape (weak
+    scaling: rows and experts never exchange data, so ranks share nothing)."""
+    if world <= 1:
+        return w
+    import dataclasses
+    return dataclasses.replace(w, seed=w.seed + rank, data_seed=w.data_seed + 100 * rank)
+
+
+def max_over_ranks(x: float, device) -> float:
+    """Largest value over the process group (the slowest rank defines the time)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_steps_per_s(ms_per_step: float, world: int) -> float:
+    """All ranks' steps per second: world layers advance one step every ms_per_step."""
+    return world * 1000.0 / ms_per_step
+
+
 def _peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -236,10 +284,7 @@ def gpu_arm(args, rank, world, local):
     from paper_2604_18556_gb300 import gsq, inputs
     from paper_2604_18556_gb300 import configs as C
 
-    w = _workload(args.workload)
-    if world > 1:   # each rank quantizes its own layer of the same shape
-        import dataclasses
-        w = dataclasses.replace(w, seed=w.seed + rank, data_seed=w.data_seed + 100 * rank)
+    w = rank_workload(_workload(args.workload), rank, world)
     W = inputs.make_weight(w, device="cuda")
     H = inputs.make_gram(w, device="cuda")
     H_host = H[0].double().cpu().numpy() if rank == 0 and not args.no_cpu_baseline else None
@@ -283,12 +328,9 @@ def gpu_arm(args, rank, world, local):
     prof = layer.profile_read()
     layer.profile_enable(False)
     layer.sync_status()
-    if world > 1:
-        tt = torch.tensor([ms_total], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ms_total, torch.device("cuda", local))
     ms_step = ms_total / args.steps
-    value = world * 1000.0 / ms_step
+    value = whole_job_steps_per_s(ms_step, world)
 
     hbm, tf_burst, tf_sust, peak_src = _peaks()
     n = w.n
@@ -301,11 +343,7 @@ def gpu_arm(args, rank, world, local):
     flops = w.gemm_flops_per_step()
     bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
     gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
-    traffic = None
-    tf_path = os.path.join(ROOT, "profiles", "dram_traffic.json")
-    if os.path.exists(tf_path):
-        with open(tf_path) as f:
-            traffic = json.load(f).get(w.name, {}).get("backward_bytes_per_launch")
+    traffic = committed_traffic(w.name)
     roofline = {"kernel": "k_backward (fused backward + Lion + next forward)", "bound": "hbm",
                 "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
                 "traffic": traffic, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",

@@ -209,6 +209,7 @@ struct gsq_layer {
   int num_sms;
   int grid_fwd, grid_bwd;
   bool tc;
+  int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
   // pending forward (D valid for these arguments)
   bool d_ready;
   uint64_t d_step;
@@ -350,6 +351,7 @@ gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
     g.G = fptr(L, L->lay.G);
     g.alpha = 2.0f;
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+    g.tile_n = L->tile_n;
     e = launch_tc_gemm(g, L->num_sms, s);
   } else {
     SimtGemm g;
@@ -487,6 +489,12 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   };
   L->grid_fwd = clamp_grid(ew_grid_size(sh.K, 0, L->num_sms));
   L->grid_bwd = clamp_grid(ew_grid_size(sh.K, 1, L->num_sms));
+  L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
+                             L->num_sms);
+  if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128 or 256: override the choice
+    const int v = std::atoi(tn);
+    if (v == 128 || v == 256) L->tile_n = v;
+  }
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   DevFlags* flags = reinterpret_cast<DevFlags*>(L->ws + lay.flags);

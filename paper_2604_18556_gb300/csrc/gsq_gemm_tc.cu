@@ -24,19 +24,25 @@
 namespace gsq {
 namespace {
 
-constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
+constexpr int TC_BM = 128, TC_BK = 64;
 constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;
-constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;
-constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr int TC_THREADS = 192;
-constexpr int TC_TMEM_COLS = 2 * TC_BN;
-constexpr int TC_SMEM_BYTES = TC_STAGES * TC_STAGE_BYTES + 256 + 1024;
-// kind::f16 instruction descriptor: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1),
-// B bf16 (10-12 = 1), both K-major (bits 15, 16 = 0), N>>3 at 17-22, M>>4 at 24-28.
-constexpr uint32_t TC_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                              (static_cast<uint32_t>(TC_BN >> 3) << 17) |
-                              (static_cast<uint32_t>(TC_BM >> 4) << 24);
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// Tile shape M = 128 x N = BN (256 or 128) x 64; the pipeline depth fills ~192 KiB.
+template <int BN>
+struct TcCfg {
+  static constexpr int kBBytes = BN * TC_BK * 2;
+  static constexpr int kStageBytes = TC_A_BYTES + kBBytes;
+  static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
+  static constexpr int kTmemCols = 2 * BN;  // double-buffered fp32 accumulator
+  static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
+  // kind::f16 instruction descriptor: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1),
+  // B bf16 (10-12 = 1), both K-major (bits 15, 16 = 0), N>>3 at 17-22, M>>4 at 24-28.
+  static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                                     (static_cast<uint32_t>(BN >> 3) << 17) |
+                                     (static_cast<uint32_t>(TC_BM >> 4) << 24);
+};
 
 struct TcArgs {
   int E, R, C;
@@ -117,12 +123,13 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          (static_cast<uint64_t>(2) << 61);
 }
 
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t da, uint64_t db, uint32_t accum) {
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t da, uint64_t db, uint32_t idesc,
+                                          uint32_t accum) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
-      "l"(da), "l"(db), "r"(TC_IDESC), "r"(accum));
+      "l"(da), "l"(db), "r"(idesc), "r"(accum));
 }
 
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
@@ -160,9 +167,15 @@ __device__ __forceinline__ void tile_coords(int tile, int Mt, int Nt, int& e, in
   m = r - n * Mt;
 }
 
+template <int BN>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const TcArgs args) {
+  constexpr int TC_BN = BN;
+  constexpr int TC_STAGES = TcCfg<BN>::kStages;
+  constexpr int TC_STAGE_BYTES = TcCfg<BN>::kStageBytes;
+  constexpr int TC_TMEM_COLS = TcCfg<BN>::kTmemCols;
+  constexpr uint32_t TC_IDESC = TcCfg<BN>::kIdesc;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -202,6 +215,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int Mt = (args.R + TC_BM - 1) / TC_BM;
   const int Nt = (args.C + TC_BN - 1) / TC_BN;
   const int KB = (args.C + TC_BK - 1) / TC_BK;
+  static_assert(TC_STAGES >= 2, "pipeline depth");
   const int tiles = args.E * Mt * Nt;
 
   if (warp == 0) {
@@ -265,7 +279,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           const uint64_t db = sw128_desc(sa + TC_A_BYTES);
 #pragma unroll
           for (int k = 0; k < TC_BK / 16; ++k)  // advance 16 bf16 = 32 B = 2 units of 16 B
-            umma_bf16(d_tmem, da + 2 * k, db + 2 * k, (kb | k) != 0 ? 1u : 0u);
+            umma_bf16(d_tmem, da + 2 * k, db + 2 * k, TC_IDESC, (kb | k) != 0 ? 1u : 0u);
           umma_commit(empty_bar + stage);
           if (++stage == TC_STAGES) {
             stage = 0;
@@ -360,19 +374,24 @@ bool encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-}  // namespace
-
-bool tc_gemm_supported(int device) {
+bool tc_supported_impl(int device) {
   cudaDeviceProp prop;
   if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return false;
   return prop.major == 10 && prop.minor == 3 && get_encode_fn() != nullptr;
 }
 
-cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
+// Fraction of the last wave's SMs that have a tile: tiles / (waves * SMs).
+double wave_balance(int64_t tiles, int num_sms) {
+  const int64_t waves = (tiles + num_sms - 1) / num_sms;
+  return static_cast<double>(tiles) / static_cast<double>(waves * num_sms);
+}
+
+template <int BN>
+cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e =
-        cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM_BYTES);
+    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         TcCfg<BN>::kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
@@ -380,7 +399,7 @@ cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
   if (!encode_kmajor_bf16(&ta, g.D, static_cast<uint64_t>(g.C),
                           static_cast<uint64_t>(g.E) * g.R, TC_BM) ||
       !encode_kmajor_bf16(&tb, g.H, static_cast<uint64_t>(g.C),
-                          static_cast<uint64_t>(g.E) * g.C, TC_BN))
+                          static_cast<uint64_t>(g.E) * g.C, BN))
     return cudaErrorInvalidValue;
   TcArgs a;
   a.E = g.E;
@@ -389,11 +408,33 @@ cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
   a.G = g.G;
   a.alpha = g.alpha;
   a.flags = g.flags;
-  const int Mt = (g.R + TC_BM - 1) / TC_BM, Nt = (g.C + TC_BN - 1) / TC_BN;
+  const int Mt = (g.R + TC_BM - 1) / TC_BM, Nt = (g.C + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  k_tc_gemm<<<grid, TC_THREADS, TC_SMEM_BYTES, s>>>(ta, tb, a);
+  k_tc_gemm<BN><<<grid, TC_THREADS, TcCfg<BN>::kSmemBytes, s>>>(ta, tb, a);
   return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
+
+int tc_gemm_tile_n(int E, int R, int C, int num_sms) {
+  // 128 x 256 tiles unless their last wave leaves many SMs idle and 128 x 128
+  // tiles balance clearly better (e.g. a 4096 x 4096 layer: 3.37 waves of 256-wide
+  // tiles on 152 SMs, 6.74 waves of 128-wide ones).
+  const int64_t mt = (R + TC_BM - 1) / TC_BM;
+  const double b256 = wave_balance(static_cast<int64_t>(E) * mt * ((C + 255) / 256), num_sms);
+  const double b128 = wave_balance(static_cast<int64_t>(E) * mt * ((C + 127) / 128), num_sms);
+  // Measured on GB300: 128-wide tiles lose more to the narrower MMA than they
+  // gain in balance (4096 x 4096 layer: 142 us vs 114 us), so 256 stays the
+  // choice unless the balance gap is extreme.
+  return (b256 < 0.6 && b128 > b256 + 0.25) ? 128 : 256;
+}
+
+cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
+  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.R, g.C, num_sms);
+  return bn == 128 ? launch_tc_gemm_bn<128>(g, num_sms, s) : launch_tc_gemm_bn<256>(g, num_sms, s);
 }
 
 }  // namespace gsq

@@ -148,8 +148,10 @@ struct TcGemm {
   float* G;
   float alpha;
   DevFlags* flags;
+  int tile_n;  // 0: choose 128 or 256 by wave balance
 };
 bool tc_gemm_supported(int device);
+int tc_gemm_tile_n(int E, int R, int C, int num_sms);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 
 }  // namespace gsq

@@ -262,3 +262,22 @@ def test_trajectory_ternary_full_run():
     keep = om >= 1e-5
     assert np.array_equal(gc[keep], oc[keep])
     assert_close(gpu.scales, st.scales, TOL_F32, "scales after 50 steps")
+
+
+@pytest.mark.parametrize("tile_n", ["128", "256"])
+@pytest.mark.parametrize("name", ["q_proj", "gate_proj", "moe_kquant"])
+def test_tc_gemm_tile_widths(name, tile_n, monkeypatch):
+    """Both tensor-core tile widths (chosen per layer by wave balance) on ragged
+    shapes, against exact products of the kernel's own bf16 operands."""
+    monkeypatch.setenv("GSQ_GEMM_TILE_N", tile_n)
+    w = SMALL[name]
+    case = Case(w, gemm="bf16")
+    loss = torch.zeros(1, device="cuda")
+    case.layer.step(0, TAU[name], 1.0, loss=loss)
+    torch.cuda.synchronize()
+    D, H, G = case.D(), case.H_operand(), case.G()
+    rows = np.arange(w.experts * w.rows)
+    for e in range(w.experts):
+        sel = rows // w.rows == e
+        assert_gemm_bound(G[sel], D[sel], H[e], f"tile N = {tile_n}, expert {e}")
+    assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())

@@ -30,6 +30,10 @@ What one step computes (paper references):
              generalised from the binary threshold to K levels)
   packing    symmetric group-wise b-bit codes + fp16 scale per group (§4.1),
              or a two-level K-Quant-like super-block (§4.4, App. E).
+  local shift  (§3.2 "Higher bit-widths", Fig. 1): instead of one logit per grid
+             level, 5 logits per weight for shifts delta in {-2..2} around the
+             initial index j0; the level of shift delta is G[clip(j0 + delta)], so
+             the same relaxation runs over a per-weight window of 5 levels.
 
 Readings where the paper is silent are listed at the top of the design notes
 (kappa multiplies the logit; summed, un-normalised loss; Philox stream; absmax
@@ -46,6 +50,7 @@ import numpy as np
 from . import philox
 
 SUB_BLOCK = 16      # K-Quant-like sub-block (one 6-bit sub-scale code)
+SHIFTS = 5          # local-shift logits: delta in {-2, -1, 0, 1, 2} (§3.2)
 SUPER_BLOCK = 256   # K-Quant-like super-block (one fp16 d)
 
 
@@ -71,9 +76,15 @@ class Problem:
     wd_logits: float = 1.0
     wd_scales: float = 0.0
     noise: bool = True
+    shift: bool = False                 # local-shift parameterisation (§3.2)
 
     @property
     def K(self) -> int:
+        """Number of logits per weight: the grid size, or 5 shifts."""
+        return SHIFTS if self.shift else int(len(self.grid))
+
+    @property
+    def levels(self) -> int:
         return int(len(self.grid))
 
 
@@ -91,12 +102,14 @@ class RowState:
     m_scales: np.ndarray                # float32 [nr, C // group]
     kq_d: Optional[np.ndarray] = None   # float32 [nr, C // 256] (fp16 values) for kquant2
     kq_sc: Optional[np.ndarray] = None  # int32 [nr, C // 16] for kquant2
+    j0: Optional[np.ndarray] = None     # uint8 [nr, C]: initial grid index (local shift)
 
     def copy(self) -> "RowState":
         return RowState(self.row_ids.copy(), self.W.copy(), self.logits.copy(),
                         self.scales.copy(), self.m_logits.copy(), self.m_scales.copy(),
                         None if self.kq_d is None else self.kq_d.copy(),
-                        None if self.kq_sc is None else self.kq_sc.copy())
+                        None if self.kq_sc is None else self.kq_sc.copy(),
+                        None if self.j0 is None else self.j0.copy())
 
     def subset(self, idx) -> "RowState":
         idx = np.asarray(idx)
@@ -104,7 +117,8 @@ class RowState:
                         self.logits[:, idx].copy(), self.scales[idx].copy(),
                         self.m_logits[:, idx].copy(), self.m_scales[idx].copy(),
                         None if self.kq_d is None else self.kq_d[idx].copy(),
-                        None if self.kq_sc is None else self.kq_sc[idx].copy())
+                        None if self.kq_sc is None else self.kq_sc[idx].copy(),
+                        None if self.j0 is None else self.j0[idx].copy())
 
 
 def flat_index(prob: Problem, row_ids: np.ndarray) -> np.ndarray:
@@ -142,6 +156,22 @@ def noise(prob: Problem, st: RowState, t: int) -> np.ndarray:
     return philox.gumbel(prob.seed, t, flat_index(prob, st.row_ids), prob.K)
 
 
+def shift_index(j0: np.ndarray, levels: int) -> np.ndarray:
+    """Grid index of every shift: clip(j0 + delta, 0, levels - 1), delta = -2..2
+    (§3.2: j_i = clip(j_i^0 + delta_i, 1, 2^b) with 1-based indices).  [5, ...]."""
+    delta = np.arange(-2, 3).reshape((SHIFTS,) + (1,) * np.ndim(j0))
+    return np.clip(np.asarray(j0, dtype=np.int64)[None] + delta, 0, levels - 1)
+
+
+def level_values(prob: Problem, st: RowState) -> np.ndarray:
+    """q_k for every logit k of every weight, broadcastable against [K, nr, C]:
+    the grid itself, or each weight's window G[clip(j0 + delta)] (local shift)."""
+    grid = np.asarray(prob.grid, dtype=np.float64)
+    if prob.shift:
+        return grid[shift_index(st.j0, prob.levels)]
+    return grid[:, None, None]
+
+
 @dataclass
 class Forward:
     g: np.ndarray
@@ -155,7 +185,7 @@ class Forward:
 def forward(prob: Problem, st: RowState, t: int, tau: float, kappa: float) -> Forward:
     g = noise(prob, st, t)
     p = relax(st.logits, g, tau, kappa)
-    wtil = soft_value(p, prob.grid)
+    wtil = np.sum(p * level_values(prob, st), axis=0)     # w~ = sum_k p_k q_k
     s = expand_scales(st.scales, prob.group)
     What = s * wtil
     return Forward(g=g, p=p, wtil=wtil, s=s, What=What, D=What - st.W)
@@ -204,9 +234,10 @@ def loss_bruteforce(W: np.ndarray, What: np.ndarray, X: np.ndarray) -> float:
 # ----------------------------------------------------------------------------
 # backward (App. B softmax Jacobian) and Lion (§3.3, App. B)
 # ----------------------------------------------------------------------------
-def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float):
-    """dL/dl [K, nr, C] and dL/ds [nr, C/G]."""
-    q = np.asarray(prob.grid, dtype=np.float64)[:, None, None]
+def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float, q=None):
+    """dL/dl [K, nr, C] and dL/ds [nr, C/G]; q: level values of every logit."""
+    if q is None:
+        q = np.asarray(prob.grid, dtype=np.float64)[:, None, None]
     d_logits = (kappa / tau) * (G * fw.s)[None] * fw.p * (q - fw.wtil[None])
     nr, C = G.shape
     d_scales = (G * fw.wtil).reshape(nr, C // prob.group, prob.group).sum(axis=2)
@@ -245,7 +276,7 @@ def step(prob: Problem, st: RowState, t: int, tau: float, kappa: float,
     place unless update=False; the reported loss is this step's forward loss."""
     fw = forward(prob, st, t, tau, kappa)
     L, G = loss_and_grad(prob, st.row_ids, fw.D)
-    d_logits, d_scales = backward(prob, fw, G, tau, kappa)
+    d_logits, d_scales = backward(prob, fw, G, tau, kappa, q=level_values(prob, st))
     if scales_frozen(prob):
         d_scales = None
     if update:
@@ -352,23 +383,31 @@ def init_state(prob: Problem, W, row_ids, init_bias: float = 2.0) -> RowState:
         s = init_group_scales(W32, prob.group, prob.grid)
     codes = rtn_codes(W32, np.repeat(s, prob.group, axis=1), prob.grid)
     logits = np.zeros((prob.K, nr, C), dtype=np.float32)
-    for k in range(prob.K):
-        logits[k][codes == k] = np.float32(init_bias)
+    j0 = None
+    if prob.shift:
+        logits[2] = np.float32(init_bias)             # delta = 0: stay on the RTN level
+        j0 = codes.astype(np.uint8)
+    else:
+        for k in range(prob.K):
+            logits[k][codes == k] = np.float32(init_bias)
     return RowState(row_ids=np.asarray(row_ids, dtype=np.int64), W=W32.astype(np.float64),
                     logits=logits, scales=s.astype(np.float32),
                     m_logits=np.zeros_like(logits), m_scales=np.zeros_like(s, dtype=np.float32),
-                    kq_d=kq_d, kq_sc=kq_sc)
+                    kq_d=kq_d, kq_sc=kq_sc, j0=j0)
 
 
 # ----------------------------------------------------------------------------
 # hard projection (Alg. 2, final lines, generalised to K levels)
 # ----------------------------------------------------------------------------
-def project(logits32: np.ndarray):
-    """k* = argmax_k l_k (lowest k on ties) and margin = l_(1) - l_(2) in fp32."""
-    codes = np.argmax(logits32, axis=0).astype(np.uint8)
+def project(logits32: np.ndarray, j0=None, levels: int = 0):
+    """k* = argmax_k l_k (lowest k on ties) and margin = l_(1) - l_(2) in fp32.
+    With local shift the grid code is clip(j0 + k* - 2) (§3.2)."""
+    k = np.argmax(logits32, axis=0)
     srt = np.sort(logits32, axis=0)
     margin = (srt[-1] - srt[-2]).astype(np.float32)
-    return codes, margin
+    if j0 is not None:
+        k = np.clip(np.asarray(j0, dtype=np.int64) + k - 2, 0, levels - 1)
+    return k.astype(np.uint8), margin
 
 
 # ----------------------------------------------------------------------------

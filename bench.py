@@ -172,11 +172,11 @@ def _workload(name):
 
 def _config(w, extra=None):
     cfg = {"workload": f"{w.name}: E={w.experts} R={w.rows} C={w.cols} K={w.K} G={w.group} "
-                       f"W={w.w_dtype} scales={w.scale_mode}",
+                       f"W={w.w_dtype} scales={w.scale_mode} logits/weight={w.L}",
            "tau": f"{w.tau0}->{w.tau1} over {w.steps} steps", "kappa": w.kappa,
            "gemm": "tcgen05 bf16 x bf16 -> fp32",
            "l2": "working set larger than L2 (logits + momenta = "
-                 f"{8 * w.K * w.n / 2**20:.0f} MiB vs 126 MiB L2)"}
+                 f"{8 * w.L * w.n / 2**20:.0f} MiB vs 126 MiB L2)"}
     if extra:
         cfg.update(extra)
     return cfg
@@ -191,7 +191,7 @@ def _oracle_problem(w, H_host, rows):
     prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float), group=w.group,
                      seed=w.seed, scale_mode=w.scale_mode, H=H_host, lr_logits=w.lr_logits,
                      lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2, wd_logits=w.wd_logits,
-                     wd_scales=w.wd_scales)
+                     wd_scales=w.wd_scales, shift=w.param == "shift5")
     return prob
 
 
@@ -291,7 +291,7 @@ def gpu_arm(args, rank, world, local):
     layer = gsq.Layer(W, H, w.grid, w.group, calib_kind="H", scale_mode=w.scale_mode, gemm="bf16",
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                      wd_logits=w.wd_logits, wd_scales=w.wd_scales)
+                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param)
     stream = torch.cuda.current_stream()
     loss = torch.zeros(1, device="cuda")
     T = w.steps
@@ -398,7 +398,7 @@ def e2e_run(args, w, W, H, gsq, torch, rank, world):
     layer = gsq.Layer(Wd, Hd, w.grid, w.group, scale_mode=w.scale_mode, gemm="bf16",
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                      wd_logits=w.wd_logits, wd_scales=w.wd_scales)
+                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param)
     loss = torch.zeros(K, device="cuda")
     for t in range(K):
         layer.step(t, w.tau(t % w.steps), w.kappa, next_tau=w.tau((t + 1) % w.steps),

@@ -72,6 +72,7 @@ enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1 };
 enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
 enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
 enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel draw */
+enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1 };
 
 /* Layer problem (Eq. 1 with a linear f; §3.2; §4.1; Table 5 for the defaults).
  *
@@ -96,6 +97,12 @@ enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel dra
  * gemm_precision  GSQ_GEMM_BF16: the loss contraction G = D (H + H^T) runs on the
  *              tensor cores with bf16 D and H and fp32 accumulation;
  *              GSQ_GEMM_F32: fp32 D and H on the CUDA cores (validation).
+ * param_mode   GSQ_PARAM_FULL: one logit per grid level (§3.2, l in R^{d x 2^b}).
+ *              GSQ_PARAM_SHIFT5: local shift (§3.2 "Higher bit-widths", Fig. 1):
+ *              five logits per weight for shifts delta = -2..2 around the initial
+ *              (round-to-nearest) index j0; shift delta uses level
+ *              grid[clip(j0 + delta, 0, K - 1)].  The projection gives the code
+ *              clip(j0 + argmax - 2).  Logit tensors then hold 5 planes.
  * Limits: 1 <= E, 1 <= R, 8 <= C, C % 8 == 0, E*R*C < 2^40, 2 <= K <= 8.
  */
 typedef struct gsq_layer_desc {
@@ -121,7 +128,7 @@ typedef struct gsq_layer_desc {
   float wd_logits;
   float wd_scales;
   int32_t gemm_precision;
-  int32_t reserved;
+  int32_t param_mode;
 } gsq_layer_desc;
 
 typedef struct gsq_layer gsq_layer; /* opaque handle, host memory owned by libgsq */
@@ -156,8 +163,8 @@ GSQ_API gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, s
  *              step's forward, before the update).
  * grad_logits_dev / grad_scales_dev  device, nullable.  If either is non-null
  *              the step runs in gradient-export mode: it writes the raw
- *              gradients ([K][E][R][C] fp32 and [E][R][C/G] fp32), skips the Lion
- *              update and ignores next_tau.
+ *              gradients ([L][E][R][C] fp32, L logits per weight, and
+ *              [E][R][C/G] fp32), skips the Lion update and ignores next_tau.
  * Never synchronises; graph-capturable for a fixed argument list. */
 GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float kappa, float next_tau,
                     float next_kappa, void* stream, float* loss_dev, float* grad_logits_dev,
@@ -190,16 +197,19 @@ GSQ_API gsq_status gsq_pack(gsq_layer* layer, void* stream, void* out_dev, size_
 
 /* State tensors for inspection, checkpoint and resume. */
 enum {
-  GSQ_T_LOGITS = 0,     /* fp32 [K][E][R][C]                                   */
+  GSQ_T_LOGITS = 0,     /* fp32 [L][E][R][C], L = K (FULL) or 5 (SHIFT5)       */
   GSQ_T_SCALES = 1,     /* fp32 [E][R][C/G] (effective scale d*sc for KQUANT2)  */
-  GSQ_T_MOM_LOGITS = 2, /* fp32 [K][E][R][C]                                   */
+  GSQ_T_MOM_LOGITS = 2, /* fp32 [L][E][R][C]                                   */
   GSQ_T_MOM_SCALES = 3, /* fp32 [E][R][C/G]                                    */
   GSQ_T_D = 4,          /* last forward's D = W^ - W, [E][R][C], bf16 or fp32  */
   GSQ_T_G = 5,          /* last step's dL/dW^, fp32 [E][R][C]                  */
   GSQ_T_W = 6,          /* stored copy of W, [E][R][C], w_dtype                */
   GSQ_T_H = 7,          /* GEMM operand H (symmetrised), [E][C][C], bf16/fp32  */
   GSQ_T_KQ_D = 8,       /* fp16 bits [E*R*C/256] (KQUANT2 only)                */
-  GSQ_T_KQ_SC = 9       /* int8 [E*R*C/16] (KQUANT2 only)                      */
+  GSQ_T_KQ_SC = 9,      /* int8 [E*R*C/16] (KQUANT2 only)                      */
+  GSQ_T_J0 = 10         /* uint8 [E][R][C] initial grid index (SHIFT5 only);   *
+                         * a value >= K set through gsq_set_tensor acts as K-1  *
+                         * (every index is clipped to the grid before use)      */
 };
 
 /* Byte size of tensor `which` (0 when the layer has no such tensor). */
@@ -248,8 +258,9 @@ GSQ_API gsq_status gsq_profile_read(gsq_layer* layer, gsq_profile* out);
  *   recompute noise and p for (step, tau, kappa); dL/dl and dL/ds from G;
  *   Lion on logits and scales in place; loss_dev (nullable) = 1/2 sum D*G with
  *   D = s w~ - W rounded to d_dtype (as the loss GEMM consumed it).
- * Layouts are those of gsq_get_tensor: logits and m_logits [K][E][R][C] fp32,
- * scales and m_scales [E][R][C/G] fp32, W [E][R][C] (w_dtype), G [E][R][C] fp32.
+ * Full parameterisation only (one logit per level).  Layouts are those of
+ * gsq_get_tensor: logits and m_logits [K][E][R][C] fp32, scales and m_scales
+ * [E][R][C/G] fp32, W [E][R][C] (w_dtype), G [E][R][C] fp32.
  * Its only scratch (a counter and one double per thread block) is a static
  * 131,328-byte device array inside libgsq that every GPU loading the library
  * holds until the process exits; nothing is allocated, so E*R*C is limited to

@@ -52,10 +52,16 @@ class Workload:
     wd_scales: float = 0.0
     data_seed: int = 0
     pack: bool = False
+    param: str = "full"        # "full": one logit per level; "shift5": local shift (§3.2)
 
     @property
     def K(self) -> int:
         return len(self.grid)
+
+    @property
+    def L(self) -> int:
+        """Logits per weight: K, or 5 shifts around the initial index."""
+        return 5 if self.param == "shift5" else self.K
 
     @property
     def n(self) -> int:
@@ -73,9 +79,10 @@ class Workload:
     def elementwise_bytes_per_weight(self) -> int:
         """Algorithmic HBM bytes per weight of one steady-state step's fused
         elementwise kernel (backward t + Lion + forward t+1):
-        read logits, logit momentum (4K each), G (4), W (b_W);
-        write logits, logit momentum (4K each), D for the next step (2)."""
-        return 16 * self.K + 4 + self.w_bytes() + 2
+        read logits, logit momentum (4L each, L logits per weight), G (4), W (b_W),
+        the initial index j0 with local shift (1);
+        write logits, logit momentum (4L each), D for the next step (2)."""
+        return 16 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
 
     def gemm_flops_per_step(self) -> int:
         return 2 * self.experts * self.rows * self.cols * self.cols
@@ -101,6 +108,12 @@ WORKLOADS = {
                  group=16, w_dtype="bf16", calib="H", tokens=4096, token_dist="normal",
                  outliers=72, outlier_scale=30.0, steps=100, tau0=1.0, tau1=1.0,
                  scale_mode=SCALE_KQUANT2, lr_scales=0.0, data_seed=5000, pack=True),
+        # The paper's own 3-bit method (§3.2 "Higher bit-widths"): the down_proj layer
+        # with 5 local-shift logits per weight instead of 8.
+        Workload(name="llama8b_down_proj_shift5", experts=1, rows=4096, cols=14336,
+                 grid=GRID_3BIT_SYM, group=128, w_dtype="bf16", calib="H", tokens=256 * 2048,
+                 token_dist="student_t3", outliers=0, outlier_scale=1.0, steps=200, tau0=0.5,
+                 tau1=0.5, data_seed=3000, param="shift5"),
     ]
 }
 

@@ -79,14 +79,15 @@ bool injected(const char* fn) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
-  size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch;
+  size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch, j0;
   size_t total;
 };
 
 struct Shape {
   int64_t E, R, C, n, ng;
   int K, group;
-  bool kquant, d_bf16, w_bf16, x_mode;
+  int L;  // logits per weight: K, or 5 with local shift
+  bool kquant, d_bf16, w_bf16, x_mode, shift;
 };
 
 Shape shape_of(const gsq_layer_desc& d) {
@@ -102,6 +103,8 @@ Shape shape_of(const gsq_layer_desc& d) {
   s.d_bf16 = d.gemm_precision == GSQ_GEMM_BF16;
   s.w_bf16 = d.w_dtype == GSQ_DTYPE_BF16;
   s.x_mode = d.calib_kind == GSQ_CALIB_X;
+  s.shift = d.param_mode == GSQ_PARAM_SHIFT5;
+  s.L = s.shift ? 5 : s.K;
   return s;
 }
 
@@ -116,8 +119,8 @@ Layout layout_of(const Shape& s) {
   const size_t n = static_cast<size_t>(s.n), ng = static_cast<size_t>(s.ng);
   L.flags = take(sizeof(DevFlags));
   L.partials = take(sizeof(double) * kMaxPartials);
-  L.logits = take(4 * n * s.K);
-  L.m_logits = take(4 * n * s.K);
+  L.logits = take(4 * n * s.L);
+  L.m_logits = take(4 * n * s.L);
   L.scales = take(4 * ng);
   L.m_scales = take(4 * ng);
   L.W = take(n * (s.w_bf16 ? 2 : 4));
@@ -127,6 +130,7 @@ Layout layout_of(const Shape& s) {
   L.kq_d = s.kquant ? take(2 * (n / kSuperBlock)) : off;
   L.kq_sc = s.kquant ? take(n / kSubBlock) : off;
   L.hscratch = s.x_mode ? take(static_cast<size_t>(s.E) * s.C * s.C * 4) : off;
+  L.j0 = s.shift ? take(n) : off;
   L.total = off;
   return L;
 }
@@ -174,6 +178,8 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
     return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
   if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE))
     return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
+  if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5)
+    return fail(GSQ_ERR_INVALID_ARG, "bad param_mode %d", d->param_mode);
   const float hp[] = {d->init_bias, d->lr_logits, d->lr_scales, d->beta1, d->beta2, d->wd_logits, d->wd_scales};
   for (float v : hp)
     if (!std::isfinite(v)) return fail(GSQ_ERR_INVALID_ARG, "non-finite hyper-parameter");
@@ -254,7 +260,9 @@ EwParams base_params(gsq_layer* L) {
   const gsq_layer_desc& d = L->desc;
   p.n = s.n;
   p.nq = s.n / 4;
-  p.K = s.K;
+  p.K = s.L;
+  p.nlev = s.K;
+  p.j0 = s.shift ? L->ws + L->lay.j0 : nullptr;
   p.group = s.group;
   int lg = 0;
   while ((1 << lg) < s.group) ++lg;
@@ -384,7 +392,7 @@ size_t tensor_bytes(const gsq_layer* L, int which) {
   const size_t n = static_cast<size_t>(s.n), ng = static_cast<size_t>(s.ng);
   switch (which) {
     case GSQ_T_LOGITS:
-    case GSQ_T_MOM_LOGITS: return 4 * n * s.K;
+    case GSQ_T_MOM_LOGITS: return 4 * n * s.L;
     case GSQ_T_SCALES:
     case GSQ_T_MOM_SCALES: return 4 * ng;
     case GSQ_T_D: return n * (s.d_bf16 ? 2 : 4);
@@ -393,6 +401,7 @@ size_t tensor_bytes(const gsq_layer* L, int which) {
     case GSQ_T_H: return static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4);
     case GSQ_T_KQ_D: return s.kquant ? 2 * (n / kSuperBlock) : 0;
     case GSQ_T_KQ_SC: return s.kquant ? n / kSubBlock : 0;
+    case GSQ_T_J0: return s.shift ? n : 0;
     default: return 0;
   }
 }
@@ -409,6 +418,7 @@ size_t tensor_offset(const gsq_layer* L, int which) {
     case GSQ_T_H: return L->lay.H;
     case GSQ_T_KQ_D: return L->lay.kq_d;
     case GSQ_T_KQ_SC: return L->lay.kq_sc;
+    case GSQ_T_J0: return L->lay.j0;
     default: return 0;
   }
 }
@@ -487,8 +497,8 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if (v > kMaxPartials) v = kMaxPartials;
     return static_cast<int>(v < 1 ? 1 : v);
   };
-  L->grid_fwd = clamp_grid(ew_grid_size(sh.K, 0, L->num_sms));
-  L->grid_bwd = clamp_grid(ew_grid_size(sh.K, 1, L->num_sms));
+  L->grid_fwd = clamp_grid(ew_grid_size(sh.L, 0, L->num_sms, sh.shift));
+  L->grid_bwd = clamp_grid(ew_grid_size(sh.L, 1, L->num_sms, sh.shift));
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
                              L->num_sms);
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128 or 256: override the choice
@@ -558,6 +568,7 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   ip.m_scales = fptr(L, lay.m_scales);
   ip.kq_d = sh.kquant ? reinterpret_cast<uint16_t*>(L->ws + lay.kq_d) : nullptr;
   ip.kq_sc = sh.kquant ? reinterpret_cast<int8_t*>(L->ws + lay.kq_sc) : nullptr;
+  ip.j0 = sh.shift ? L->ws + lay.j0 : nullptr;
   if ((e = launch_init_state(ip, L->num_sms, s)) != cudaSuccess) return bail(cuda_fail(e, "init state"));
   prof_end(L, slot, s);
 
@@ -643,7 +654,9 @@ gsq_status gsq_project(gsq_layer* L, void* stream, uint8_t* codes_dev, float* ma
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   ProjectParams p;
   p.n = L->shape.n;
-  p.K = L->shape.K;
+  p.K = L->shape.L;
+  p.nlev = L->shape.K;
+  p.j0 = L->shape.shift ? L->ws + L->lay.j0 : nullptr;
   p.logits = fptr(L, L->lay.logits);
   p.codes = codes_dev;
   p.margin = margin_dev;
@@ -673,7 +686,9 @@ gsq_status gsq_pack(gsq_layer* L, void* stream, void* out_dev, size_t cap, size_
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   PackParams p;
   p.n = L->shape.n;
-  p.K = L->shape.K;
+  p.K = L->shape.L;
+  p.nlev = L->shape.K;
+  p.j0 = L->shape.shift ? L->ws + L->lay.j0 : nullptr;
   p.group = L->shape.group;
   p.kquant = L->shape.kquant;
   p.logits = fptr(L, L->lay.logits);
@@ -695,7 +710,7 @@ gsq_status gsq_tensor_size(const gsq_layer* L, int32_t which, size_t* bytes) {
   GSQ_INJECT("gsq_tensor_size");
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
   if (!bytes) return fail(GSQ_ERR_INVALID_ARG, "bytes is NULL");
-  if (which < GSQ_T_LOGITS || which > GSQ_T_KQ_SC) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
+  if (which < GSQ_T_LOGITS || which > GSQ_T_J0) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
   *bytes = tensor_bytes(L, which);
   return GSQ_OK;
 }
@@ -703,7 +718,7 @@ gsq_status gsq_tensor_size(const gsq_layer* L, int32_t which, size_t* bytes) {
 static gsq_status copy_tensor(gsq_layer* L, int32_t which, void* dst, const void* src, size_t bytes,
                               void* stream, const char* fn) {
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
-  if (which < GSQ_T_LOGITS || which > GSQ_T_KQ_SC) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
+  if (which < GSQ_T_LOGITS || which > GSQ_T_J0) return fail(GSQ_ERR_INVALID_ARG, "bad tensor id %d", which);
   const size_t need = tensor_bytes(L, which);
   if (need == 0) return fail(GSQ_ERR_INVALID_ARG, "%s: layer has no tensor %d", fn, which);
   if (bytes != need) return fail(GSQ_ERR_INVALID_ARG, "%s: bytes %zu != tensor size %zu", fn, bytes, need);

@@ -145,6 +145,44 @@ __device__ __forceinline__ void draw_noise2(const PhiloxKeys& keys, uint32_t t, 
   }
 }
 
+// Level value of every logit for two weights.  Full parameterisation: the grid
+// (the same for every weight).  Local shift (§3.2): logit d of a weight with
+// initial index j0 stands for grid[clip(j0 + d - 2, 0, nlev - 1)]; the grid is
+// read from a shared-memory copy (8 words in 8 banks: no conflicts).
+// The full grid is kept as scalars (no per-pair copy held in registers).
+template <int K, bool kShift>
+struct Levels2;
+
+template <int K>
+struct Levels2<K, false> {
+  float q[K];
+  __device__ __forceinline__ Levels2(const float (&q_)[kMaxLevels], const float*, int, uint32_t,
+                                     uint32_t) {
+#pragma unroll
+    for (int k = 0; k < K; ++k) q[k] = q_[k];
+  }
+  __device__ __forceinline__ float x(int k) const { return q[k]; }
+  __device__ __forceinline__ float y(int k) const { return q[k]; }
+  __device__ __forceinline__ float2 operator[](int k) const { return f2(q[k]); }
+};
+
+template <int K>
+struct Levels2<K, true> {
+  float2 v[K];
+  __device__ __forceinline__ Levels2(const float (&)[kMaxLevels], const float* sgrid, int nlev,
+                                     uint32_t ja, uint32_t jb) {
+#pragma unroll
+    for (int d = 0; d < K; ++d) {
+      const int ia = min(max(static_cast<int>(ja) + d - 2, 0), nlev - 1);
+      const int ib = min(max(static_cast<int>(jb) + d - 2, 0), nlev - 1);
+      v[d] = make_float2(sgrid[ia], sgrid[ib]);
+    }
+  }
+  __device__ __forceinline__ float x(int k) const { return v[k].x; }
+  __device__ __forceinline__ float y(int k) const { return v[k].y; }
+  __device__ __forceinline__ float2 operator[](int k) const { return v[k]; }
+};
+
 // Tempered softmax over the levels and the soft value (Alg. 1), two weights:
 //   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k,
 // evaluated as p_k = 2^((z'_k - z'_max)/tau) / sum_j 2^(...) with z' from the
@@ -158,22 +196,22 @@ struct Soft2 {
   float2 delta;
 };
 
-template <int K>
+template <int K, class Lv>
 __device__ __forceinline__ void relax2(const float2 (&l)[K], const float2 (&h)[K],
-                                       float kappa_log2, float inv_tau,
-                                       const float (&q)[kMaxLevels], Soft2<K>& s) {
+                                       float kappa_log2, float inv_tau, const Lv& qv,
+                                       Soft2<K>& s) {
   float2 z[K];
-  float zx = -INFINITY, zy = -INFINITY, qx = q[0], qy = q[0];
+  float zx = -INFINITY, zy = -INFINITY, qx = qv.x(0), qy = qv.y(0);
 #pragma unroll
   for (int k = 0; k < K; ++k) {
     z[k] = fma2(f2(kappa_log2), l[k], h[k]);
     if (z[k].x > zx) {
       zx = z[k].x;
-      qx = q[k];
+      qx = qv.x(k);
     }
     if (z[k].y > zy) {
       zy = z[k].y;
-      qy = q[k];
+      qy = qv.y(k);
     }
   }
   const float2 qm = make_float2(qx, qy);
@@ -183,7 +221,7 @@ __device__ __forceinline__ void relax2(const float2 (&l)[K], const float2 (&h)[K
   for (int k = 0; k < K; ++k) {
     s.p[k] = exp2_2(fma2(z[k], f2(inv_tau), off));
     sum = add2(sum, s.p[k]);
-    delta = fma2(s.p[k], add2(f2(q[k]), neg2(qm)), delta);
+    delta = fma2(s.p[k], add2(qv[k], neg2(qm)), delta);
   }
   const float2 inv = rcp2(sum);
 #pragma unroll
@@ -194,10 +232,9 @@ __device__ __forceinline__ void relax2(const float2 (&l)[K], const float2 (&h)[K
 
 // Soft value only (forward), two weights:
 //   w~ = sum_k 2^((z'_k - z'_max)/tau) q_k / sum_k 2^(...).
-template <int K>
+template <int K, class Lv>
 __device__ __forceinline__ float2 soft_value2(const float2 (&l)[K], const float2 (&h)[K],
-                                              float kappa_log2, float inv_tau,
-                                              const float (&q)[kMaxLevels]) {
+                                              float kappa_log2, float inv_tau, const Lv& qv) {
   float2 z[K];
   float zx = -INFINITY, zy = -INFINITY;
 #pragma unroll
@@ -212,7 +249,7 @@ __device__ __forceinline__ float2 soft_value2(const float2 (&l)[K], const float2
   for (int k = 0; k < K; ++k) {
     const float2 e = exp2_2(fma2(z[k], f2(inv_tau), off));
     sum = add2(sum, e);
-    num = fma2(e, f2(q[k]), num);
+    num = fma2(e, qv[k], num);
   }
   return mul2(num, rcp2(sum));
 }
@@ -265,6 +302,16 @@ __device__ __forceinline__ void load_grid(const EwParams& P, float (&q)[kMaxLeve
   for (int k = 0; k < kMaxLevels; ++k) q[k] = P.grid[k];
 }
 
+// Block-wide shared copy of the grid (local shift reads it with per-lane indices).
+__device__ __forceinline__ void fill_shared_grid(const EwParams& P, float* sgrid) {
+  if (threadIdx.x < kMaxLevels) sgrid[threadIdx.x] = P.grid[threadIdx.x];
+  __syncthreads();
+}
+
+__device__ __forceinline__ uint32_t load_j0(const EwParams& P, int64_t q) {
+  return reinterpret_cast<const uint32_t*>(P.j0)[q];
+}
+
 // Deterministic loss reduction: per-block double partials, summed in block
 // order by the last block to finish (no device-side wait).
 __device__ __forceinline__ void reduce_loss(float acc, const EwParams& P) {
@@ -297,10 +344,12 @@ __device__ __forceinline__ void reduce_loss(float acc, const EwParams& P) {
 // Forward: D = s * w~ - W for step (t, tau, kappa); optional W^ export.
 // Bytes per weight: read 4K (logits) + b_W, write 2 or 4 (D).
 // ---------------------------------------------------------------------------
-template <int K>
+template <int K, bool kShift>
 __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
+  __shared__ float sgrid[kMaxLevels];
+  if (kShift) fill_shared_grid(P, sgrid);
   const PhiloxKeys& keys = P.keys;
   const int lane = threadIdx.x & 31;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -317,14 +366,17 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
     float w[4];
     load_w4(P.W, qi, P.w_bf16, w);
     const float s = __ldg(P.scales + ((qi * 4) >> P.log2_group));
+    const uint32_t j4 = kShift ? load_j0(P, qi) : 0u;
     float d[4], what[4];
 #pragma unroll
     for (int pr = 0; pr < 2; ++pr) {
       float2 l2[K], h[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+      const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
+                                  (j4 >> (16 * pr + 8)) & 0xFFu);
       draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
-      const float2 wt = soft_value2<K>(l2, h, P.kappa_log2, P.inv_tau, q);
+      const float2 wt = soft_value2<K>(l2, h, P.kappa_log2, P.inv_tau, qv);
       // D = s w~ - W as one rounding per weight (identical in every kernel that forms D)
       const float2 wh = mul2(f2(s), wt);
       const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
@@ -349,10 +401,12 @@ struct BwdOcc {
   static constexpr int value = 2;
 };
 
-template <int K, bool kExport>
+template <int K, bool kExport, bool kShift>
 __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const EwParams P) {
   float q[kMaxLevels];
   load_grid(P, q);
+  __shared__ float sgrid[kMaxLevels];
+  if (kShift) fill_shared_grid(P, sgrid);
   const PhiloxKeys& keys = P.keys;
   const int lane = threadIdx.x & 31;
   const int seg = P.group >> 2;  // lanes per scale group
@@ -390,15 +444,18 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
     s = __ldg(P.scales + gidx);
     if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
     const float2 Gq[2] = {make_float2(gv.x, gv.y), make_float2(gv.z, gv.w)};
+    const uint32_t j4 = kShift ? load_j0(P, qc) : 0u;
     float2 ds2 = f2(0.0f);
 #pragma unroll
     for (int pr = 0; pr < 2; ++pr) {
       float2 l2[K], h[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+      const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
+                                  (j4 >> (16 * pr + 8)) & 0xFFu);
       draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
       Soft2<K> sm;
-      relax2<K>(l2, h, P.kappa_log2, P.inv_tau, q, sm);
+      relax2<K>(l2, h, P.kappa_log2, P.inv_tau, qv, sm);
       const float2 wt = add2(sm.qm, sm.delta);
       const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
       const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
@@ -408,7 +465,7 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
 #pragma unroll
       for (int k = 0; k < K; ++k) {
         // dL/dl_k = (kappa/tau) G s p_k (q_k - w~)   (softmax Jacobian, App. B)
-        const float2 dk = add2(add2(f2(q[k]), neg2(sm.qm)), neg2(sm.delta));
+        const float2 dk = add2(add2(qv[k], neg2(sm.qm)), neg2(sm.delta));
         const float2 dl = mul2(A, mul2(sm.p[k], dk));
         if (kExport) {
           m[k][2 * pr] = dl.x;
@@ -466,8 +523,10 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
           float2 l2[K], h[K];
 #pragma unroll
           for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
+          const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
+                                      (j4 >> (16 * pr + 8)) & 0xFFu);
           draw_noise2<K>(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
-          const float2 wt = soft_value2<K>(l2, h, P.kappa_log2_next, P.inv_tau_next, q);
+          const float2 wt = soft_value2<K>(l2, h, P.kappa_log2_next, P.inv_tau_next, qv);
           const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
           d[2 * pr] = dd.x;
           d[2 * pr + 1] = dd.y;
@@ -522,13 +581,26 @@ __device__ __forceinline__ InitConsts init_consts(const InitParams& P) {
   return c;
 }
 
+// Logits of a quad: init_bias on the RTN level (or, with local shift, on the
+// delta = 0 logit, with the RTN index stored as j0); momenta 0.
 __device__ __forceinline__ void write_init_quad(const InitParams& P, int64_t qi, const int (&code)[4]) {
-  for (int k = 0; k < P.K; ++k) {
+  if (P.j0) {
+    reinterpret_cast<uint32_t*>(P.j0)[qi] =
+        static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
+        (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
+  }
+  const int logits = P.j0 ? 5 : P.K;
+  for (int k = 0; k < logits; ++k) {
     float4 v;
-    v.x = code[0] == k ? P.init_bias : 0.0f;
-    v.y = code[1] == k ? P.init_bias : 0.0f;
-    v.z = code[2] == k ? P.init_bias : 0.0f;
-    v.w = code[3] == k ? P.init_bias : 0.0f;
+    if (P.j0) {
+      const float b = k == 2 ? P.init_bias : 0.0f;
+      v = make_float4(b, b, b, b);
+    } else {
+      v.x = code[0] == k ? P.init_bias : 0.0f;
+      v.y = code[1] == k ? P.init_bias : 0.0f;
+      v.z = code[2] == k ? P.init_bias : 0.0f;
+      v.w = code[3] == k ? P.init_bias : 0.0f;
+    }
     reinterpret_cast<float4*>(P.logits + k * P.n)[qi] = v;
     reinterpret_cast<float4*>(P.m_logits + k * P.n)[qi] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
@@ -647,6 +719,11 @@ __device__ __forceinline__ void argmax_margin(const float* logits, int64_t n, in
   margin = best - second;
 }
 
+// Grid code of logit index k: k itself, or clip(j0 + k - 2) with local shift.
+__device__ __forceinline__ int grid_code(int k, const uint8_t* j0, int64_t i, int nlev) {
+  return j0 ? min(max(static_cast<int>(j0[i]) + k - 2, 0), nlev - 1) : k;
+}
+
 __global__ void __launch_bounds__(kEwThreads) k_project(const ProjectParams P) {
   const int64_t nq = P.n >> 2;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -673,6 +750,12 @@ __global__ void __launch_bounds__(kEwThreads) k_project(const ProjectParams P) {
         }
       }
     }
+    if (P.j0) {
+      const uint32_t j4 = reinterpret_cast<const uint32_t*>(P.j0)[qi];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        code[j] = min(max(static_cast<int>((j4 >> (8 * j)) & 0xFFu) + code[j] - 2, 0), P.nlev - 1);
+    }
     if (P.codes) {
       const uint32_t packed = static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
                               (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
@@ -697,7 +780,7 @@ __device__ __forceinline__ uint32_t stream_word(uint32_t code, int bits, int lan
 
 __global__ void __launch_bounds__(kEwThreads) k_pack_group(const PackParams P) {
   const int lane = threadIdx.x & 31;
-  const int bits = P.K <= 4 ? 2 : 3;
+  const int bits = P.nlev <= 4 ? 2 : 3;
   const int64_t nchunks = (P.n + 31) / 32;
   const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
   uint32_t* words = reinterpret_cast<uint32_t*>(P.out);
@@ -709,7 +792,7 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_group(const PackParams P) {
       int c;
       float mg;
       argmax_margin(P.logits, P.n, P.K, i, c, mg);
-      code = static_cast<uint32_t>(c);
+      code = static_cast<uint32_t>(grid_code(c, P.j0, i, P.nlev));
     }
     for (int wd = 0; wd < bits; ++wd) {
       const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(code, bits, lane, wd));
@@ -739,7 +822,9 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
     for (int ch = 0; ch < 8; ++ch) {
       int c;
       float mg;
-      argmax_margin(P.logits, P.n, P.K, sb * kSuperBlock + ch * 32 + lane, c, mg);
+      const int64_t wi = sb * kSuperBlock + ch * 32 + lane;
+      argmax_margin(P.logits, P.n, P.K, wi, c, mg);
+      c = grid_code(c, P.j0, wi, P.nlev);
       for (int wd = 0; wd < 3; ++wd) {
         const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(static_cast<uint32_t>(c), 3, lane, wd));
         if (lane == wd) rec[wib][ch * 3 + wd] = v;
@@ -760,11 +845,11 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
   }
 }
 
-template <int K>
+template <int K, bool kShift>
 void set_max_smem_carveout() {
-  cudaFuncSetAttribute(k_forward<K>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
-  cudaFuncSetAttribute(k_backward<K, false>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
-  cudaFuncSetAttribute(k_backward<K, true>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_forward<K, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_backward<K, false, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_backward<K, true, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
 }
 
 int grid_for(const void* fn, int num_sms, int threads) {
@@ -789,38 +874,57 @@ int grid_for(const void* fn, int num_sms, int threads) {
     default: return cudaErrorInvalidValue;          \
   }
 
-int ew_grid_size(int K, int which, int num_sms) {
+// Local shift always has 5 logits per weight; it is instantiated for K = 5 only.
+int ew_grid_size(int K, int which, int num_sms, bool shift) {
   int g = num_sms;
-  auto pick = [&](auto kk) {
+  auto pick = [&](auto kk, auto sh) {
     constexpr int KK = decltype(kk)::value;
-    set_max_smem_carveout<KK>();
-    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<KK>), num_sms, kEwThreads)
-                   : grid_for(reinterpret_cast<const void*>(k_backward<KK, false>), num_sms, kEwThreads);
+    constexpr bool SH = decltype(sh)::value;
+    set_max_smem_carveout<KK, SH>();
+    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<KK, SH>), num_sms, kEwThreads)
+                   : grid_for(reinterpret_cast<const void*>(k_backward<KK, false, SH>), num_sms,
+                              kEwThreads);
   };
+  using F = std::false_type;
+  if (shift) {
+    if (K == 5) pick(std::integral_constant<int, 5>{}, std::true_type{});
+    return g;
+  }
   switch (K) {
-    case 2: pick(std::integral_constant<int, 2>{}); break;
-    case 3: pick(std::integral_constant<int, 3>{}); break;
-    case 4: pick(std::integral_constant<int, 4>{}); break;
-    case 5: pick(std::integral_constant<int, 5>{}); break;
-    case 6: pick(std::integral_constant<int, 6>{}); break;
-    case 7: pick(std::integral_constant<int, 7>{}); break;
-    case 8: pick(std::integral_constant<int, 8>{}); break;
+    case 2: pick(std::integral_constant<int, 2>{}, F{}); break;
+    case 3: pick(std::integral_constant<int, 3>{}, F{}); break;
+    case 4: pick(std::integral_constant<int, 4>{}, F{}); break;
+    case 5: pick(std::integral_constant<int, 5>{}, F{}); break;
+    case 6: pick(std::integral_constant<int, 6>{}, F{}); break;
+    case 7: pick(std::integral_constant<int, 7>{}, F{}); break;
+    case 8: pick(std::integral_constant<int, 8>{}, F{}); break;
     default: break;
   }
   return g;
 }
 
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s) {
-  GSQ_DISPATCH_K(p.K, (k_forward<KK><<<grid, kEwThreads, 0, s>>>(p)));
+  if (p.j0) {
+    if (p.K != 5) return cudaErrorInvalidValue;
+    k_forward<5, true><<<grid, kEwThreads, 0, s>>>(p);
+  } else {
+    GSQ_DISPATCH_K(p.K, (k_forward<KK, false><<<grid, kEwThreads, 0, s>>>(p)));
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
   const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
-  if (export_mode) {
-    GSQ_DISPATCH_K(p.K, (k_backward<KK, true><<<grid, kEwThreads, 0, s>>>(p)));
+  if (p.j0) {
+    if (p.K != 5) return cudaErrorInvalidValue;
+    if (export_mode)
+      k_backward<5, true, true><<<grid, kEwThreads, 0, s>>>(p);
+    else
+      k_backward<5, false, true><<<grid, kEwThreads, 0, s>>>(p);
+  } else if (export_mode) {
+    GSQ_DISPATCH_K(p.K, (k_backward<KK, true, false><<<grid, kEwThreads, 0, s>>>(p)));
   } else {
-    GSQ_DISPATCH_K(p.K, (k_backward<KK, false><<<grid, kEwThreads, 0, s>>>(p)));
+    GSQ_DISPATCH_K(p.K, (k_backward<KK, false, false><<<grid, kEwThreads, 0, s>>>(p)));
   }
   return cudaGetLastError();
 }

@@ -32,7 +32,9 @@ struct EwParams {
   // shape
   int64_t n;          // E*R*C weights
   int64_t nq;         // n / 4 quads
-  int K;
+  int K;              // logits per weight: grid levels, or 5 shifts (local shift)
+  int nlev;           // grid levels
+  const uint8_t* j0;  // local shift: initial grid index per weight [n]; null otherwise
   int group;          // scale group (16 for K-Quant)
   int log2_group;
   int w_bf16;         // W storage: 1 bf16, 0 fp32
@@ -75,11 +77,12 @@ gsq_status set_last_error(gsq_status st, const char* msg);
 // ---- launchers (gsq_elementwise.cu) ----------------------------------------
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
-int ew_grid_size(int K, int which, int num_sms);  // which: 0 forward, 1 backward
+int ew_grid_size(int K, int which, int num_sms, bool shift);  // which: 0 forward, 1 backward
 
 struct InitParams {
   int64_t n;
-  int K;
+  int K;               // grid levels
+  uint8_t* j0;         // local shift: receives the RTN index; logits then hold 5 planes
   int group;
   int kquant;
   int w_bf16;
@@ -99,7 +102,9 @@ cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16,
 
 struct ProjectParams {
   int64_t n;
-  int K;
+  int K;               // logits per weight
+  int nlev;            // grid levels
+  const uint8_t* j0;   // local shift (null otherwise): code = clip(j0 + argmax - 2)
   const float* logits;
   uint8_t* codes;
   float* margin;
@@ -108,7 +113,9 @@ cudaError_t launch_project(const ProjectParams& p, int num_sms, cudaStream_t s);
 
 struct PackParams {
   int64_t n;
-  int K;
+  int K;               // logits per weight
+  int nlev;            // grid levels (code width)
+  const uint8_t* j0;   // local shift (null otherwise)
   int group;
   int kquant;
   const float* logits;

@@ -99,6 +99,7 @@ extern "C" GSQ_API gsq_status gsq_backward_update_noalloc(const gsq_backward_arg
   p.n = n;
   p.nq = n / 4;
   p.K = a->num_levels;
+  p.nlev = a->num_levels;
   p.group = g;
   int lg = 0;
   while ((1 << lg) < g) ++lg;

@@ -29,8 +29,9 @@ GSQ_CALIB_H, GSQ_CALIB_X = 0, 1
 GSQ_SCALE_GROUP, GSQ_SCALE_KQUANT2 = 0, 1
 GSQ_GEMM_BF16, GSQ_GEMM_F32 = 0, 1
 GSQ_FLAG_NO_NOISE = 1
+GSQ_PARAM_FULL, GSQ_PARAM_SHIFT5 = 0, 1
 (GSQ_T_LOGITS, GSQ_T_SCALES, GSQ_T_MOM_LOGITS, GSQ_T_MOM_SCALES, GSQ_T_D, GSQ_T_G, GSQ_T_W,
- GSQ_T_H, GSQ_T_KQ_D, GSQ_T_KQ_SC) = range(10)
+ GSQ_T_H, GSQ_T_KQ_D, GSQ_T_KQ_SC, GSQ_T_J0) = range(11)
 (GSQ_K_FORWARD, GSQ_K_GEMM, GSQ_K_BACKWARD, GSQ_K_PROJECT, GSQ_K_PACK, GSQ_K_INIT) = range(6)
 GSQ_K_COUNT = 6
 KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init"]
@@ -49,7 +50,7 @@ class gsq_layer_desc(Structure):
         ("group_size", c_int32), ("scale_mode", c_int32), ("init_bias", c_float),
         ("flags", c_uint32), ("seed", c_uint64), ("lr_logits", c_float), ("lr_scales", c_float),
         ("beta1", c_float), ("beta2", c_float), ("wd_logits", c_float), ("wd_scales", c_float),
-        ("gemm_precision", c_int32), ("reserved", c_int32),
+        ("gemm_precision", c_int32), ("param_mode", c_int32),
     ]
 
 
@@ -209,7 +210,7 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
               init_bias: float = 2.0, seed: int = 0, lr_logits: float = 1e-4,
               lr_scales: float = 5e-5, beta1: float = 0.9, beta2: float = 0.95,
               wd_logits: float = 1.0, wd_scales: float = 0.0, gemm: int = GSQ_GEMM_BF16,
-              noise: bool = True) -> gsq_layer_desc:
+              noise: bool = True, param_mode: int = GSQ_PARAM_FULL) -> gsq_layer_desc:
     d = gsq_layer_desc()
     d.num_experts, d.out_features, d.in_features = experts, rows, cols
     d.w_dtype = w_dtype
@@ -228,6 +229,7 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
     d.beta1, d.beta2 = beta1, beta2
     d.wd_logits, d.wd_scales = wd_logits, wd_scales
     d.gemm_precision = gemm
+    d.param_mode = param_mode
     return d
 
 
@@ -238,7 +240,8 @@ class Layer:
     (CUDA).  The workspace is a torch uint8 tensor owned by this object."""
 
     def __init__(self, W, calib, grid: Sequence[float], group_size: int, *, calib_kind: str = "H",
-                 scale_mode: str = "group", gemm: str = "bf16", stream=None, **hyper):
+                 scale_mode: str = "group", gemm: str = "bf16", param: str = "full", stream=None,
+                 **hyper):
         import torch
         self._torch = torch
         assert W.is_cuda and calib.is_cuda and W.dim() == 3 and calib.dim() == 3
@@ -247,6 +250,7 @@ class Layer:
         E, R, C = W.shape
         self.shape = (E, R, C)
         self.K = len(grid)
+        self.L = 5 if param == "shift5" else self.K   # logits per weight
         self.group_size = group_size
         self.desc = make_desc(
             experts=E, rows=R, cols=C, grid=grid, group_size=group_size,
@@ -255,7 +259,8 @@ class Layer:
             calib_kind=GSQ_CALIB_X if calib_kind == "X" else GSQ_CALIB_H,
             n_tokens=calib.shape[1] if calib_kind == "X" else 0,
             scale_mode=GSQ_SCALE_KQUANT2 if scale_mode == "kquant2" else GSQ_SCALE_GROUP,
-            gemm=GSQ_GEMM_F32 if gemm == "f32" else GSQ_GEMM_BF16, **hyper)
+            gemm=GSQ_GEMM_F32 if gemm == "f32" else GSQ_GEMM_BF16,
+            param_mode=GSQ_PARAM_SHIFT5 if param == "shift5" else GSQ_PARAM_FULL, **hyper)
         if W.dtype not in (torch.float32, torch.bfloat16):
             raise TypeError("W must be fp32 or bf16")
         nbytes = gsq_workspace_size(self.desc)

@@ -67,7 +67,7 @@ def assert_gemm_bound(G, D, H, what="", alpha=2.0):
     return worst
 
 
-def grad_bounds(ref, prob, tol):
+def grad_bounds(ref, prob, tol, q=None):
     """Elementwise bounds for the logit and scale gradients when the only
     reduced-precision input is G (the bf16 tensor-core GEMM): both gradients
     are linear in G,
@@ -76,7 +76,8 @@ def grad_bounds(ref, prob, tol):
     G = ref.G
     gscale = tol * (np.abs(G) + np.sqrt(np.mean(G * G)))
     fw = ref.fw
-    q = np.asarray(prob.grid, np.float64)[:, None, None]
+    if q is None:
+        q = np.asarray(prob.grid, np.float64)[:, None, None]
     f = np.abs(fw.s[None] * fw.p * (q - fw.wtil[None]))        # |f_k| / (kappa/tau)
     bl = None
     nr, C = G.shape
@@ -84,8 +85,8 @@ def grad_bounds(ref, prob, tol):
     return f, gscale, bs
 
 
-def assert_grad_close(got_l, got_s, ref, prob, tau, kappa, tol, what=""):
-    f, gscale, bs = grad_bounds(ref, prob, tol)
+def assert_grad_close(got_l, got_s, ref, prob, tau, kappa, tol, what="", q=None):
+    f, gscale, bs = grad_bounds(ref, prob, tol, q)
     bl = (kappa / tau) * f * gscale[None] + tol * np.abs(ref.d_logits)
     err = np.abs(np.asarray(got_l, np.float64).reshape(ref.d_logits.shape) - ref.d_logits)
     bad = err > bl * 1.0001 + 1e-30
@@ -95,6 +96,38 @@ def assert_grad_close(got_l, got_s, ref, prob, tau, kappa, tol, what=""):
         err = np.abs(np.asarray(got_s, np.float64).reshape(ref.d_scales.shape) - ref.d_scales)
         bad = err > bsc * 1.0001 + 1e-30
         assert not bad.any(), (what + " dL/dscales", int(bad.sum()))
+
+
+def check_lion(gpu, orc, theta_in, c_orc, lr, flip_frac, what):
+    """Lion results agree to rounding except where the sign of the momentum mix
+    c is decided by a difference below the path's tolerance; such flips move a
+    parameter by at most 2 lr."""
+    gpu = np.asarray(gpu, np.float64).reshape(-1)
+    orc = np.asarray(orc, np.float64).reshape(-1)
+    theta_in = np.asarray(theta_in, np.float64).reshape(-1)
+    c = np.abs(np.asarray(c_orc, np.float64).reshape(-1))
+    diff = np.abs(gpu - orc)
+    # rounding is relative to the operands (theta, lr), not to a result that may
+    # cancel to ~0 (theta = lr, sign(c) = +1)
+    mag = np.maximum(np.maximum(np.abs(orc), np.abs(theta_in)), lr)
+    same = diff <= 4 * np.spacing(mag.astype(np.float32)).astype(np.float64)
+    flip = ~same
+    assert np.all(diff[flip] <= 2.0 * lr * 1.001 + 1e-7), what
+    thresh = flip_frac * np.sqrt(np.mean(c * c))
+    assert np.all(c[flip] <= thresh), (what, int(flip.sum()), float(c[flip].max()), thresh)
+    return int(flip.sum())
+
+
+def check_momentum(gpu, orc, grad_bound, b2, what):
+    """m' = b2 m + (1 - b2) g with the same m on both sides: the difference is
+    (1 - b2) times the gradient difference, so the gradient's bound carries
+    over, plus fp32 rounding of m'."""
+    gpu = np.asarray(gpu, np.float64).reshape(-1)
+    orc = np.asarray(orc, np.float64).reshape(-1)
+    bound = (1 - b2) * np.asarray(grad_bound, np.float64).reshape(-1) + \
+        2 * np.spacing(np.abs(orc).astype(np.float32)).astype(np.float64)
+    bad = np.abs(gpu - orc) > bound
+    assert not bad.any(), (what, int(bad.sum()))
 
 
 def rel_err(a, b) -> float:
@@ -120,12 +153,12 @@ class Case:
                      lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise)
         self.layer = g.Layer(self.W, self.calib, w.grid, w.group, calib_kind=w.calib,
-                             scale_mode=w.scale_mode, gemm=gemm, **hyper)
+                             scale_mode=w.scale_mode, gemm=gemm, param=w.param, **hyper)
         self.prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float),
                               group=w.group, seed=hyper["seed"], scale_mode=w.scale_mode,
                               lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1,
                               beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
-                              noise=noise)
+                              noise=noise, shift=w.param == "shift5")
         if keep_calib_host:
             host = self.calib.double().cpu().numpy()
             if w.calib == "X":
@@ -140,14 +173,14 @@ class Case:
 
     def logits(self):
         g = gsq()
-        E, R, Cc, K = self.w.experts, self.w.rows, self.w.cols, self.w.K
-        return self.tensor(g.GSQ_T_LOGITS, torch.float32).view(K, E * R, Cc).cpu().numpy()
+        E, R, Cc, L = self.w.experts, self.w.rows, self.w.cols, self.w.L
+        return self.tensor(g.GSQ_T_LOGITS, torch.float32).view(L, E * R, Cc).cpu().numpy()
 
     def state(self, rows=None) -> O.RowState:
         g = gsq()
         w = self.w
         nr = w.experts * w.rows
-        K = w.K
+        K = w.L
         f = lambda which: self.tensor(which, torch.float32).cpu().numpy()
         st = O.RowState(row_ids=np.arange(nr, dtype=np.int64), W=self.W_host.astype(np.float64),
                         logits=f(g.GSQ_T_LOGITS).reshape(K, nr, w.cols),
@@ -159,6 +192,8 @@ class Case:
             st.kq_d = O.f16_bits_to_f32(d16).reshape(nr, w.cols // 256)
             st.kq_sc = self.tensor(g.GSQ_T_KQ_SC, torch.int8).cpu().numpy().astype(np.int32).reshape(
                 nr, w.cols // 16)
+        if w.param == "shift5":
+            st.j0 = self.tensor(g.GSQ_T_J0, torch.uint8).cpu().numpy().reshape(nr, w.cols)
         return st if rows is None else st.subset(rows)
 
     def G(self):

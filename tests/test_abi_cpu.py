@@ -82,14 +82,17 @@ def test_workspace_size_formula(lib):
                           calib_kind=lib.GSQ_CALIB_X if w.calib == "X" else lib.GSQ_CALIB_H,
                           n_tokens=w.tokens if w.calib == "X" else 0,
                           scale_mode=lib.GSQ_SCALE_KQUANT2 if w.scale_mode == "kquant2" else lib.GSQ_SCALE_GROUP,
-                          lr_scales=w.lr_scales)
-        n, K = w.n, w.K
-        expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * K * n) + 2 * _align(4 * n // w.group)
+                          lr_scales=w.lr_scales,
+                          param_mode=lib.GSQ_PARAM_SHIFT5 if w.param == "shift5" else lib.GSQ_PARAM_FULL)
+        n, L = w.n, w.L
+        expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * L * n) + 2 * _align(4 * n // w.group)
         expect += _align(n * w.w_bytes()) + _align(w.experts * w.cols ** 2 * 2) + _align(2 * n) + _align(4 * n)
         if w.scale_mode == "kquant2":
             expect += _align(2 * n // 256) + _align(n // 16)
         if w.calib == "X":
             expect += _align(4 * w.experts * w.cols ** 2)
+        if w.param == "shift5":
+            expect += _align(n)                                    # j0, one byte per weight
         assert lib.gsq_workspace_size(d) == expect, w.name
     # the largest workload fits comfortably in one GB300's HBM
     big = WORKLOADS["moe64_kquant3"]

@@ -8,7 +8,7 @@ import pytest
 import torch
 
 from gpu_common import (TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound,
-                        assert_grad_close, grad_bounds, gsq)
+                        assert_grad_close, check_lion, check_momentum, grad_bounds, gsq)
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -86,38 +86,6 @@ def test_step_loss_and_gradients(name, gemm):
         assert_close(loss.cpu().numpy(), [0.5 * np.sum(D * case.G())], 1e-5, "loss = 1/2 sum D*G")
 
 
-def _check_lion(gpu, orc, theta_in, c_orc, lr, flip_frac, what):
-    """Lion results agree to rounding except where the sign of the momentum mix
-    c is decided by a difference below the path's tolerance; such flips move a
-    parameter by at most 2 lr."""
-    gpu = np.asarray(gpu, np.float64).reshape(-1)
-    orc = np.asarray(orc, np.float64).reshape(-1)
-    theta_in = np.asarray(theta_in, np.float64).reshape(-1)
-    c = np.abs(np.asarray(c_orc, np.float64).reshape(-1))
-    diff = np.abs(gpu - orc)
-    # rounding is relative to the operands (theta, lr), not to a result that may
-    # cancel to ~0 (theta = lr, sign(c) = +1)
-    mag = np.maximum(np.maximum(np.abs(orc), np.abs(theta_in)), lr)
-    same = diff <= 4 * np.spacing(mag.astype(np.float32)).astype(np.float64)
-    flip = ~same
-    assert np.all(diff[flip] <= 2.0 * lr * 1.001 + 1e-7), what
-    thresh = flip_frac * np.sqrt(np.mean(c * c))
-    assert np.all(c[flip] <= thresh), (what, int(flip.sum()), float(c[flip].max()), thresh)
-    return int(flip.sum())
-
-
-def _check_momentum(gpu, orc, grad_bound, b2, what):
-    """m' = b2 m + (1 - b2) g with the same m on both sides: the difference is
-    (1 - b2) times the gradient difference, so the gradient's bound carries
-    over, plus fp32 rounding of m'."""
-    gpu = np.asarray(gpu, np.float64).reshape(-1)
-    orc = np.asarray(orc, np.float64).reshape(-1)
-    bound = (1 - b2) * np.asarray(grad_bound, np.float64).reshape(-1) + \
-        2 * np.spacing(np.abs(orc).astype(np.float32)).astype(np.float64)
-    bad = np.abs(gpu - orc) > bound
-    assert not bad.any(), (what, int(bad.sum()))
-
-
 @pytest.mark.parametrize("gemm", ["f32", "bf16"])
 @pytest.mark.parametrize("name", list(SMALL))
 def test_step_update(name, gemm):
@@ -139,7 +107,7 @@ def test_step_update(name, gemm):
         assert_close(loss.cpu().numpy(), [res.loss], tol, f"loss t={t}")
         m0 = st_gpu_before.m_logits.astype(np.float64)
         c_l = w.beta1 * m0 + (1 - w.beta1) * res.d_logits
-        _check_lion(gpu.logits, st_sync.logits, st_gpu_before.logits, c_l, w.lr_logits, 2 * tol,
+        check_lion(gpu.logits, st_sync.logits, st_gpu_before.logits, c_l, w.lr_logits, 2 * tol,
                     "logits")
         if gemm == "f32":
             gb_l = tol * (np.abs(res.d_logits) + np.sqrt(np.mean(res.d_logits ** 2)))
@@ -149,12 +117,12 @@ def test_step_update(name, gemm):
             f, gscale, bs = grad_bounds(res, case.prob, tol)
             gb_l = (1.0 / TAU[name]) * f * gscale[None] + tol * np.abs(res.d_logits)
             gb_s = None if res.d_scales is None else bs + tol * np.abs(res.d_scales)
-        _check_momentum(gpu.m_logits, st_sync.m_logits, gb_l, w.beta2, "logit momentum")
+        check_momentum(gpu.m_logits, st_sync.m_logits, gb_l, w.beta2, "logit momentum")
         if res.d_scales is not None:
             c_s = w.beta1 * st_gpu_before.m_scales.astype(np.float64) + (1 - w.beta1) * res.d_scales
-            _check_lion(gpu.scales, st_sync.scales, st_gpu_before.scales, c_s, w.lr_scales,
+            check_lion(gpu.scales, st_sync.scales, st_gpu_before.scales, c_s, w.lr_scales,
                         2 * tol, "scales")
-            _check_momentum(gpu.m_scales, st_sync.m_scales, gb_s, w.beta2, "scale momentum")
+            check_momentum(gpu.m_scales, st_sync.m_scales, gb_s, w.beta2, "scale momentum")
         else:
             assert np.array_equal(gpu.scales, st_gpu_before.scales)
         losses.append(float(loss.item()))

@@ -34,6 +34,12 @@ What one step computes (paper references):
              level, 5 logits per weight for shifts delta in {-2..2} around the
              initial index j0; the level of shift delta is G[clip(j0 + delta)], so
              the same relaxation runs over a per-weight window of 5 levels.
+  mask x sign  (§3.1, Alg. 2): ternary weights s * m * b with a mask logit l_m
+             and a sign logit l_b per weight, each relaxed by a binary GS over
+             {0, 1} resp. {-1, 1} with the tied logits (-l, l) (§3 notation
+             paragraph: a sigmoid of the noisy logit 2l); hard rule
+             m = [l_m >= 0], b = 2 [l_b >= 0] - 1.  The grid must be {-a, 0, a};
+             w~ = a * m~ * b~.
 
 Readings where the paper is silent are listed at the top of the design notes
 (kappa multiplies the logit; summed, un-normalised loss; Philox stream; absmax
@@ -77,10 +83,20 @@ class Problem:
     wd_scales: float = 0.0
     noise: bool = True
     shift: bool = False                 # local-shift parameterisation (§3.2)
+    mask_sign: bool = False             # ternary mask x sign parameterisation (§3.1, Alg. 2)
+
+    def __post_init__(self):
+        if self.mask_sign:
+            g = np.asarray(self.grid, dtype=np.float64)
+            assert g.shape == (3,) and g[1] == 0.0 and g[0] == -g[2] and g[2] > 0, \
+                "mask x sign needs the grid {-a, 0, a}"
+            assert not self.shift
 
     @property
     def K(self) -> int:
-        """Number of logits per weight: the grid size, or 5 shifts."""
+        """Number of logits per weight: the grid size, 5 shifts, or 2 (mask, sign)."""
+        if self.mask_sign:
+            return 2
         return SHIFTS if self.shift else int(len(self.grid))
 
     @property
@@ -151,8 +167,12 @@ def soft_value(p: np.ndarray, grid: np.ndarray) -> np.ndarray:
 
 
 def noise(prob: Problem, st: RowState, t: int) -> np.ndarray:
+    """Gumbel draws [K, nr, C]; for mask x sign, one logistic draw per binary
+    instance [2, nr, C] (mask, sign), the difference of its two Gumbel draws."""
     if not prob.noise:
         return np.zeros((prob.K, len(st.row_ids), prob.C))
+    if prob.mask_sign:
+        return philox.logistic(prob.seed, t, flat_index(prob, st.row_ids), 2)
     return philox.gumbel(prob.seed, t, flat_index(prob, st.row_ids), prob.K)
 
 
@@ -180,10 +200,33 @@ class Forward:
     s: np.ndarray
     What: np.ndarray
     D: np.ndarray
+    soft: Optional[np.ndarray] = None   # mask x sign: [2, nr, C] = (m~, b~)
+
+
+BINARY_VALUES = (np.array([0.0, 1.0]), np.array([-1.0, 1.0]))   # mask {0,1}, sign {-1,1}
+
+
+def binary_gs(l, lam, values, tau: float, kappa: float):
+    """One binary GS instance of Alg. 2: Alg. 1 over the two values with the
+    tied logits (-l, l) (§3 notation paragraph) and the noise pair (0, lam),
+    lam being the difference of the pair's two Gumbel draws (only the
+    difference enters the softmax).  Returns (p [2, ...], soft value)."""
+    l = np.asarray(l, dtype=np.float64)
+    p = relax(np.stack([-l, l]), np.stack([np.zeros_like(lam), lam]), tau, kappa)
+    return p, soft_value(p, values)
 
 
 def forward(prob: Problem, st: RowState, t: int, tau: float, kappa: float) -> Forward:
     g = noise(prob, st, t)
+    if prob.mask_sign:
+        a = float(prob.grid[2])
+        pm, mt = binary_gs(st.logits[0], g[0], BINARY_VALUES[0], tau, kappa)
+        pb, bt = binary_gs(st.logits[1], g[1], BINARY_VALUES[1], tau, kappa)
+        wtil = a * mt * bt                                # w~ = a m~ b~ (Alg. 2)
+        s = expand_scales(st.scales, prob.group)
+        What = s * wtil
+        return Forward(g=g, p=np.stack([pm, pb]), wtil=wtil, s=s, What=What, D=What - st.W,
+                       soft=np.stack([mt, bt]))
     p = relax(st.logits, g, tau, kappa)
     wtil = np.sum(p * level_values(prob, st), axis=0)     # w~ = sum_k p_k q_k
     s = expand_scales(st.scales, prob.group)
@@ -234,12 +277,29 @@ def loss_bruteforce(W: np.ndarray, What: np.ndarray, X: np.ndarray) -> float:
 # ----------------------------------------------------------------------------
 # backward (App. B softmax Jacobian) and Lion (§3.3, App. B)
 # ----------------------------------------------------------------------------
+def binary_gs_grad(p, soft, values, tau: float, kappa: float):
+    """d(soft value)/dl of a binary instance: the softmax Jacobian (App. B)
+    d w~/d l_k = (kappa/tau) p_k (d_k - w~), chained through the tied logits
+    l_1 = l, l_0 = -l."""
+    d0, d1 = values
+    return (kappa / tau) * (p[1] * (d1 - soft) - p[0] * (d0 - soft))
+
+
 def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float, q=None):
     """dL/dl [K, nr, C] and dL/ds [nr, C/G]; q: level values of every logit."""
+    nr, C = G.shape
+    if prob.mask_sign:
+        a = float(prob.grid[2])
+        mt, bt = fw.soft
+        gm = binary_gs_grad(fw.p[0], mt, BINARY_VALUES[0], tau, kappa)
+        gb = binary_gs_grad(fw.p[1], bt, BINARY_VALUES[1], tau, kappa)
+        Gs = G * fw.s
+        d_logits = np.stack([Gs * a * bt * gm, Gs * a * mt * gb])   # W^ = s a m~ b~
+        d_scales = (G * fw.wtil).reshape(nr, C // prob.group, prob.group).sum(axis=2)
+        return d_logits, d_scales
     if q is None:
         q = np.asarray(prob.grid, dtype=np.float64)[:, None, None]
     d_logits = (kappa / tau) * (G * fw.s)[None] * fw.p * (q - fw.wtil[None])
-    nr, C = G.shape
     d_scales = (G * fw.wtil).reshape(nr, C // prob.group, prob.group).sum(axis=2)
     return d_logits, d_scales
 
@@ -276,7 +336,8 @@ def step(prob: Problem, st: RowState, t: int, tau: float, kappa: float,
     place unless update=False; the reported loss is this step's forward loss."""
     fw = forward(prob, st, t, tau, kappa)
     L, G = loss_and_grad(prob, st.row_ids, fw.D)
-    d_logits, d_scales = backward(prob, fw, G, tau, kappa, q=level_values(prob, st))
+    q = None if prob.mask_sign else level_values(prob, st)
+    d_logits, d_scales = backward(prob, fw, G, tau, kappa, q=q)
     if scales_frozen(prob):
         d_scales = None
     if update:
@@ -384,7 +445,13 @@ def init_state(prob: Problem, W, row_ids, init_bias: float = 2.0) -> RowState:
     codes = rtn_codes(W32, np.repeat(s, prob.group, axis=1), prob.grid)
     logits = np.zeros((prob.K, nr, C), dtype=np.float32)
     j0 = None
-    if prob.shift:
+    if prob.mask_sign:
+        # Eq. 3 with the RTN code in place of the GPTQ one, scaled by init_bias:
+        # l_m = +1 if the code is nonzero else -1; l_b = sign of the code (0 for 0)
+        b = np.float32(init_bias)
+        logits[0] = np.where(codes != 1, b, -b)
+        logits[1] = np.where(codes == 2, b, np.where(codes == 0, -b, np.float32(0.0)))
+    elif prob.shift:
         logits[2] = np.float32(init_bias)             # delta = 0: stay on the RTN level
         j0 = codes.astype(np.uint8)
     else:
@@ -399,9 +466,25 @@ def init_state(prob: Problem, W, row_ids, init_bias: float = 2.0) -> RowState:
 # ----------------------------------------------------------------------------
 # hard projection (Alg. 2, final lines, generalised to K levels)
 # ----------------------------------------------------------------------------
-def project(logits32: np.ndarray, j0=None, levels: int = 0):
+def project_mask_sign(logits32: np.ndarray):
+    """Alg. 2, final lines: m = [l_m >= 0], b = 2 [l_b >= 0] - 1; grid code of
+    s * m * b on {-a, 0, a}: 0, 1 or 2.  Margin: the top-two logit gap 2|l| of
+    every instance that decides the code (the mask; the sign when m = 1)."""
+    lm, lb = logits32[0], logits32[1]
+    m = lm >= 0
+    b = lb >= 0
+    codes = np.where(m, np.where(b, 2, 0), 1).astype(np.uint8)
+    gm = 2 * np.abs(lm.astype(np.float32))
+    gb = 2 * np.abs(lb.astype(np.float32))
+    margin = np.where(m, np.minimum(gm, gb), gm).astype(np.float32)
+    return codes, margin
+
+
+def project(logits32: np.ndarray, j0=None, levels: int = 0, mask_sign: bool = False):
     """k* = argmax_k l_k (lowest k on ties) and margin = l_(1) - l_(2) in fp32.
     With local shift the grid code is clip(j0 + k* - 2) (§3.2)."""
+    if mask_sign:
+        return project_mask_sign(logits32)
     k = np.argmax(logits32, axis=0)
     srt = np.sort(logits32, axis=0)
     margin = (srt[-1] - srt[-2]).astype(np.float32)

@@ -16,6 +16,11 @@ Stream layout (a reading; the paper is silent):
   grid level; level k takes 32-bit word (k mod 4) of that block.
   u = ((x mod 2^23) + 1/2) * 2^-23     (low 23 bits; exactly representable in fp32, in (0,1))
   g = -ln(-ln(u))                       (inverse-CDF of Gumbel(0, 1)), in fp64.
+
+Binary instances (the ternary mask x sign variant, Alg. 2) need only the
+difference of their two Gumbel draws, which is Logistic(0, 1); it is drawn
+directly by its inverse CDF from one word: lambda = ln(u) - ln(1 - u), with
+instance k taking word k of block 0.
 """
 from __future__ import annotations
 
@@ -75,3 +80,11 @@ def gumbel(seed: int, t: int, flat_index, K: int) -> np.ndarray:
     every step t (§3.3).  fp64."""
     u = uniform_from_word(level_words(seed, t, flat_index, K))
     return -np.log(-np.log(u))
+
+
+def logistic(seed: int, t: int, flat_index, n: int) -> np.ndarray:
+    """lam[k, ...] ~ Logistic(0, 1), the law of g1 - g0 for two independent
+    Gumbel(0, 1) draws: one per binary instance k < n and weight, fresh for
+    every step t.  Inverse CDF: lam = ln(u / (1 - u)).  fp64."""
+    u = uniform_from_word(level_words(seed, t, flat_index, n))
+    return np.log(u) - np.log1p(-u)

@@ -191,7 +191,8 @@ def _oracle_problem(w, H_host, rows):
     prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float), group=w.group,
                      seed=w.seed, scale_mode=w.scale_mode, H=H_host, lr_logits=w.lr_logits,
                      lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2, wd_logits=w.wd_logits,
-                     wd_scales=w.wd_scales, shift=w.param == "shift5")
+                     wd_scales=w.wd_scales, shift=w.param == "shift5",
+                     mask_sign=w.param == "mask_sign")
     return prob
 
 

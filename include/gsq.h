@@ -72,7 +72,7 @@ enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1 };
 enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
 enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
 enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel draw */
-enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1 };
+enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1, GSQ_PARAM_MASK_SIGN = 2 };
 
 /* Layer problem (Eq. 1 with a linear f; §3.2; §4.1; Table 5 for the defaults).
  *
@@ -103,6 +103,13 @@ enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1 };
  *              (round-to-nearest) index j0; shift delta uses level
  *              grid[clip(j0 + delta, 0, K - 1)].  The projection gives the code
  *              clip(j0 + argmax - 2).  Logit tensors then hold 5 planes.
+ *              GSQ_PARAM_MASK_SIGN: ternary mask x sign (§3.1, Alg. 2): the grid
+ *              must be {-a, 0, a} (a > 0); two logits per weight, plane 0 the
+ *              mask l_m and plane 1 the sign l_b, each relaxed by a binary GS
+ *              with tied logits (-l, l); W^ = s a m~ b~.  Init: Eq. 3 applied to
+ *              the round-to-nearest code, times init_bias.  Projection:
+ *              m = [l_m >= 0], b = 2 [l_b >= 0] - 1; code 0, 1, 2 for -a, 0, a;
+ *              margin = 2|l_m|, or min(2|l_m|, 2|l_b|) when m = 1.
  * Limits: 1 <= E, 1 <= R, 8 <= C, C % 8 == 0, E*R*C < 2^40, 2 <= K <= 8.
  */
 typedef struct gsq_layer_desc {

@@ -52,7 +52,8 @@ class Workload:
     wd_scales: float = 0.0
     data_seed: int = 0
     pack: bool = False
-    param: str = "full"        # "full": one logit per level; "shift5": local shift (§3.2)
+    param: str = "full"        # "full": one logit per level; "shift5": local shift (§3.2);
+    #                            "mask_sign": ternary mask x sign (§3.1, Alg. 2)
 
     @property
     def K(self) -> int:
@@ -60,8 +61,8 @@ class Workload:
 
     @property
     def L(self) -> int:
-        """Logits per weight: K, or 5 shifts around the initial index."""
-        return 5 if self.param == "shift5" else self.K
+        """Logits per weight: K, 5 shifts around the initial index, or (mask, sign)."""
+        return {"shift5": 5, "mask_sign": 2}.get(self.param, self.K)
 
     @property
     def n(self) -> int:
@@ -114,6 +115,12 @@ WORKLOADS = {
                  grid=GRID_3BIT_SYM, group=128, w_dtype="bf16", calib="H", tokens=256 * 2048,
                  token_dist="student_t3", outliers=0, outlier_scale=1.0, steps=200, tau0=0.5,
                  tau1=0.5, data_seed=3000, param="shift5"),
+        # The paper's ternary method (§3.1, Alg. 2) on the q_proj layer: mask and sign
+        # logits per weight, grid {-1, 0, 1}.
+        Workload(name="llama8b_q_proj_mask_sign", experts=1, rows=4096, cols=4096,
+                 grid=GRID_TERNARY, group=128, w_dtype="bf16", calib="H", tokens=128 * 2048,
+                 token_dist="normal", outliers=41, outlier_scale=30.0, steps=500, tau0=1.0,
+                 tau1=0.1, data_seed=2000, param="mask_sign"),
     ]
 }
 

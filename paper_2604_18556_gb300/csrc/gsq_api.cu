@@ -86,8 +86,9 @@ struct Layout {
 struct Shape {
   int64_t E, R, C, n, ng;
   int K, group;
-  int L;  // logits per weight: K, or 5 with local shift
-  bool kquant, d_bf16, w_bf16, x_mode, shift;
+  int L;     // logits per weight: K, 5 with local shift, 2 with mask x sign
+  int mode;  // GSQ_PARAM_*
+  bool kquant, d_bf16, w_bf16, x_mode, shift, mask_sign;
 };
 
 Shape shape_of(const gsq_layer_desc& d) {
@@ -103,8 +104,10 @@ Shape shape_of(const gsq_layer_desc& d) {
   s.d_bf16 = d.gemm_precision == GSQ_GEMM_BF16;
   s.w_bf16 = d.w_dtype == GSQ_DTYPE_BF16;
   s.x_mode = d.calib_kind == GSQ_CALIB_X;
+  s.mode = d.param_mode;
   s.shift = d.param_mode == GSQ_PARAM_SHIFT5;
-  s.L = s.shift ? 5 : s.K;
+  s.mask_sign = d.param_mode == GSQ_PARAM_MASK_SIGN;
+  s.L = s.shift ? 5 : (s.mask_sign ? 2 : s.K);
   return s;
 }
 
@@ -178,8 +181,12 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
     return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
   if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE))
     return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
-  if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5)
+  if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5 &&
+      d->param_mode != GSQ_PARAM_MASK_SIGN)
     return fail(GSQ_ERR_INVALID_ARG, "bad param_mode %d", d->param_mode);
+  if (d->param_mode == GSQ_PARAM_MASK_SIGN &&
+      !(d->num_levels == 3 && d->grid[1] == 0.f && d->grid[0] == -d->grid[2]))
+    return fail(GSQ_ERR_INVALID_ARG, "GSQ_PARAM_MASK_SIGN needs the grid {-a, 0, a}");
   const float hp[] = {d->init_bias, d->lr_logits, d->lr_scales, d->beta1, d->beta2, d->wd_logits, d->wd_scales};
   for (float v : hp)
     if (!std::isfinite(v)) return fail(GSQ_ERR_INVALID_ARG, "non-finite hyper-parameter");
@@ -262,6 +269,7 @@ EwParams base_params(gsq_layer* L) {
   p.nq = s.n / 4;
   p.K = s.L;
   p.nlev = s.K;
+  p.mode = s.mode;
   p.j0 = s.shift ? L->ws + L->lay.j0 : nullptr;
   p.group = s.group;
   int lg = 0;
@@ -497,8 +505,8 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if (v > kMaxPartials) v = kMaxPartials;
     return static_cast<int>(v < 1 ? 1 : v);
   };
-  L->grid_fwd = clamp_grid(ew_grid_size(sh.L, 0, L->num_sms, sh.shift));
-  L->grid_bwd = clamp_grid(ew_grid_size(sh.L, 1, L->num_sms, sh.shift));
+  L->grid_fwd = clamp_grid(ew_grid_size(sh.L, 0, L->num_sms, sh.mode));
+  L->grid_bwd = clamp_grid(ew_grid_size(sh.L, 1, L->num_sms, sh.mode));
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
                              L->num_sms);
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128 or 256: override the choice
@@ -569,6 +577,7 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   ip.kq_d = sh.kquant ? reinterpret_cast<uint16_t*>(L->ws + lay.kq_d) : nullptr;
   ip.kq_sc = sh.kquant ? reinterpret_cast<int8_t*>(L->ws + lay.kq_sc) : nullptr;
   ip.j0 = sh.shift ? L->ws + lay.j0 : nullptr;
+  ip.mask_sign = sh.mask_sign;
   if ((e = launch_init_state(ip, L->num_sms, s)) != cudaSuccess) return bail(cuda_fail(e, "init state"));
   prof_end(L, slot, s);
 
@@ -656,6 +665,7 @@ gsq_status gsq_project(gsq_layer* L, void* stream, uint8_t* codes_dev, float* ma
   p.n = L->shape.n;
   p.K = L->shape.L;
   p.nlev = L->shape.K;
+  p.mask_sign = L->shape.mask_sign;
   p.j0 = L->shape.shift ? L->ws + L->lay.j0 : nullptr;
   p.logits = fptr(L, L->lay.logits);
   p.codes = codes_dev;
@@ -688,6 +698,7 @@ gsq_status gsq_pack(gsq_layer* L, void* stream, void* out_dev, size_t cap, size_
   p.n = L->shape.n;
   p.K = L->shape.L;
   p.nlev = L->shape.K;
+  p.mask_sign = L->shape.mask_sign;
   p.j0 = L->shape.shift ? L->ws + L->lay.j0 : nullptr;
   p.group = L->shape.group;
   p.kquant = L->shape.kquant;

@@ -341,11 +341,132 @@ __device__ __forceinline__ void reduce_loss(float acc, const EwParams& P) {
 }
 
 // ---------------------------------------------------------------------------
+// Relaxation policies: how a pair of weights' logits and noise become their
+// soft values w~ and how dw~/dl flows back.  One fused kernel skeleton serves
+// all of them.
+//   L             logits per weight (planes of the logit tensors)
+//   noise(...)    the step's draws for the pair, in log2 units
+//   relax(...)    w~ of the pair; keeps what dsoft() needs
+//   dsoft(k)      dw~/dl_k divided by kappa/tau
+//   value(...)    w~ only (forward)
+// ---------------------------------------------------------------------------
+// Categorical GS over the K grid levels (Alg. 1), or over 5 local shifts.
+template <int K, bool kShift>
+struct CatRelax {
+  static constexpr int L = K;
+  Levels2<K, kShift> qv;
+  Soft2<K> sm;
+  __device__ __forceinline__ CatRelax(const float (&q)[kMaxLevels], const float* sgrid, int nlev,
+                                      uint32_t ja, uint32_t jb)
+      : qv(q, sgrid, nlev, ja, jb) {}
+  __device__ static __forceinline__ void noise(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
+                                               int on, float2 (&h)[L]) {
+    draw_noise2<K>(keys, t, i0, on, h);
+  }
+  __device__ __forceinline__ float2 relax(const float2 (&l)[L], const float2 (&h)[L],
+                                          float kappa_log2, float inv_tau) {
+    relax2<K>(l, h, kappa_log2, inv_tau, qv, sm);
+    return add2(sm.qm, sm.delta);
+  }
+  // softmax Jacobian (App. B): dw~/dl_k = (kappa/tau) p_k (q_k - w~)
+  __device__ __forceinline__ float2 dsoft(int k) const {
+    return mul2(sm.p[k], add2(add2(qv[k], neg2(sm.qm)), neg2(sm.delta)));
+  }
+  __device__ __forceinline__ float2 value(const float2 (&l)[L], const float2 (&h)[L],
+                                          float kappa_log2, float inv_tau) const {
+    return soft_value2<K>(l, h, kappa_log2, inv_tau, qv);
+  }
+};
+
+// Logistic(0, 1) draws in log2 units, log2(u / (1 - u)), for weights i0 and
+// i0 + 1: the mask instance takes word 0 and the sign instance word 1 of the
+// weight's first Philox block.  A binary GS over tied logits (-l, l) sees only
+// the difference g1 - g0 of its two Gumbel draws, whose law this is.  u and
+// 1 - u are both exact: the complemented 23 bits give 1 - u.
+__device__ __forceinline__ void draw_logistic2(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
+                                               int on, float2 (&h)[2]) {
+  if (!on) {
+    h[0] = h[1] = f2(0.0f);
+    return;
+  }
+  const uint32_t lo = static_cast<uint32_t>(i0), hi = static_cast<uint32_t>(i0 >> 32);
+  const uint4 a = philox4x32_10(lo, hi, t, 0u, keys);
+  const uint4 b = philox4x32_10(lo + 1u, hi, t, 0u, keys);
+  const float half = __uint_as_float(0x3F7FFFFFu);  // 1 - 2^-24
+  auto unit = [&](uint32_t x) { return __uint_as_float(0x3F800000u | (x & 0x007FFFFFu)) - half; };
+  // ratio u / (1 - u) of the mask (x) and sign (y) draws, for each weight
+  const float2 ua = make_float2(unit(a.x), unit(a.y)), va = make_float2(unit(~a.x), unit(~a.y));
+  const float2 ub = make_float2(unit(b.x), unit(b.y)), vb = make_float2(unit(~b.x), unit(~b.y));
+  const float2 ra = mul2(ua, rcp2(va)), rb = mul2(ub, rcp2(vb));
+  const float2 la = log2_unit2(ra), lb = log2_unit2(rb);  // (mask, sign) of each weight
+  h[0] = make_float2(la.x, lb.x);
+  h[1] = make_float2(la.y, lb.y);
+}
+
+// Ternary mask x sign (§3.1, Alg. 2): w~ = a m~ b~ on the grid {-a, 0, a}, with
+// m~ = GS({0,1}, (-l_m, l_m)) and b~ = GS({-1,1}, (-l_b, l_b)); each binary GS
+// is a sigmoid of the noisy logit 2l (§3 notation paragraph):
+//   y = (2 kappa log2(e) l + log2(u/(1-u))) / tau,  p1 = 1 / (1 + 2^-y).
+// With e = 2^-|y| and r = 1/(1+e): the larger of p0, p1 is r, the smaller e r
+// (no overflow for any y), p0 p1 = e r^2, p1 - p0 = sign(y) (1 - e) r.
+// dm~/dl_m = 2 (kappa/tau) p0 p1, db~/dl_b = 4 (kappa/tau) p0 p1.
+struct MaskSignRelax {
+  static constexpr int L = 2;
+  float a;
+  float2 mt, bt, gm, gb;
+  __device__ __forceinline__ MaskSignRelax(const float (&q)[kMaxLevels], const float*, int, uint32_t,
+                                           uint32_t)
+      : a(q[2]) {}
+  __device__ static __forceinline__ void noise(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
+                                               int on, float2 (&h)[L]) {
+    draw_logistic2(keys, t, i0, on, h);
+  }
+  struct Bin {
+    float2 hi, lo, y;   // max(p0,p1), min(p0,p1), y
+  };
+  __device__ static __forceinline__ Bin binary(float2 l, float2 h, float kappa_log2, float inv_tau) {
+    Bin b;
+    b.y = mul2(fma2(f2(2.0f * kappa_log2), l, h), f2(inv_tau));
+    const float2 e = exp2_2(make_float2(-fabsf(b.y.x), -fabsf(b.y.y)));
+    b.hi = rcp2(add2(e, f2(1.0f)));
+    b.lo = mul2(e, b.hi);
+    return b;
+  }
+  __device__ static __forceinline__ float2 p1(const Bin& b) {
+    return make_float2(b.y.x >= 0.0f ? b.hi.x : b.lo.x, b.y.y >= 0.0f ? b.hi.y : b.lo.y);
+  }
+  __device__ static __forceinline__ float2 pm(const Bin& b) {   // p1 - p0
+    const float2 d = add2(b.hi, neg2(b.lo));
+    return make_float2(copysignf(d.x, b.y.x), copysignf(d.y, b.y.y));
+  }
+  __device__ __forceinline__ float2 relax(const float2 (&l)[L], const float2 (&h)[L],
+                                          float kappa_log2, float inv_tau) {
+    const Bin m = binary(l[0], h[0], kappa_log2, inv_tau);
+    const Bin b = binary(l[1], h[1], kappa_log2, inv_tau);
+    mt = p1(m);
+    bt = pm(b);
+    gm = mul2(f2(2.0f), mul2(m.hi, m.lo));
+    gb = mul2(f2(4.0f), mul2(b.hi, b.lo));
+    return mul2(f2(a), mul2(mt, bt));
+  }
+  __device__ __forceinline__ float2 dsoft(int k) const {
+    return k == 0 ? mul2(f2(a), mul2(bt, gm)) : mul2(f2(a), mul2(mt, gb));
+  }
+  __device__ __forceinline__ float2 value(const float2 (&l)[L], const float2 (&h)[L],
+                                          float kappa_log2, float inv_tau) const {
+    const Bin m = binary(l[0], h[0], kappa_log2, inv_tau);
+    const Bin b = binary(l[1], h[1], kappa_log2, inv_tau);
+    return mul2(f2(a), mul2(p1(m), pm(b)));
+  }
+};
+
+// ---------------------------------------------------------------------------
 // Forward: D = s * w~ - W for step (t, tau, kappa); optional W^ export.
 // Bytes per weight: read 4K (logits) + b_W, write 2 or 4 (D).
 // ---------------------------------------------------------------------------
-template <int K, bool kShift>
+template <class Rx, bool kShift>
 __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
+  constexpr int K = Rx::L;
   float q[kMaxLevels];
   load_grid(P, q);
   __shared__ float sgrid[kMaxLevels];
@@ -373,10 +494,9 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
       float2 l2[K], h[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
-      const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
-                                  (j4 >> (16 * pr + 8)) & 0xFFu);
-      draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
-      const float2 wt = soft_value2<K>(l2, h, P.kappa_log2, P.inv_tau, qv);
+      const Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
+      Rx::noise(keys, P.t, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+      const float2 wt = rx.value(l2, h, P.kappa_log2, P.inv_tau);
       // D = s w~ - W as one rounding per weight (identical in every kernel that forms D)
       const float2 wh = mul2(f2(s), wt);
       const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
@@ -389,11 +509,11 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
 }
 
 // ---------------------------------------------------------------------------
-// Fused backward for step t: recompute the noise and p, loss partial
-// 1/2 D*G, gradients (App. B softmax Jacobian), per-group scale gradient by
+// Fused backward for step t: recompute the noise and the relaxation, loss
+// partial 1/2 D*G, logit gradients (App. B), per-group scale gradient by
 // warp shuffles, Lion in place; then (look-ahead) the forward of step t+1 from
-// the updated registers.  Bytes per weight with look-ahead: read 8K + 4 + b_W,
-// write 8K + 2 (D bf16).
+// the updated registers.  Bytes per weight with look-ahead (L logits per
+// weight): read 8L + 4 + b_W (+1 for j0), write 8L + 2 (D bf16).
 // ---------------------------------------------------------------------------
 // Blocks per SM the register budget aims for (measured best on GB300).
 template <int K>
@@ -401,8 +521,9 @@ struct BwdOcc {
   static constexpr int value = 2;
 };
 
-template <int K, bool kExport, bool kShift>
-__global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const EwParams P) {
+template <class Rx, bool kExport, bool kShift>
+__global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(const EwParams P) {
+  constexpr int K = Rx::L;
   float q[kMaxLevels];
   load_grid(P, q);
   __shared__ float sgrid[kMaxLevels];
@@ -451,12 +572,9 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
       float2 l2[K], h[K];
 #pragma unroll
       for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
-      const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
-                                  (j4 >> (16 * pr + 8)) & 0xFFu);
-      draw_noise2<K>(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
-      Soft2<K> sm;
-      relax2<K>(l2, h, P.kappa_log2, P.inv_tau, qv, sm);
-      const float2 wt = add2(sm.qm, sm.delta);
+      Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
+      Rx::noise(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
+      const float2 wt = rx.relax(l2, h, P.kappa_log2, P.inv_tau);
       const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
       const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
       loss2 = fma2(mul2(f2(0.5f), dj), Gq[pr], loss2);
@@ -464,9 +582,8 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
       const float2 A = mul2(f2(P.kappa_over_tau * s), Gq[pr]);
 #pragma unroll
       for (int k = 0; k < K; ++k) {
-        // dL/dl_k = (kappa/tau) G s p_k (q_k - w~)   (softmax Jacobian, App. B)
-        const float2 dk = add2(add2(qv[k], neg2(sm.qm)), neg2(sm.delta));
-        const float2 dl = mul2(A, mul2(sm.p[k], dk));
+        // dL/dl_k = (kappa/tau) G s dw~/dl_k
+        const float2 dl = mul2(A, rx.dsoft(k));
         if (kExport) {
           m[k][2 * pr] = dl.x;
           m[k][2 * pr + 1] = dl.y;
@@ -523,10 +640,9 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<K>::value) k_backward(const
           float2 l2[K], h[K];
 #pragma unroll
           for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
-          const Levels2<K, kShift> qv(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu,
-                                      (j4 >> (16 * pr + 8)) & 0xFFu);
-          draw_noise2<K>(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
-          const float2 wt = soft_value2<K>(l2, h, P.kappa_log2_next, P.inv_tau_next, qv);
+          const Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
+          Rx::noise(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+          const float2 wt = rx.value(l2, h, P.kappa_log2_next, P.inv_tau_next);
           const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
           d[2 * pr] = dd.x;
           d[2 * pr + 1] = dd.y;
@@ -588,6 +704,22 @@ __device__ __forceinline__ void write_init_quad(const InitParams& P, int64_t qi,
     reinterpret_cast<uint32_t*>(P.j0)[qi] =
         static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
         (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
+  }
+  if (P.mask_sign) {
+    // Eq. 3 on the RTN code (0, 1, 2 for -a, 0, a), times init_bias:
+    // l_m = +b if the code is nonzero else -b; l_b = +b, -b or 0 by its sign
+    const float b = P.init_bias;
+    float lm[4], lb[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      lm[j] = code[j] != 1 ? b : -b;
+      lb[j] = code[j] == 2 ? b : (code[j] == 0 ? -b : 0.0f);
+    }
+    reinterpret_cast<float4*>(P.logits)[qi] = make_float4(lm[0], lm[1], lm[2], lm[3]);
+    reinterpret_cast<float4*>(P.logits + P.n)[qi] = make_float4(lb[0], lb[1], lb[2], lb[3]);
+    for (int k = 0; k < 2; ++k)
+      reinterpret_cast<float4*>(P.m_logits + k * P.n)[qi] = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
   }
   const int logits = P.j0 ? 5 : P.K;
   for (int k = 0; k < logits; ++k) {
@@ -724,10 +856,46 @@ __device__ __forceinline__ int grid_code(int k, const uint8_t* j0, int64_t i, in
   return j0 ? min(max(static_cast<int>(j0[i]) + k - 2, 0), nlev - 1) : k;
 }
 
+// Mask x sign hard rule (Alg. 2): m = [l_m >= 0], b = 2 [l_b >= 0] - 1; code
+// 1 (zero) when the mask is off, else 2 or 0 by the sign.  Margin: the top-two
+// logit gap 2|l| of every instance that decides the code.
+__device__ __forceinline__ void mask_sign_code(float lm, float lb, int& code, float& margin) {
+  const bool m = lm >= 0.0f;
+  code = m ? (lb >= 0.0f ? 2 : 0) : 1;
+  margin = m ? fminf(2.0f * fabsf(lm), 2.0f * fabsf(lb)) : 2.0f * fabsf(lm);
+}
+
+// Final code and margin of weight i under any parameterisation.
+template <class P_>
+__device__ __forceinline__ void decide(const P_& P, int64_t i, int& code, float& margin) {
+  if (P.mask_sign) {
+    mask_sign_code(__ldcs(P.logits + i), __ldcs(P.logits + P.n + i), code, margin);
+    return;
+  }
+  argmax_margin(P.logits, P.n, P.K, i, code, margin);
+  code = grid_code(code, P.j0, i, P.nlev);
+}
+
 __global__ void __launch_bounds__(kEwThreads) k_project(const ProjectParams P) {
   const int64_t nq = P.n >> 2;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t qi = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; qi < nq; qi += stride) {
+    if (P.mask_sign) {
+      const float4 a = __ldcs(reinterpret_cast<const float4*>(P.logits) + qi);
+      const float4 b = __ldcs(reinterpret_cast<const float4*>(P.logits + P.n) + qi);
+      int c[4];
+      float mg[4];
+      mask_sign_code(a.x, b.x, c[0], mg[0]);
+      mask_sign_code(a.y, b.y, c[1], mg[1]);
+      mask_sign_code(a.z, b.z, c[2], mg[2]);
+      mask_sign_code(a.w, b.w, c[3], mg[3]);
+      if (P.codes)
+        reinterpret_cast<uint32_t*>(P.codes)[qi] =
+            static_cast<uint32_t>(c[0]) | (static_cast<uint32_t>(c[1]) << 8) |
+            (static_cast<uint32_t>(c[2]) << 16) | (static_cast<uint32_t>(c[3]) << 24);
+      if (P.margin) reinterpret_cast<float4*>(P.margin)[qi] = make_float4(mg[0], mg[1], mg[2], mg[3]);
+      continue;
+    }
     float best[4], second[4];
     int code[4] = {0, 0, 0, 0};
     {
@@ -791,8 +959,8 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_group(const PackParams P) {
     if (i < P.n) {
       int c;
       float mg;
-      argmax_margin(P.logits, P.n, P.K, i, c, mg);
-      code = static_cast<uint32_t>(grid_code(c, P.j0, i, P.nlev));
+      decide(P, i, c, mg);
+      code = static_cast<uint32_t>(c);
     }
     for (int wd = 0; wd < bits; ++wd) {
       const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(code, bits, lane, wd));
@@ -823,8 +991,7 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
       int c;
       float mg;
       const int64_t wi = sb * kSuperBlock + ch * 32 + lane;
-      argmax_margin(P.logits, P.n, P.K, wi, c, mg);
-      c = grid_code(c, P.j0, wi, P.nlev);
+      decide(P, wi, c, mg);
       for (int wd = 0; wd < 3; ++wd) {
         const uint32_t v = __reduce_or_sync(0xffffffffu, stream_word(static_cast<uint32_t>(c), 3, lane, wd));
         if (lane == wd) rec[wib][ch * 3 + wd] = v;
@@ -845,11 +1012,13 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
   }
 }
 
-template <int K, bool kShift>
+template <class Rx, bool kShift>
 void set_max_smem_carveout() {
-  cudaFuncSetAttribute(k_forward<K, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
-  cudaFuncSetAttribute(k_backward<K, false, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
-  cudaFuncSetAttribute(k_backward<K, true, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_forward<Rx, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+  cudaFuncSetAttribute(k_backward<Rx, false, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                       0);
+  cudaFuncSetAttribute(k_backward<Rx, true, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                       0);
 }
 
 int grid_for(const void* fn, int num_sms, int threads) {
@@ -862,71 +1031,73 @@ int grid_for(const void* fn, int num_sms, int threads) {
 
 }  // namespace
 
-#define GSQ_DISPATCH_K(K_, EXPR)                    \
-  switch (K_) {                                     \
-    case 2: { constexpr int KK = 2; EXPR; } break;  \
-    case 3: { constexpr int KK = 3; EXPR; } break;  \
-    case 4: { constexpr int KK = 4; EXPR; } break;  \
-    case 5: { constexpr int KK = 5; EXPR; } break;  \
-    case 6: { constexpr int KK = 6; EXPR; } break;  \
-    case 7: { constexpr int KK = 7; EXPR; } break;  \
-    case 8: { constexpr int KK = 8; EXPR; } break;  \
-    default: return cudaErrorInvalidValue;          \
-  }
 
-// Local shift always has 5 logits per weight; it is instantiated for K = 5 only.
-int ew_grid_size(int K, int which, int num_sms, bool shift) {
-  int g = num_sms;
-  auto pick = [&](auto kk, auto sh) {
-    constexpr int KK = decltype(kk)::value;
-    constexpr bool SH = decltype(sh)::value;
-    set_max_smem_carveout<KK, SH>();
-    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<KK, SH>), num_sms, kEwThreads)
-                   : grid_for(reinterpret_cast<const void*>(k_backward<KK, false, SH>), num_sms,
-                              kEwThreads);
-  };
-  using F = std::false_type;
-  if (shift) {
-    if (K == 5) pick(std::integral_constant<int, 5>{}, std::true_type{});
-    return g;
+template <class T>
+struct Tag {
+  using type = T;
+};
+
+// The relaxation policy of a layer: categorical over K levels, local shift
+// (K = 5 only) or mask x sign (2 logits).
+template <class F>
+cudaError_t with_relax(int K, int mode, F&& f) {
+  switch (mode) {
+    case GSQ_PARAM_SHIFT5:
+      if (K != 5) return cudaErrorInvalidValue;
+      f(Tag<CatRelax<5, true>>{}, std::true_type{});
+      return cudaSuccess;
+    case GSQ_PARAM_MASK_SIGN:
+      if (K != 2) return cudaErrorInvalidValue;
+      f(Tag<MaskSignRelax>{}, std::false_type{});
+      return cudaSuccess;
+    default:
+      break;
   }
   switch (K) {
-    case 2: pick(std::integral_constant<int, 2>{}, F{}); break;
-    case 3: pick(std::integral_constant<int, 3>{}, F{}); break;
-    case 4: pick(std::integral_constant<int, 4>{}, F{}); break;
-    case 5: pick(std::integral_constant<int, 5>{}, F{}); break;
-    case 6: pick(std::integral_constant<int, 6>{}, F{}); break;
-    case 7: pick(std::integral_constant<int, 7>{}, F{}); break;
-    case 8: pick(std::integral_constant<int, 8>{}, F{}); break;
-    default: break;
+    case 2: f(Tag<CatRelax<2, false>>{}, std::false_type{}); break;
+    case 3: f(Tag<CatRelax<3, false>>{}, std::false_type{}); break;
+    case 4: f(Tag<CatRelax<4, false>>{}, std::false_type{}); break;
+    case 5: f(Tag<CatRelax<5, false>>{}, std::false_type{}); break;
+    case 6: f(Tag<CatRelax<6, false>>{}, std::false_type{}); break;
+    case 7: f(Tag<CatRelax<7, false>>{}, std::false_type{}); break;
+    case 8: f(Tag<CatRelax<8, false>>{}, std::false_type{}); break;
+    default: return cudaErrorInvalidValue;
   }
+  return cudaSuccess;
+}
+
+int ew_grid_size(int K, int which, int num_sms, int mode) {
+  int g = num_sms;
+  with_relax(K, mode, [&](auto rx, auto sh) {
+    using Rx = typename decltype(rx)::type;
+    constexpr bool SH = decltype(sh)::value;
+    set_max_smem_carveout<Rx, SH>();
+    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<Rx, SH>), num_sms, kEwThreads)
+                   : grid_for(reinterpret_cast<const void*>(k_backward<Rx, false, SH>), num_sms,
+                              kEwThreads);
+  });
   return g;
 }
 
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s) {
-  if (p.j0) {
-    if (p.K != 5) return cudaErrorInvalidValue;
-    k_forward<5, true><<<grid, kEwThreads, 0, s>>>(p);
-  } else {
-    GSQ_DISPATCH_K(p.K, (k_forward<KK, false><<<grid, kEwThreads, 0, s>>>(p)));
-  }
-  return cudaGetLastError();
+  const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
+    using Rx = typename decltype(rx)::type;
+    k_forward<Rx, decltype(sh)::value><<<grid, kEwThreads, 0, s>>>(p);
+  });
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
   const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
-  if (p.j0) {
-    if (p.K != 5) return cudaErrorInvalidValue;
+  const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
+    using Rx = typename decltype(rx)::type;
+    constexpr bool SH = decltype(sh)::value;
     if (export_mode)
-      k_backward<5, true, true><<<grid, kEwThreads, 0, s>>>(p);
+      k_backward<Rx, true, SH><<<grid, kEwThreads, 0, s>>>(p);
     else
-      k_backward<5, false, true><<<grid, kEwThreads, 0, s>>>(p);
-  } else if (export_mode) {
-    GSQ_DISPATCH_K(p.K, (k_backward<KK, true, false><<<grid, kEwThreads, 0, s>>>(p)));
-  } else {
-    GSQ_DISPATCH_K(p.K, (k_backward<KK, false, false><<<grid, kEwThreads, 0, s>>>(p)));
-  }
-  return cudaGetLastError();
+      k_backward<Rx, false, SH><<<grid, kEwThreads, 0, s>>>(p);
+  });
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s) {

@@ -32,8 +32,9 @@ struct EwParams {
   // shape
   int64_t n;          // E*R*C weights
   int64_t nq;         // n / 4 quads
-  int K;              // logits per weight: grid levels, or 5 shifts (local shift)
+  int K;              // logits per weight: grid levels, 5 shifts, or 2 (mask, sign)
   int nlev;           // grid levels
+  int mode;           // GSQ_PARAM_FULL / GSQ_PARAM_SHIFT5 / GSQ_PARAM_MASK_SIGN
   const uint8_t* j0;  // local shift: initial grid index per weight [n]; null otherwise
   int group;          // scale group (16 for K-Quant)
   int log2_group;
@@ -77,11 +78,12 @@ gsq_status set_last_error(gsq_status st, const char* msg);
 // ---- launchers (gsq_elementwise.cu) ----------------------------------------
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
-int ew_grid_size(int K, int which, int num_sms, bool shift);  // which: 0 forward, 1 backward
+int ew_grid_size(int K, int which, int num_sms, int mode);  // which: 0 forward, 1 backward
 
 struct InitParams {
   int64_t n;
   int K;               // grid levels
+  int mask_sign;       // logits are the (mask, sign) planes, Eq. 3 from the RTN code
   uint8_t* j0;         // local shift: receives the RTN index; logits then hold 5 planes
   int group;
   int kquant;
@@ -104,6 +106,7 @@ struct ProjectParams {
   int64_t n;
   int K;               // logits per weight
   int nlev;            // grid levels
+  int mask_sign;       // code from the hard rule l >= 0 of the mask and sign logits
   const uint8_t* j0;   // local shift (null otherwise): code = clip(j0 + argmax - 2)
   const float* logits;
   uint8_t* codes;
@@ -115,6 +118,7 @@ struct PackParams {
   int64_t n;
   int K;               // logits per weight
   int nlev;            // grid levels (code width)
+  int mask_sign;       // code from the hard rule l >= 0 of the mask and sign logits
   const uint8_t* j0;   // local shift (null otherwise)
   int group;
   int kquant;

@@ -29,7 +29,8 @@ GSQ_CALIB_H, GSQ_CALIB_X = 0, 1
 GSQ_SCALE_GROUP, GSQ_SCALE_KQUANT2 = 0, 1
 GSQ_GEMM_BF16, GSQ_GEMM_F32 = 0, 1
 GSQ_FLAG_NO_NOISE = 1
-GSQ_PARAM_FULL, GSQ_PARAM_SHIFT5 = 0, 1
+GSQ_PARAM_FULL, GSQ_PARAM_SHIFT5, GSQ_PARAM_MASK_SIGN = 0, 1, 2
+PARAM_MODES = {"full": GSQ_PARAM_FULL, "shift5": GSQ_PARAM_SHIFT5, "mask_sign": GSQ_PARAM_MASK_SIGN}
 (GSQ_T_LOGITS, GSQ_T_SCALES, GSQ_T_MOM_LOGITS, GSQ_T_MOM_SCALES, GSQ_T_D, GSQ_T_G, GSQ_T_W,
  GSQ_T_H, GSQ_T_KQ_D, GSQ_T_KQ_SC, GSQ_T_J0) = range(11)
 (GSQ_K_FORWARD, GSQ_K_GEMM, GSQ_K_BACKWARD, GSQ_K_PROJECT, GSQ_K_PACK, GSQ_K_INIT) = range(6)
@@ -250,7 +251,9 @@ class Layer:
         E, R, C = W.shape
         self.shape = (E, R, C)
         self.K = len(grid)
-        self.L = 5 if param == "shift5" else self.K   # logits per weight
+        if param not in PARAM_MODES:
+            raise ValueError(f"param must be one of {sorted(PARAM_MODES)}")
+        self.L = {"full": self.K, "shift5": 5, "mask_sign": 2}[param]   # logits per weight
         self.group_size = group_size
         self.desc = make_desc(
             experts=E, rows=R, cols=C, grid=grid, group_size=group_size,
@@ -260,7 +263,7 @@ class Layer:
             n_tokens=calib.shape[1] if calib_kind == "X" else 0,
             scale_mode=GSQ_SCALE_KQUANT2 if scale_mode == "kquant2" else GSQ_SCALE_GROUP,
             gemm=GSQ_GEMM_F32 if gemm == "f32" else GSQ_GEMM_BF16,
-            param_mode=GSQ_PARAM_SHIFT5 if param == "shift5" else GSQ_PARAM_FULL, **hyper)
+            param_mode=PARAM_MODES[param], **hyper)
         if W.dtype not in (torch.float32, torch.bfloat16):
             raise TypeError("W must be fp32 or bf16")
         nbytes = gsq_workspace_size(self.desc)

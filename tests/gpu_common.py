@@ -158,7 +158,8 @@ class Case:
                               group=w.group, seed=hyper["seed"], scale_mode=w.scale_mode,
                               lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1,
                               beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
-                              noise=noise, shift=w.param == "shift5")
+                              noise=noise, shift=w.param == "shift5",
+                              mask_sign=w.param == "mask_sign")
         if keep_calib_host:
             host = self.calib.double().cpu().numpy()
             if w.calib == "X":

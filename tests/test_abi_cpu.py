@@ -83,7 +83,7 @@ def test_workspace_size_formula(lib):
                           n_tokens=w.tokens if w.calib == "X" else 0,
                           scale_mode=lib.GSQ_SCALE_KQUANT2 if w.scale_mode == "kquant2" else lib.GSQ_SCALE_GROUP,
                           lr_scales=w.lr_scales,
-                          param_mode=lib.GSQ_PARAM_SHIFT5 if w.param == "shift5" else lib.GSQ_PARAM_FULL)
+                          param_mode=lib.PARAM_MODES[w.param])
         n, L = w.n, w.L
         expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * L * n) + 2 * _align(4 * n // w.group)
         expect += _align(n * w.w_bytes()) + _align(w.experts * w.cols ** 2 * 2) + _align(2 * n) + _align(4 * n)
@@ -117,6 +117,10 @@ def test_workspace_size_formula(lib):
     (dict(calib_kind=1, n_tokens=0), 1),
     (dict(gemm=5), 1),
     (dict(beta1=1.5), 1),
+    (dict(param_mode=3), 1),                     # unknown parameterisation
+    (dict(param_mode=2), 1),                     # mask x sign needs {-a, 0, a}
+    (dict(param_mode=2, grid=(-1.0, 0.0, 2.0)), 1),
+    (dict(param_mode=2, grid=(-1.0, 0.5, 1.0)), 1),
 ])
 def test_descriptor_validation(lib, kw, status):
     d = _desc(lib, **kw)
@@ -128,6 +132,16 @@ def test_descriptor_validation(lib, kw, status):
         lib.gsq_workspace_size(d)
     assert ei.value.status == status
     assert lib.gsq_last_error()
+
+
+def test_parameterisations_size_their_logit_planes(lib):
+    """The logit tensors hold K, 5 (local shift) or 2 (mask x sign) planes."""
+    base = lib.gsq_workspace_size(_desc(lib, grid=(-1.0, 0.0, 1.0)))
+    ms = lib.gsq_workspace_size(_desc(lib, grid=(-1.0, 0.0, 1.0), param_mode=2))
+    sh = lib.gsq_workspace_size(_desc(lib, grid=(-1.0, 0.0, 1.0), param_mode=1))
+    n = 64 * 256
+    assert base - ms == 2 * 4 * n            # logits + momenta, one plane fewer
+    assert sh - base == 2 * 2 * 4 * n + n    # two planes more, plus j0
 
 
 def test_init_rejects_bad_buffers_before_cuda(lib):

@@ -172,7 +172,7 @@ def noise(prob: Problem, st: RowState, t: int) -> np.ndarray:
     if not prob.noise:
         return np.zeros((prob.K, len(st.row_ids), prob.C))
     if prob.mask_sign:
-        return philox.logistic(prob.seed, t, flat_index(prob, st.row_ids), 2)
+        return philox.logistic(prob.seed, t, flat_index(prob, st.row_ids))
     return philox.gumbel(prob.seed, t, flat_index(prob, st.row_ids), prob.K)
 
 

@@ -19,8 +19,10 @@ Stream layout (a reading; the paper is silent):
 
 Binary instances (the ternary mask x sign variant, Alg. 2) need only the
 difference of their two Gumbel draws, which is Logistic(0, 1); it is drawn
-directly by its inverse CDF from one word: lambda = ln(u) - ln(1 - u), with
-instance k taking word k of block 0.
+directly by its inverse CDF from one word: lambda = ln(u) - ln(1 - u).  Two
+weights share one block: weight i takes the block of counter
+(lo32(i'), hi32(i'), t, 0) with i' = i - (i mod 2), and instance k (0 mask,
+1 sign) takes word 2 (i mod 2) + k.
 """
 from __future__ import annotations
 
@@ -82,9 +84,21 @@ def gumbel(seed: int, t: int, flat_index, K: int) -> np.ndarray:
     return -np.log(-np.log(u))
 
 
-def logistic(seed: int, t: int, flat_index, n: int) -> np.ndarray:
+def pair_words(seed: int, t: int, flat_index) -> np.ndarray:
+    """Words [2, ...] of the two binary instances of every weight: one Philox
+    block per pair of weights (2j, 2j + 1), words (0, 1) for the even weight and
+    (2, 3) for the odd one."""
+    i = np.asarray(flat_index, dtype=np.uint64)
+    odd = (i & np.uint64(1)).astype(bool)
+    even = i - (i & np.uint64(1))
+    k0, k1 = int(seed) & 0xFFFFFFFF, (int(seed) >> 32) & 0xFFFFFFFF
+    w = philox4x32_10(even & _MASK32, even >> np.uint64(32), np.uint64(t), np.uint64(0), k0, k1)
+    return np.stack([np.where(odd, w[2], w[0]), np.where(odd, w[3], w[1])])
+
+
+def logistic(seed: int, t: int, flat_index) -> np.ndarray:
     """lam[k, ...] ~ Logistic(0, 1), the law of g1 - g0 for two independent
-    Gumbel(0, 1) draws: one per binary instance k < n and weight, fresh for
-    every step t.  Inverse CDF: lam = ln(u / (1 - u)).  fp64."""
-    u = uniform_from_word(level_words(seed, t, flat_index, n))
+    Gumbel(0, 1) draws: one per binary instance (k = 0 mask, 1 sign) and
+    weight, fresh for every step t.  Inverse CDF: lam = ln(u / (1 - u)).  fp64."""
+    u = uniform_from_word(pair_words(seed, t, flat_index))
     return np.log(u) - np.log1p(-u)

@@ -378,29 +378,27 @@ struct CatRelax {
   }
 };
 
-// Logistic(0, 1) draws in log2 units, log2(u / (1 - u)), for weights i0 and
-// i0 + 1: the mask instance takes word 0 and the sign instance word 1 of the
-// weight's first Philox block.  A binary GS over tied logits (-l, l) sees only
-// the difference g1 - g0 of its two Gumbel draws, whose law this is.  u and
-// 1 - u are both exact: the complemented 23 bits give 1 - u.
+// Logistic(0, 1) draws in log2 units, log2(u / (1 - u)), for weights i0 (even)
+// and i0 + 1, which share one Philox block (counter of i0, block 0): words 0
+// and 1 are the mask and sign draws of i0, words 2 and 3 those of i0 + 1.  A
+// binary GS over tied logits (-l, l) sees only the difference g1 - g0 of its
+// two Gumbel draws, whose law this is.  u and 1 - u are both exact: the
+// complemented 23 bits give 1 - u.
 __device__ __forceinline__ void draw_logistic2(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
                                                int on, float2 (&h)[2]) {
   if (!on) {
     h[0] = h[1] = f2(0.0f);
     return;
   }
-  const uint32_t lo = static_cast<uint32_t>(i0), hi = static_cast<uint32_t>(i0 >> 32);
-  const uint4 a = philox4x32_10(lo, hi, t, 0u, keys);
-  const uint4 b = philox4x32_10(lo + 1u, hi, t, 0u, keys);
+  const uint4 a = philox4x32_10(static_cast<uint32_t>(i0), static_cast<uint32_t>(i0 >> 32), t, 0u,
+                                keys);
   const float half = __uint_as_float(0x3F7FFFFFu);  // 1 - 2^-24
   auto unit = [&](uint32_t x) { return __uint_as_float(0x3F800000u | (x & 0x007FFFFFu)) - half; };
-  // ratio u / (1 - u) of the mask (x) and sign (y) draws, for each weight
-  const float2 ua = make_float2(unit(a.x), unit(a.y)), va = make_float2(unit(~a.x), unit(~a.y));
-  const float2 ub = make_float2(unit(b.x), unit(b.y)), vb = make_float2(unit(~b.x), unit(~b.y));
-  const float2 ra = mul2(ua, rcp2(va)), rb = mul2(ub, rcp2(vb));
-  const float2 la = log2_unit2(ra), lb = log2_unit2(rb);  // (mask, sign) of each weight
-  h[0] = make_float2(la.x, lb.x);
-  h[1] = make_float2(la.y, lb.y);
+  // u / (1 - u) for (mask, mask) and (sign, sign) of the two weights
+  const float2 um = make_float2(unit(a.x), unit(a.z)), vm = make_float2(unit(~a.x), unit(~a.z));
+  const float2 ub = make_float2(unit(a.y), unit(a.w)), vb = make_float2(unit(~a.y), unit(~a.w));
+  h[0] = log2_unit2(mul2(um, rcp2(vm)));
+  h[1] = log2_unit2(mul2(ub, rcp2(vb)));
 }
 
 // Ternary mask x sign (§3.1, Alg. 2): w~ = a m~ b~ on the grid {-a, 0, a}, with
@@ -515,10 +513,15 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
 // the updated registers.  Bytes per weight with look-ahead (L logits per
 // weight): read 8L + 4 + b_W (+1 for j0), write 8L + 2 (D bf16).
 // ---------------------------------------------------------------------------
-// Blocks per SM the register budget aims for (measured best on GB300).
+// Blocks per SM the register budget aims for (measured best on GB300): two;
+// three for the two-logit relaxations, which fit in 85 registers.
 template <int K>
 struct BwdOcc {
   static constexpr int value = 2;
+};
+template <>
+struct BwdOcc<2> {
+  static constexpr int value = 3;
 };
 
 template <class Rx, bool kExport, bool kShift>

@@ -67,11 +67,26 @@ def test_logistic_noise_hand_values_and_symmetry():
                                rtol=1e-12, atol=1e-12)
 
 
+def test_pair_words_layout():
+    """Weights 2j and 2j + 1 split the four words of one block (counter of the
+    even weight, block 0): the even weight takes words (0, 1), the odd (2, 3)."""
+    idx = np.array([0, 1, 6, 7, 2 ** 33 + 4, 2 ** 33 + 5], dtype=np.uint64)
+    got = philox.pair_words(99, 12, idx)
+    for j, i in enumerate(idx):
+        e = int(i) - int(i) % 2
+        w = philox.philox4x32_10(e & 0xFFFFFFFF, e >> 32, 12, 0, 99, 0)
+        o = 2 * (int(i) % 2)
+        assert (got[0, j], got[1, j]) == (w[o], w[o + 1])
+    # the even weight's words equal the first two words of its own block
+    assert np.array_equal(philox.pair_words(5, 1, np.arange(0, 64, 2)),
+                          philox.level_words(5, 1, np.arange(0, 64, 2), 2))
+
+
 def test_logistic_law_matches_gumbel_difference():
     """The drawn lambda and the difference of two independent Gumbel draws both
     follow F(x) = 1 / (1 + e^-x) (Kolmogorov-Smirnov at n = 200000)."""
     idx = np.arange(200_000)
-    lam = philox.logistic(7, 3, idx, 2)
+    lam = philox.logistic(7, 3, idx)
     g = philox.gumbel(7, 5, idx, 2)
     cdf = lambda x: 1.0 / (1.0 + np.exp(-x))
     for sample in (lam[0], lam[1], g[1] - g[0]):

@@ -463,6 +463,52 @@ def init_state(prob: Problem, W, row_ids, init_bias: float = 2.0) -> RowState:
                     kq_d=kq_d, kq_sc=kq_sc, j0=j0)
 
 
+def prior_logits(prob: Problem, codes) -> np.ndarray:
+    """The noise-free warm-start logits l_GPTQ around a supplied code vector
+    ([K, nr, C] float64), for the code of every weight (a grid index):
+      mask x sign (Eq. 3): l_m = +1 if the code is nonzero else -1;
+                           l_b = +1, -1 or 0 by the code's sign;
+      full grid (App. A, b = 2): l_k = -(c_k - mu)^2 / 2 with the candidates
+                           c_k the grid values and mu the coded value;
+      local shift (App. A, b > 2): the candidates are the shifts -2..2 and
+                           mu = 0;
+    in the last two cases minus each weight's mean logit (App. A)."""
+    codes = np.asarray(codes, dtype=np.int64)
+    if prob.mask_sign:
+        lm = np.where(codes != 1, 1.0, -1.0)
+        lb = np.where(codes == 2, 1.0, np.where(codes == 0, -1.0, 0.0))
+        return np.stack([lm, lb])
+    if prob.shift:
+        c = np.arange(-2, 3, dtype=np.float64).reshape((SHIFTS,) + (1,) * codes.ndim)
+        mu = np.zeros(codes.shape)
+    else:
+        grid = np.asarray(prob.grid, dtype=np.float64)
+        c = grid.reshape((len(grid),) + (1,) * codes.ndim)
+        mu = grid[codes]
+    l = -0.5 * (c - mu[None]) ** 2
+    return l - l.mean(axis=0, keepdims=True)
+
+
+def init_from_codes(prob: Problem, W, row_ids, codes, eps, alpha: float, sigma: float,
+                    scales=None) -> RowState:
+    """Warm start from a supplied solution (§3.1 "Initialization", Eq. 3-4;
+    App. A): logits l = sigma (eps + alpha l_GPTQ) with eps ~ N(0, I) given by
+    the caller ([K, nr, C]; None for eps = 0), zero momenta, the given scales
+    (default: the absmax scales of init_state), and for local shift j0 = the
+    supplied codes."""
+    st = init_state(prob, W, row_ids)
+    codes = np.asarray(codes, dtype=np.int64)
+    lg = prior_logits(prob, codes)
+    e = np.zeros_like(lg) if eps is None else np.asarray(eps, dtype=np.float64)
+    st.logits = (sigma * (e + alpha * lg)).astype(np.float32)
+    st.m_logits = np.zeros_like(st.logits)
+    if scales is not None:
+        st.scales = np.asarray(scales, dtype=np.float32).copy()
+    if prob.shift:
+        st.j0 = codes.astype(np.uint8)
+    return st
+
+
 # ----------------------------------------------------------------------------
 # hard projection (Alg. 2, final lines, generalised to K levels)
 # ----------------------------------------------------------------------------

@@ -154,6 +154,26 @@ GSQ_API gsq_status gsq_workspace_size(const gsq_layer_desc* desc, size_t* bytes)
 GSQ_API gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t bytes,
                           void* stream, gsq_layer** out);
 
+/* Warm start from a supplied solution (§3.1 "Initialization", Eq. 3-4; App. A),
+ * on `stream`, replacing the logits of gsq_init_layer:
+ *   l = sigma * (eps + alpha * l_prior), logit momenta = 0, where l_prior is,
+ *   for every weight with supplied code c (a grid index):
+ *     GSQ_PARAM_FULL       -(q_k - q_c)^2 / 2 minus its mean over k (App. A, b = 2);
+ *     GSQ_PARAM_SHIFT5     -d^2 / 2 for d = -2..2 minus its mean (App. A, b > 2),
+ *                          and j0 := c (the window is re-centred on the code);
+ *     GSQ_PARAM_MASK_SIGN  Eq. 3: l_m = +1 if c != 1 else -1, l_b = +1/-1/0 for
+ *                          c = 2/0/1.
+ * codes_dev  device uint8 [E][R][C], caller-owned; a code >= K acts as K-1.
+ * eps_dev    device fp32 [L][E][R][C] (L logit planes), caller-owned, nullable
+ *            (eps = 0): the N(0, I) draw of Eq. 4, made by the caller.
+ * alpha, sigma  Eq. 4's warm-start strength and logit scale (finite).
+ * Scales and scale momenta are left as they are (set them with gsq_set_tensor
+ * to start from the solution's scales).  Never synchronises.
+ * Errors: GSQ_ERR_INVALID_ARG (handle, NULL codes_dev, non-finite alpha or
+ * sigma), GSQ_ERR_CUDA. */
+GSQ_API gsq_status gsq_init_logits(gsq_layer* layer, const uint8_t* codes_dev, const float* eps_dev,
+                           float alpha, float sigma, void* stream);
+
 /* One optimisation step t (Alg. 2 loop body generalised to K levels):
  *   forward   noise for step t, p = softmax((kappa l + g)/tau), W^, D = W^ - W
  *             (skipped when the previous call already produced D for

@@ -655,6 +655,38 @@ gsq_status gsq_forward(gsq_layer* L, uint64_t step, float tau, float kappa, void
   return launch_fwd(L, step, tau, kappa, what_dev, static_cast<cudaStream_t>(stream));
 }
 
+gsq_status gsq_init_logits(gsq_layer* L, const uint8_t* codes_dev, const float* eps_dev, float alpha,
+                           float sigma, void* stream) {
+  GSQ_INJECT("gsq_init_logits");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!codes_dev) return fail(GSQ_ERR_INVALID_ARG, "codes_dev is NULL");
+  if (!std::isfinite(alpha) || !std::isfinite(sigma))
+    return fail(GSQ_ERR_INVALID_ARG, "alpha and sigma must be finite");
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Shape& sh = L->shape;
+  InitCodesParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.n = sh.n;
+  p.K = sh.K;
+  p.mode = sh.mode;
+  for (int k = 0; k < kMaxLevels; ++k) p.grid[k] = k < sh.K ? L->desc.grid[k] : 0.f;
+  p.codes = codes_dev;
+  p.eps = eps_dev;
+  p.alpha = alpha;
+  p.sigma = sigma;
+  p.logits = fptr(L, L->lay.logits);
+  p.m_logits = fptr(L, L->lay.m_logits);
+  p.j0 = sh.shift ? L->ws + L->lay.j0 : nullptr;
+  int slot;
+  prof_begin(L, GSQ_K_INIT, s, slot);
+  const cudaError_t e = launch_init_from_codes(p, L->num_sms, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "init from codes");
+  L->d_ready = false;
+  return GSQ_OK;
+}
+
 gsq_status gsq_project(gsq_layer* L, void* stream, uint8_t* codes_dev, float* margin_dev) {
   GSQ_INJECT("gsq_project");
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");

@@ -819,6 +819,57 @@ __global__ void __launch_bounds__(kEwThreads) k_init_kquant(const InitParams P) 
   }
 }
 
+// Warm start from supplied codes (Eq. 3-4, App. A): l = sigma (eps + alpha l_prior)
+// per logit plane, momenta 0; one quad of weights per thread and iteration.
+__device__ __forceinline__ float prior_logit(const InitCodesParams& P, int k, int c) {
+  if (P.mode == GSQ_PARAM_MASK_SIGN) {          // Eq. 3
+    if (k == 0) return c != 1 ? 1.0f : -1.0f;
+    return c == 2 ? 1.0f : (c == 0 ? -1.0f : 0.0f);
+  }
+  if (P.mode == GSQ_PARAM_SHIFT5) {             // -(d^2)/2 for d = k - 2, mean -1 removed
+    const float d = static_cast<float>(k - 2);
+    return 1.0f - 0.5f * d * d;
+  }
+  // -(q_k - q_c)^2 / 2 minus its mean over the K levels
+  const float mu = P.grid[c];
+  float mean = 0.0f;
+  for (int j = 0; j < P.K; ++j) {
+    const float e = P.grid[j] - mu;
+    mean += e * e;
+  }
+  mean = -0.5f * mean / static_cast<float>(P.K);
+  const float e = P.grid[k] - mu;
+  return -0.5f * e * e - mean;
+}
+
+__global__ void __launch_bounds__(kEwThreads) k_init_from_codes(const InitCodesParams P) {
+  const int L = P.mode == GSQ_PARAM_SHIFT5 ? 5 : (P.mode == GSQ_PARAM_MASK_SIGN ? 2 : P.K);
+  const int64_t nq = P.n >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t qi = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; qi < nq; qi += stride) {
+    uint32_t c4 = reinterpret_cast<const uint32_t*>(P.codes)[qi];
+    int c[4];
+    uint32_t clamped = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      c[j] = min(static_cast<int>((c4 >> (8 * j)) & 0xFFu), P.K - 1);
+      clamped |= static_cast<uint32_t>(c[j]) << (8 * j);
+    }
+    if (P.j0) reinterpret_cast<uint32_t*>(P.j0)[qi] = clamped;
+    for (int k = 0; k < L; ++k) {
+      float4 e = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (P.eps) e = __ldcs(reinterpret_cast<const float4*>(P.eps + k * P.n) + qi);
+      float4 v;
+      v.x = P.sigma * fmaf(P.alpha, prior_logit(P, k, c[0]), e.x);
+      v.y = P.sigma * fmaf(P.alpha, prior_logit(P, k, c[1]), e.y);
+      v.z = P.sigma * fmaf(P.alpha, prior_logit(P, k, c[2]), e.z);
+      v.w = P.sigma * fmaf(P.alpha, prior_logit(P, k, c[3]), e.w);
+      reinterpret_cast<float4*>(P.logits + k * P.n)[qi] = v;
+      reinterpret_cast<float4*>(P.m_logits + k * P.n)[qi] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+}
+
 __global__ void k_nonfinite(const void* x, int64_t count, int bf16, unsigned int* counter) {
   unsigned int bad = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -1114,6 +1165,13 @@ cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s) 
     const int grid = static_cast<int>(blocks < 16LL * num_sms ? blocks : 16LL * num_sms);
     k_init_group<<<grid > 0 ? grid : 1, kEwThreads, 0, s>>>(p);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_init_from_codes(const InitCodesParams& p, int num_sms, cudaStream_t s) {
+  const int64_t blocks = ((p.n >> 2) + kEwThreads - 1) / kEwThreads;
+  const int grid = static_cast<int>(blocks < 8LL * num_sms ? blocks : 8LL * num_sms);
+  k_init_from_codes<<<grid > 0 ? grid : 1, kEwThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

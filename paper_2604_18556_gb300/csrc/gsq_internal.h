@@ -99,6 +99,20 @@ struct InitParams {
   int8_t* kq_sc;       // [n/16]
 };
 cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s);
+
+struct InitCodesParams {
+  int64_t n;
+  int K;               // grid levels
+  int mode;            // GSQ_PARAM_*
+  float grid[kMaxLevels];
+  const uint8_t* codes;
+  const float* eps;    // [L][n] or null
+  float alpha, sigma;
+  float* logits;       // [L][n]
+  float* m_logits;     // [L][n]
+  uint8_t* j0;         // local shift: receives the codes
+};
+cudaError_t launch_init_from_codes(const InitCodesParams& p, int num_sms, cudaStream_t s);
 cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16,
                                   unsigned int* counter, cudaStream_t s);
 

@@ -40,7 +40,7 @@ KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init"]
 EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "gsq_project",
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
             "gsq_sync_status", "gsq_profile_enable", "gsq_profile_read", "gsq_destroy",
-            "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc"]
+            "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc", "gsq_init_logits"]
 
 
 class gsq_layer_desc(Structure):
@@ -100,6 +100,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "gsq_last_error": (c_char_p, []),
         "gsq_version": (c_char_p, []),
         "gsq_backward_update_noalloc": (c_int32, [POINTER(gsq_backward_args), P]),
+        "gsq_init_logits": (c_int32, [P, P, P, c_float, c_float, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -141,6 +142,10 @@ def gsq_step(handle: int, step: int, tau: float, kappa: float, next_tau: float, 
 
 def gsq_forward(handle: int, step: int, tau: float, kappa: float, stream: int, what_ptr=None) -> None:
     _check(_lib.gsq_forward(handle, step, tau, kappa, stream, what_ptr))
+
+
+def gsq_init_logits(handle: int, codes_ptr, eps_ptr, alpha: float, sigma: float, stream: int) -> None:
+    _check(_lib.gsq_init_logits(handle, codes_ptr, eps_ptr, alpha, sigma, stream))
 
 
 def gsq_project(handle: int, stream: int, codes_ptr=None, margin_ptr=None) -> None:
@@ -284,6 +289,12 @@ class Layer:
 
     def forward(self, t: int, tau: float, kappa: float = 1.0, what=None) -> None:
         gsq_forward(self.handle, t, tau, kappa, self._stream(), _ptr(what))
+
+    def init_logits(self, codes, eps=None, alpha: float = 1.0, sigma: float = 1.0) -> None:
+        """Warm start from supplied codes (uint8 [E, R, C]) and optional eps ([L, E, R, C] fp32)."""
+        codes = codes.contiguous()
+        eps = None if eps is None else eps.contiguous()
+        gsq_init_logits(self.handle, _ptr(codes), _ptr(eps), alpha, sigma, self._stream())
 
     def project(self, codes=None, margin=None) -> None:
         gsq_project(self.handle, self._stream(), _ptr(codes), _ptr(margin))

@@ -168,7 +168,9 @@ def test_handle_checks(lib):
                      (lib._lib.gsq_project, (None, None, None, None)),
                      (lib._lib.gsq_destroy, (None,)),
                      (lib._lib.gsq_destroy, (987654321,)),
-                     (lib._lib.gsq_sync_status, (None, None))]:
+                     (lib._lib.gsq_sync_status, (None, None)),
+                     (lib._lib.gsq_init_logits, (None, 4096, None, 1.0, 1.0, None)),
+                     (lib._lib.gsq_init_logits, (24681357, 4096, None, 1.0, 1.0, None))]:
         assert fn(*args) == lib.GSQ_ERR_INVALID_ARG
     assert lib.gsq_version().count(".") == 2
 

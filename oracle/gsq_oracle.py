@@ -34,6 +34,9 @@ What one step computes (paper references):
              level, 5 logits per weight for shifts delta in {-2..2} around the
              initial index j0; the level of shift delta is G[clip(j0 + delta)], so
              the same relaxation runs over a per-weight window of 5 levels.
+  micro-batches (§3.3 "Objective", "Gradient accumulation"): a step on per-step
+             token batches X_j; every forward pass draws fresh noise; the update
+             uses the mean of the micro-batches' gradients.
   mask x sign  (§3.1, Alg. 2): ternary weights s * m * b with a mask logit l_m
              and a sign logit l_b per weight, each relaxed by a binary GS over
              {0, 1} resp. {-1, 1} with the tied logits (-l, l) (§3 notation
@@ -48,7 +51,7 @@ sign(0) = 0; lowest index wins argmax ties; packing bit order; fp16 RNE).
 """
 from __future__ import annotations
 
-from dataclasses import dataclass, field
+from dataclasses import dataclass, field, replace
 from typing import Optional
 
 import numpy as np
@@ -347,6 +350,45 @@ def step(prob: Problem, st: RowState, t: int, tau: float, kappa: float,
             st.scales, st.m_scales = lion(st.scales, st.m_scales, d_scales, prob.lr_scales,
                                           prob.beta1, prob.beta2, prob.wd_scales)
     return StepResult(loss=L, fw=fw, G=G, d_logits=d_logits, d_scales=d_scales)
+
+
+@dataclass
+class MicroStepResult:
+    losses: list                        # L_j of every micro-batch (before the update)
+    d_logits: np.ndarray                # mean over the micro-batches
+    d_scales: Optional[np.ndarray]
+
+
+def step_microbatches(prob: Problem, st: RowState, t: int, batches, tau: float, kappa: float,
+                      update: bool = True) -> MicroStepResult:
+    """One optimisation step on per-step calibration tokens with gradient
+    accumulation over resampled noise (§3.3 "Objective" and "Gradient
+    accumulation").  batches: M token arrays X_j [E, T_j, C].  Micro-batch j
+    draws fresh noise (counter t*M + j: every forward pass is a new draw),
+    forms W^_j, its loss L_j = sum over its tokens of ||(W^_j - W) x||^2 (Eq. 1)
+    and the gradients; the update applies the mean gradient over the
+    micro-batches.  The state is unchanged until that update."""
+    M = len(batches)
+    q = None if prob.mask_sign else level_values(prob, st)
+    acc_l = acc_s = None
+    losses = []
+    for j, X in enumerate(batches):
+        pj = replace(prob, X=np.asarray(X, dtype=np.float64), H=None)
+        fw = forward(pj, st, t * M + j, tau, kappa)
+        L, G = loss_and_grad(pj, st.row_ids, fw.D)
+        dl, ds = backward(pj, fw, G, tau, kappa, q=q)
+        acc_l = dl if acc_l is None else acc_l + dl
+        acc_s = ds if acc_s is None else acc_s + ds
+        losses.append(L)
+    d_logits = acc_l / M
+    d_scales = None if scales_frozen(prob) else acc_s / M
+    if update:
+        st.logits, st.m_logits = lion(st.logits, st.m_logits, d_logits, prob.lr_logits,
+                                      prob.beta1, prob.beta2, prob.wd_logits)
+        if d_scales is not None:
+            st.scales, st.m_scales = lion(st.scales, st.m_scales, d_scales, prob.lr_scales,
+                                          prob.beta1, prob.beta2, prob.wd_scales)
+    return MicroStepResult(losses=losses, d_logits=d_logits, d_scales=d_scales)
 
 
 # ----------------------------------------------------------------------------

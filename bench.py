@@ -246,11 +246,62 @@ def run_oracle_sample(w, step_budget_s: float, n_steps: int, n_warm: int, Wt=Non
     return per * (w.experts * w.rows) / rows, rows, float(sum(times))
 
 
+def run_oracle_tokens_sample(w, n_steps: int, rows: int = 256, tok=(512, 4096)):
+    """Oracle step on per-step token batches, sampled in rows and tokens.  The
+    micro-batch cost is linear in its tokens (the loss contractions) plus a part
+    that is not (noise, softmax, backward, Lion): both are fitted from one
+    micro-batch of tok[0] and of tok[1] tokens on `rows` rows, then scaled to the
+    workload's tokens per micro-batch, micro-batches and rows.  Returns (seconds
+    per full step, description of the sample, seconds measured)."""
+    import dataclasses
+    import numpy as np
+    import torch
+    from oracle import gsq_oracle as O
+    from paper_2604_18556_gb300 import configs as C
+    from paper_2604_18556_gb300 import inputs
+    w1 = C.shrunk(w, experts=1)
+    Wt = inputs.make_weight(w1)[0, :rows].float().numpy()
+    prob = _oracle_problem(w1, None, None)
+    per_tok = []
+    measured = 0.0
+    for T in tok:
+        wt = dataclasses.replace(w1, tokens=T, micro=1)
+        X = inputs.make_token_batch(wt, 0, 0).double().numpy()
+        times = []
+        for t in range(n_steps + 1):
+            st = O.init_state(prob, Wt, np.arange(rows), init_bias=w.init_bias)
+            t0 = time.perf_counter()
+            O.step_microbatches(prob, st, t, [X], w.tau(t), w.kappa)
+            times.append(time.perf_counter() - t0)
+        measured += sum(times)
+        per_tok.append(float(np.median(times[1:])))
+    b = (per_tok[1] - per_tok[0]) / (tok[1] - tok[0])
+    a = max(per_tok[0] - b * tok[0], 0.0)
+    full = (a + b * w.tokens) * w.micro * (w.experts * w.rows) / rows
+    desc = (f"{rows} rows x one micro-batch of {tok[0]} and of {tok[1]} tokens, {n_steps} timed "
+            f"steps each ({measured:.1f} s measured); cost fitted as a + b*tokens and scaled to "
+            f"{w.tokens} tokens x {w.micro} micro-batches x {w.experts * w.rows} rows")
+    return full, desc, measured
+
+
 def reference_arm(args, rank, world):
     if rank != 0:
         return 0
     _single_thread_env()
     w = _workload(args.workload)
+    if w.calib == "batches":
+        full_step_s, desc, _ = run_oracle_tokens_sample(w, max(args.steps, 1))
+        value = 1.0 / full_step_s
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": full_step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config(w, {"oracle": "numpy float64, one thread"}),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return 0
     per_step_budget = 1.0
     full_step_s, rows, measured = run_oracle_sample(w, per_step_budget, args.steps, args.warmup)
     value = 1.0 / full_step_s
@@ -383,6 +434,166 @@ def gpu_arm(args, rank, world, local):
     return 0
 
 
+def gpu_arm_tokens(args, rank, world, local):
+    """One step = w.micro micro-batches of w.tokens per-step tokens (gsq_step_tokens),
+    Lion after the last; the token batches are resident in HBM and reused."""
+    import torch
+    import torch.distributed as dist
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2604_18556_gb300 import build
+    build.build()
+    from paper_2604_18556_gb300 import gsq, inputs
+
+    w = rank_workload(_workload(args.workload), rank, world)
+    W = inputs.make_weight(w, device="cuda")
+    Xs = [inputs.make_token_batch(w, 0, j, device="cuda") for j in range(w.micro)]
+    hyper = dict(init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits, lr_scales=w.lr_scales,
+                 beta1=w.beta1, beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
+                 param=w.param)
+    layer = gsq.Layer(W, None, w.grid, w.group, calib_kind="batches", tokens_per_batch=w.tokens,
+                      scale_mode=w.scale_mode, gemm="bf16", **hyper)
+    stream = torch.cuda.current_stream()
+    loss = torch.zeros(w.micro, device="cuda")
+    T = w.steps
+
+    def one_step(layer, t, Xs, loss):
+        for j, X in enumerate(Xs):
+            layer.step_tokens(t, j, w.micro, w.tau(t % T), X, kappa=w.kappa,
+                              next_tau=w.tau((t + 1) % T), next_kappa=w.kappa, loss=loss[j:j + 1])
+
+    t = 0
+    for _ in range(args.warmup):
+        one_step(layer, t, Xs, loss)
+        t += 1
+    layer.sync_status()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    layer.profile_enable(True)
+    layer.profile_read()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        one_step(layer, t, Xs, loss)
+        t += 1
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    prof = layer.profile_read()
+    layer.profile_enable(False)
+    layer.sync_status()
+    ms_step = max_over_ranks(e0.elapsed_time(e1), torch.device("cuda", local)) / args.steps
+    value = whole_job_steps_per_s(ms_step, world)
+
+    hbm, tf_burst, tf_sust, peak_src = _peaks()
+    gemm_n, gemm_ms = prof["gemm"]
+    bwd_n, bwd_ms = prof["backward"]
+    tok_n, tok_ms = prof["tokens"]
+    fwd_n, fwd_ms = prof["forward"]
+    gemm_avg = gemm_ms / max(gemm_n, 1)
+    flops_per_launch = w.gemm_flops_per_step() / w.micro      # Y = D X^T and G = 2 Y X
+    gemm_tfs = flops_per_launch / (gemm_avg * 1e-3) / 1e12
+    bytes_step = w.elementwise_bytes_per_step()
+    bwd_gbs = bytes_step / (bwd_ms / args.steps * 1e-3) / 1e9
+    roofline = {"kernel": "k_tc_gemm x 2 (Y = D X^T, then G = 2 Y X; tcgen05, bf16 in, fp32 acc)",
+                "bound": "tensor", "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
+                "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst, "traffic": None,
+                "flops_per_launch": flops_per_launch, "avg_launch_ms": gemm_avg,
+                "peak_source": f"{peak_src} bf16_tflops_sustained (MEASURED_PEAKS.json)"}
+    roofline_bwd = {"kernel": "k_backward (accumulating / Lion + next forward), all micro-batches",
+                    "bound": "hbm", "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s",
+                    "frac": bwd_gbs / hbm, "algorithmic_bytes_per_step": bytes_step,
+                    "ms_per_step": bwd_ms / args.steps}
+    launches = gemm_n * 2 + bwd_n + tok_n + fwd_n
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step)
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_tokens(args, w)
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32 (tensor-core GEMMs bf16 in, f32 acc)",
+            "data": "synthetic (seeded; Llama-3.1-8B q_proj shape, per-step token batches)",
+            "config": _config(w, {"parallelism": f"{world} independent layer(s), one per GPU",
+                                  "micro_batches": w.micro, "tokens_per_micro_batch": w.tokens,
+                                  "l2": "token batches of "
+                                        f"{w.tokens * w.cols * 4 / 2**20:.0f} MiB each, larger "
+                                        "than L2"}),
+            "roofline": roofline, "roofline_backward": roofline_bwd, "clocks": clocks,
+            "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
+            "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
+                                   "tokens": tok_ms / args.steps, "forward": fwd_ms / args.steps},
+        }), flush=True)
+    layer.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step):
+    """The whole job through the public API from pinned host buffers: W and the
+    micro-batch tokens uploaded, init, K steps (every micro-batch's loss read
+    back), projection + packing, packed download."""
+    W_host = W.cpu().pin_memory()
+    X_host = [X.cpu().pin_memory() for X in Xs]
+    K = args.steps
+    loss_host = torch.zeros(K, w.micro, dtype=torch.float32).pin_memory()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    Wd = W_host.to("cuda", non_blocking=True)
+    Xd = [X.to("cuda", non_blocking=True) for X in X_host]
+    layer = gsq.Layer(Wd, None, w.grid, w.group, calib_kind="batches", tokens_per_batch=w.tokens,
+                      scale_mode=w.scale_mode, gemm="bf16", **hyper)
+    loss = torch.zeros(K, w.micro, device="cuda")
+    for t in range(K):
+        one_step(layer, t, Xd, loss[t])
+        loss_host[t].copy_(loss[t], non_blocking=True)
+    packed = torch.empty(layer.packed_size(), dtype=torch.uint8, device="cuda")
+    layer.pack(packed)
+    packed_host = torch.empty(packed.numel(), dtype=torch.uint8).pin_memory()
+    packed_host.copy_(packed, non_blocking=True)
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    layer.close()
+    if not bool(torch.isfinite(loss_host).all()):
+        raise RuntimeError("non-finite loss in the end-to-end run")
+    h2d = W_host.numel() * W_host.element_size() + sum(X.numel() * 4 for X in X_host)
+    return {"value": world * K / dt, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
+            "d2h_bytes_per_step": (4 * K * w.micro + packed_host.numel()) / K,
+            "what": f"one {K}-step job: pinned W + {w.micro} token batches uploaded, init, "
+                    f"{K} steps with every loss read back, projection + packing, download"}
+
+
+def cpu_baseline_tokens(args, w):
+    code = ("import sys, json; sys.path.insert(0, %r)\n"
+            "import bench\n"
+            "from paper_2604_18556_gb300 import configs as C\n"
+            "full, desc, meas = bench.run_oracle_tokens_sample(C.WORKLOADS[%r], 3)\n"
+            "print(json.dumps([full, desc]))\n") % (ROOT, w.name)
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                       cwd=ROOT, timeout=900)
+    if r.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle",
+                "sample": f"failed: {r.stderr[-300:]}"}
+    full, desc = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": 1.0 / full, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
+
+
 def e2e_run(args, w, W, H, gsq, torch, rank, world):
     """The whole per-layer job through the public API with host buffers: pinned
     W and H copied to the GPU, init, K steps (each step's loss read back into
@@ -457,6 +668,8 @@ def main():
     rank, world, local = _dist()
     if args.impl == "reference":
         return reference_arm(args, rank, world)
+    if _workload(args.workload).calib == "batches":
+        return gpu_arm_tokens(args, rank, world, local)
     return gpu_arm(args, rank, world, local)
 
 

@@ -68,7 +68,7 @@ typedef int32_t gsq_status;
 /* ---- descriptor enums ---------------------------------------------------- */
 #define GSQ_MAX_LEVELS 8
 enum { GSQ_DTYPE_F32 = 0, GSQ_DTYPE_BF16 = 1 };
-enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1 };
+enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1, GSQ_CALIB_BATCHES = 2 };
 enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
 enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
 enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel draw */
@@ -83,6 +83,10 @@ enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1, GSQ_PARAM_MASK_SIGN = 2 };
  *              (symmetrised as (H + H^T)/2 on copy).
  *              GSQ_CALIB_X: tokens X_e, [E][n_tokens][C] row-major; H_e is formed
  *              from them at init (fp32, on the GPU).
+ *              GSQ_CALIB_BATCHES: no calibration at init (calib may be NULL);
+ *              tokens arrive with every micro-batch through gsq_step_tokens,
+ *              n_tokens being the most tokens per micro-batch and expert
+ *              (a multiple of 8).
  * grid         the K ordered levels q_0 < ... < q_{K-1} (host values, copied).
  * group_size   scale group along the input dim, power of two in [4, 128],
  *              in_features % group_size == 0.  GSQ_SCALE_KQUANT2 requires 16.
@@ -197,6 +201,33 @@ GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float ka
                     float next_kappa, void* stream, float* loss_dev, float* grad_logits_dev,
                     float* grad_scales_dev);
 
+/* One micro-batch of an optimisation step on per-step calibration tokens, with
+ * gradient accumulation over resampled noise (§3.3 "Objective" and "Gradient
+ * accumulation"); layers described with GSQ_CALIB_BATCHES only.
+ * Step `step` has n_micro micro-batches, issued in order micro = 0..n_micro-1
+ * (another order returns GSQ_ERR_STATE).  Micro-batch j of step t:
+ *   forward   fresh noise with the counter t*n_micro + j (every forward pass
+ *             draws anew), W^_j, D_j = W^_j - W;
+ *   loss      Y = D_j X^T, G = 2 Y X  (X = X_dev, this micro-batch's tokens),
+ *             L_j = 1/2 sum D_j*G = sum over the tokens of ||D_j x||^2;
+ *   backward  the gradients of L_j, added into an accumulator;
+ *   update    after the last micro-batch only: Lion with the mean gradient
+ *             (accumulated sum / n_micro); the state is untouched before that.
+ * Each call's kernel also draws the next pass's noise and writes its D: the
+ * next micro-batch's (same tau, kappa) or, after the last micro-batch and when
+ * next_tau > 0, micro-batch 0 of step+1 with (next_tau, next_kappa).
+ * X_dev      device fp32 [E][n_tokens][C], caller-owned, borrowed for the call;
+ *            the tensor-core path converts it to bf16.
+ * n_tokens   tokens of this micro-batch per expert: a multiple of 8, at most the
+ *            descriptor's n_tokens.
+ * loss_dev   device fp32 scalar, nullable: receives L_j.
+ * Errors: GSQ_ERR_INVALID_ARG (handle, layer not GSQ_CALIB_BATCHES, NULL X,
+ * bad n_tokens, micro >= n_micro, tau, counter >= 2^32), GSQ_ERR_STATE,
+ * GSQ_ERR_CUDA.  Never synchronises. */
+GSQ_API gsq_status gsq_step_tokens(gsq_layer* layer, uint64_t step, uint32_t micro, uint32_t n_micro,
+                           float tau, float kappa, float next_tau, float next_kappa,
+                           const float* X_dev, int64_t n_tokens, void* stream, float* loss_dev);
+
 /* Forward only (Alg. 1 for every weight): writes D for (step, tau, kappa) into
  * the workspace and, if what_dev (device fp32 [E][R][C]) is non-null, the soft
  * weight W^.  A following gsq_step with the same (step, tau, kappa) reuses D. */
@@ -266,7 +297,8 @@ enum {
   GSQ_K_PROJECT = 3,
   GSQ_K_PACK = 4,
   GSQ_K_INIT = 5,
-  GSQ_K_COUNT = 6
+  GSQ_K_TOKENS = 6,   /* per-step tokens to the tensor-core operands (bf16, X^T) */
+  GSQ_K_COUNT = 7
 };
 typedef struct gsq_profile {
   int32_t launches[GSQ_K_COUNT];

@@ -32,8 +32,8 @@ class Workload:
     grid: Tuple[float, ...]
     group: int                 # scale group along the input dim (16 = K-Quant sub-block)
     w_dtype: str               # "f32" | "bf16"
-    calib: str                 # "X" (tokens kept) | "H" (Gram matrix)
-    tokens: int                # calibration tokens per expert
+    calib: str                 # "X" (tokens kept) | "H" (Gram matrix) | "batches" (per step)
+    tokens: int                # calibration tokens per expert (per micro-batch for "batches")
     token_dist: str            # "normal" | "student_t3"
     outliers: int              # number of outlier channels
     outlier_scale: float
@@ -52,6 +52,7 @@ class Workload:
     wd_scales: float = 0.0
     data_seed: int = 0
     pack: bool = False
+    micro: int = 1             # "batches": micro-batches per step (gradient accumulation)
     param: str = "full"        # "full": one logit per level; "shift5": local shift (§3.2);
     #                            "mask_sign": ternary mask x sign (§3.1, Alg. 2)
 
@@ -86,7 +87,26 @@ class Workload:
         return 16 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
 
     def gemm_flops_per_step(self) -> int:
+        """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or
+        per micro-batch Y = D X^T and G = 2 Y X (4 R C T per expert)."""
+        if self.calib == "batches":
+            return 4 * self.experts * self.rows * self.cols * self.tokens * self.micro
         return 2 * self.experts * self.rows * self.cols * self.cols
+
+    def elementwise_bytes_per_step(self) -> int:
+        """Algorithmic HBM bytes of one step's fused elementwise kernels, all
+        micro-batches: every pass reads the logits (4L), G (4), W (b_W) and j0
+        (local shift) and writes the next D (2); the accumulator (4L) is written
+        by the first pass, read and written by the middle ones and read by the
+        last, which also reads and writes the momenta and writes the logits."""
+        n = self.n
+        if self.micro <= 1:
+            return self.elementwise_bytes_per_weight() * n
+        base = 4 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
+        first = base + 4 * self.L
+        middle = base + 8 * self.L
+        last = base + 4 * self.L + 8 * self.L + 4 * self.L
+        return (first + (self.micro - 2) * middle + last) * n
 
 
 WORKLOADS = {
@@ -121,6 +141,13 @@ WORKLOADS = {
                  grid=GRID_TERNARY, group=128, w_dtype="bf16", calib="H", tokens=128 * 2048,
                  token_dist="normal", outliers=41, outlier_scale=30.0, steps=500, tau0=1.0,
                  tau1=0.1, data_seed=2000, param="mask_sign"),
+        # Per-step calibration tokens with gradient accumulation (§3.3): the q_proj
+        # layer, one step = 8 micro-batches of 8 sequences x 4096 tokens (Table 5's
+        # batch of 64 sequences), fresh noise per micro-batch.
+        Workload(name="llama8b_q_proj_tokens", experts=1, rows=4096, cols=4096,
+                 grid=GRID_2BIT_SYM, group=128, w_dtype="bf16", calib="batches",
+                 tokens=8 * 4096, token_dist="normal", outliers=41, outlier_scale=30.0,
+                 steps=500, tau0=1.0, tau1=0.1, data_seed=2000, micro=8),
     ]
 }
 

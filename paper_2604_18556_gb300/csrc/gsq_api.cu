@@ -80,6 +80,7 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
   size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch, j0;
+  size_t tok_b, tok_t, Y, acc_l, acc_s;  // per-step token batches (GSQ_CALIB_BATCHES)
   size_t total;
 };
 
@@ -88,7 +89,8 @@ struct Shape {
   int K, group;
   int L;     // logits per weight: K, 5 with local shift, 2 with mask x sign
   int mode;  // GSQ_PARAM_*
-  bool kquant, d_bf16, w_bf16, x_mode, shift, mask_sign;
+  int64_t T;  // GSQ_CALIB_BATCHES: most tokens per micro-batch and expert
+  bool kquant, d_bf16, w_bf16, x_mode, shift, mask_sign, batches;
 };
 
 Shape shape_of(const gsq_layer_desc& d) {
@@ -104,6 +106,8 @@ Shape shape_of(const gsq_layer_desc& d) {
   s.d_bf16 = d.gemm_precision == GSQ_GEMM_BF16;
   s.w_bf16 = d.w_dtype == GSQ_DTYPE_BF16;
   s.x_mode = d.calib_kind == GSQ_CALIB_X;
+  s.batches = d.calib_kind == GSQ_CALIB_BATCHES;
+  s.T = s.batches ? d.n_tokens : 0;
   s.mode = d.param_mode;
   s.shift = d.param_mode == GSQ_PARAM_SHIFT5;
   s.mask_sign = d.param_mode == GSQ_PARAM_MASK_SIGN;
@@ -127,13 +131,19 @@ Layout layout_of(const Shape& s) {
   L.scales = take(4 * ng);
   L.m_scales = take(4 * ng);
   L.W = take(n * (s.w_bf16 ? 2 : 4));
-  L.H = take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4));
+  L.H = s.batches ? off : take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4));
   L.D = take(n * (s.d_bf16 ? 2 : 4));
   L.G = take(4 * n);
   L.kq_d = s.kquant ? take(2 * (n / kSuperBlock)) : off;
   L.kq_sc = s.kquant ? take(n / kSubBlock) : off;
   L.hscratch = s.x_mode ? take(static_cast<size_t>(s.E) * s.C * s.C * 4) : off;
   L.j0 = s.shift ? take(n) : off;
+  const size_t et = static_cast<size_t>(s.E) * static_cast<size_t>(s.T);
+  L.tok_b = s.batches && s.d_bf16 ? take(2 * et * s.C) : off;
+  L.tok_t = s.batches && s.d_bf16 ? take(2 * et * s.C) : off;
+  L.Y = s.batches ? take((s.d_bf16 ? 2 : 4) * et * s.R) : off;
+  L.acc_l = s.batches ? take(4 * n * s.L) : off;
+  L.acc_s = s.batches ? take(4 * ng) : off;
   L.total = off;
   return L;
 }
@@ -164,8 +174,12 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
     return fail(GSQ_ERR_SHAPE, "in_features %% group_size != 0");
   if (d->w_dtype != GSQ_DTYPE_F32 && d->w_dtype != GSQ_DTYPE_BF16)
     return fail(GSQ_ERR_INVALID_ARG, "bad w_dtype %d", d->w_dtype);
-  if (d->calib_kind != GSQ_CALIB_H && d->calib_kind != GSQ_CALIB_X)
+  if (d->calib_kind != GSQ_CALIB_H && d->calib_kind != GSQ_CALIB_X &&
+      d->calib_kind != GSQ_CALIB_BATCHES)
     return fail(GSQ_ERR_INVALID_ARG, "bad calib_kind %d", d->calib_kind);
+  if (d->calib_kind == GSQ_CALIB_BATCHES &&
+      (d->n_tokens < 8 || d->n_tokens > 2147483647LL || d->n_tokens % 8 != 0))
+    return fail(GSQ_ERR_INVALID_ARG, "GSQ_CALIB_BATCHES needs n_tokens in [8, 2^31), a multiple of 8");
   if (d->calib_kind == GSQ_CALIB_X && (d->n_tokens < 1 || d->n_tokens > 2147483647LL))
     return fail(GSQ_ERR_INVALID_ARG, "n_tokens must be in [1, 2^31) for GSQ_CALIB_X");
   if (d->scale_mode != GSQ_SCALE_GROUP && d->scale_mode != GSQ_SCALE_KQUANT2)
@@ -227,6 +241,9 @@ struct gsq_layer {
   bool d_ready;
   uint64_t d_step;
   float d_tau, d_kappa;
+  // micro-batch sequence of gsq_step_tokens: the next call it accepts
+  uint64_t mb_step;
+  uint32_t mb_next, mb_count;
   // profiling
   bool profiling;
   std::vector<cudaEvent_t> ev;  // pairs
@@ -358,13 +375,15 @@ gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
   prof_begin(L, GSQ_K_GEMM, s, slot);
   cudaError_t e;
   if (sh.d_bf16) {
-    TcGemm g;
+    TcGemm g;  // G = 2 D H (H symmetrised, so its rows are K-major columns)
     g.E = static_cast<int>(sh.E);
-    g.R = static_cast<int>(sh.R);
-    g.C = static_cast<int>(sh.C);
-    g.D = L->ws + L->lay.D;
-    g.H = L->ws + L->lay.H;
-    g.G = fptr(L, L->lay.G);
+    g.M = static_cast<int>(sh.R);
+    g.N = static_cast<int>(sh.C);
+    g.K = static_cast<int>(sh.C);
+    g.A = L->ws + L->lay.D;
+    g.B = L->ws + L->lay.H;
+    g.out = fptr(L, L->lay.G);
+    g.out_bf16 = 0;
     g.alpha = 2.0f;
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = L->tile_n;
@@ -406,7 +425,7 @@ size_t tensor_bytes(const gsq_layer* L, int which) {
     case GSQ_T_D: return n * (s.d_bf16 ? 2 : 4);
     case GSQ_T_G: return 4 * n;
     case GSQ_T_W: return n * (s.w_bf16 ? 2 : 4);
-    case GSQ_T_H: return static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4);
+    case GSQ_T_H: return s.batches ? 0 : static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4);
     case GSQ_T_KQ_D: return s.kquant ? 2 * (n / kSuperBlock) : 0;
     case GSQ_T_KQ_SC: return s.kquant ? n / kSubBlock : 0;
     case GSQ_T_J0: return s.shift ? n : 0;
@@ -463,7 +482,8 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   *out = nullptr;
   gsq_status st = validate_desc(desc);
   if (st != GSQ_OK) return st;
-  if (!desc->W || !desc->calib) return fail(GSQ_ERR_INVALID_ARG, "W and calib must be device pointers");
+  if (!desc->W || (!desc->calib && desc->calib_kind != GSQ_CALIB_BATCHES))
+    return fail(GSQ_ERR_INVALID_ARG, "W and calib must be device pointers");
   if (!workspace) return fail(GSQ_ERR_WORKSPACE, "workspace is NULL");
   if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
     return fail(GSQ_ERR_WORKSPACE, "workspace must be 256-byte aligned");
@@ -496,6 +516,9 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   L->num_sms = prop.multiProcessorCount;
   L->tc = tc;
   L->d_ready = false;
+  L->mb_step = 0;
+  L->mb_next = 0;
+  L->mb_count = 0;
   L->profiling = false;
   L->ev_used = 0;
   L->last_stream = nullptr;
@@ -527,9 +550,11 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     return bail(cuda_fail(e, "copy W"));
   if ((e = launch_nonfinite_scan(L->ws + lay.W, sh.n, sh.w_bf16, &flags->nonfinite, s)) != cudaSuccess)
     return bail(cuda_fail(e, "scan W"));
-  const int64_t calib_count = sh.x_mode ? sh.E * desc->n_tokens * sh.C : sh.E * sh.C * sh.C;
-  if ((e = launch_nonfinite_scan(desc->calib, calib_count, 0, &flags->nonfinite, s)) != cudaSuccess)
-    return bail(cuda_fail(e, "scan calib"));
+  if (!sh.batches) {
+    const int64_t calib_count = sh.x_mode ? sh.E * desc->n_tokens * sh.C : sh.E * sh.C * sh.C;
+    if ((e = launch_nonfinite_scan(desc->calib, calib_count, 0, &flags->nonfinite, s)) != cudaSuccess)
+      return bail(cuda_fail(e, "scan calib"));
+  }
 
   int slot;
   prof_begin(L, GSQ_K_INIT, s, slot);
@@ -556,7 +581,8 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if ((e = launch_simt_gemm(g, s)) != cudaSuccess) return bail(cuda_fail(e, "X^T X"));
     hsrc = fptr(L, lay.hscratch);
   }
-  if ((e = launch_symmetrize(hsrc, L->ws + lay.H, static_cast<int>(sh.E), static_cast<int>(sh.C),
+  if (!sh.batches &&
+      (e = launch_symmetrize(hsrc, L->ws + lay.H, static_cast<int>(sh.E), static_cast<int>(sh.C),
                              sh.d_bf16, s)) != cudaSuccess)
     return bail(cuda_fail(e, "symmetrise H"));
 
@@ -596,6 +622,8 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
                     float* grad_scales_dev) {
   GSQ_INJECT("gsq_step");
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (L->shape.batches)
+    return fail(GSQ_ERR_INVALID_ARG, "GSQ_CALIB_BATCHES layers step with gsq_step_tokens");
   if (step >= (1ull << 32)) return fail(GSQ_ERR_INVALID_ARG, "step must be < 2^32");
   if (!(tau > 0.f) || !std::isfinite(tau) || !std::isfinite(kappa))
     return fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");
@@ -641,6 +669,137 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
   } else if (!export_mode) {
     L->d_ready = false;
   }
+  return GSQ_OK;
+}
+
+gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t n_micro,
+                           float tau, float kappa, float next_tau, float next_kappa,
+                           const float* X_dev, int64_t n_tokens, void* stream, float* loss_dev) {
+  GSQ_INJECT("gsq_step_tokens");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  const Shape& sh = L->shape;
+  if (!sh.batches) return fail(GSQ_ERR_INVALID_ARG, "gsq_step_tokens needs a GSQ_CALIB_BATCHES layer");
+  if (!X_dev) return fail(GSQ_ERR_INVALID_ARG, "X_dev is NULL");
+  if (n_tokens < 8 || n_tokens > sh.T || n_tokens % 8 != 0)
+    return fail(GSQ_ERR_INVALID_ARG, "n_tokens must be a multiple of 8 in [8, %lld]",
+                static_cast<long long>(sh.T));
+  if (n_micro < 1 || micro >= n_micro) return fail(GSQ_ERR_INVALID_ARG, "need micro < n_micro");
+  const uint64_t t = step * n_micro + micro;  // noise counter of this forward pass
+  if (step >= (1ull << 32) || t + 1 >= (1ull << 32))
+    return fail(GSQ_ERR_INVALID_ARG, "step * n_micro + micro + 1 must be < 2^32");
+  if (!(tau > 0.f) || !std::isfinite(tau) || !std::isfinite(kappa))
+    return fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");
+  const bool last = micro + 1 == n_micro;
+  const bool lookahead = !last || next_tau > 0.f;
+  if (last && lookahead && (!std::isfinite(next_tau) || !std::isfinite(next_kappa)))
+    return fail(GSQ_ERR_INVALID_ARG, "next_tau / next_kappa must be finite");
+  if (micro > 0 && !(L->mb_step == step && L->mb_next == micro && L->mb_count == n_micro))
+    return fail(GSQ_ERR_STATE, "micro-batches of a step must be issued in order from 0");
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  gsq_status st;
+  if (!(L->d_ready && L->d_step == t && L->d_tau == tau && L->d_kappa == kappa)) {
+    if ((st = launch_fwd(L, t, tau, kappa, nullptr, s)) != GSQ_OK) return st;
+  }
+
+  // loss contraction on this micro-batch's tokens: Y = D X^T, G = 2 Y X
+  const int E = static_cast<int>(sh.E), R = static_cast<int>(sh.R), C = static_cast<int>(sh.C);
+  const int T = static_cast<int>(n_tokens);
+  int slot;
+  cudaError_t e = cudaSuccess;
+  void* Xb = L->ws + L->lay.tok_b;
+  void* Xt = L->ws + L->lay.tok_t;
+  if (sh.d_bf16) {
+    prof_begin(L, GSQ_K_TOKENS, s, slot);
+    e = launch_tokens_bf16(X_dev, Xb, Xt, E, T, C, T, s);
+    prof_end(L, slot, s);
+    if (e != cudaSuccess) return cuda_fail(e, "token conversion");
+  }
+  prof_begin(L, GSQ_K_GEMM, s, slot);
+  if (sh.d_bf16) {
+    TcGemm g;
+    g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+    g.tile_n = 0;
+    g.E = E;
+    if (e == cudaSuccess) {  // Y[e] = D[e] X[e]^T  (N = T, K = C), bf16 out
+      g.M = R; g.N = T; g.K = C;
+      g.A = L->ws + L->lay.D;
+      g.B = Xb;
+      g.out = L->ws + L->lay.Y;
+      g.out_bf16 = 1;
+      g.alpha = 1.0f;
+      e = launch_tc_gemm(g, L->num_sms, s);
+    }
+    if (e == cudaSuccess) {  // G[e] = 2 Y[e] X[e]  (N = C, K = T), fp32 out
+      g.M = R; g.N = C; g.K = T;
+      g.A = L->ws + L->lay.Y;
+      g.B = Xt;
+      g.out = fptr(L, L->lay.G);
+      g.out_bf16 = 0;
+      g.alpha = 2.0f;
+      e = launch_tc_gemm(g, L->num_sms, s);
+    }
+  } else {
+    SimtGemm g;  // Y[e][r][t] = sum_c D[e][r][c] X[e][t][c]
+    g.batch = E;
+    g.M = R; g.N = T; g.Kd = C;
+    g.A = L->ws + L->lay.D; g.sam = C; g.sak = 1; g.sab = static_cast<int64_t>(R) * C;
+    g.B = X_dev; g.sbk = 1; g.sbn = C; g.sbb = static_cast<int64_t>(T) * C;
+    g.C = fptr(L, L->lay.Y); g.ldc = T; g.scb = static_cast<int64_t>(R) * T;
+    g.alpha = 1.0f;
+    g.bf16_inputs = 0;
+    e = launch_simt_gemm(g, s);
+    if (e == cudaSuccess) {  // G[e][r][c] = 2 sum_t Y[e][r][t] X[e][t][c]
+      g.M = R; g.N = C; g.Kd = T;
+      g.A = fptr(L, L->lay.Y); g.sam = T; g.sak = 1; g.sab = static_cast<int64_t>(R) * T;
+      g.B = X_dev; g.sbk = C; g.sbn = 1; g.sbb = static_cast<int64_t>(T) * C;
+      g.C = fptr(L, L->lay.G); g.ldc = C; g.scb = static_cast<int64_t>(R) * C;
+      g.alpha = 2.0f;
+      e = launch_simt_gemm(g, s);
+    }
+  }
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "token loss GEMMs");
+
+  EwParams p = base_params(L);
+  p.t = static_cast<uint32_t>(t);
+  p.kappa_log2 = static_cast<float>(kappa * kLog2e);
+  p.inv_tau = static_cast<float>(1.0 / tau);
+  p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
+  const float nt = last ? next_tau : tau, nk = last ? next_kappa : kappa;
+  p.lookahead = lookahead ? 1 : 0;
+  if (lookahead) {
+    p.t_next = static_cast<uint32_t>(t + 1);
+    p.kappa_log2_next = static_cast<float>(nk * kLog2e);
+    p.inv_tau_next = static_cast<float>(1.0 / nt);
+  }
+  float* acc_l = fptr(L, L->lay.acc_l);
+  float* acc_s = fptr(L, L->lay.acc_s);
+  if (!last) {  // export this micro-batch's gradient into the accumulator
+    p.grad_logits = acc_l;
+    p.grad_scales = acc_s;
+  }
+  if (micro > 0) {  // add the earlier micro-batches' sum; the last one takes the mean
+    p.acc_in_l = acc_l;
+    p.acc_in_s = p.scales_frozen ? nullptr : acc_s;
+    p.acc_scale = last ? static_cast<float>(1.0 / n_micro) : 1.0f;
+  }
+  p.loss_out = loss_dev;
+  prof_begin(L, GSQ_K_BACKWARD, s, slot);
+  e = launch_backward(p, L->grid_bwd, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+  if (lookahead) {
+    L->d_ready = true;
+    L->d_step = t + 1;
+    L->d_tau = nt;
+    L->d_kappa = nk;
+  } else {
+    L->d_ready = false;
+  }
+  L->mb_step = step;
+  L->mb_next = last ? 0 : micro + 1;
+  L->mb_count = n_micro;
   return GSQ_OK;
 }
 

@@ -524,7 +524,7 @@ struct BwdOcc<2> {
   static constexpr int value = 3;
 };
 
-template <class Rx, bool kExport, bool kShift>
+template <class Rx, bool kExport, bool kShift, bool kAcc>
 __global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(const EwParams P) {
   constexpr int K = Rx::L;
   float q[kMaxLevels];
@@ -586,7 +586,11 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(c
 #pragma unroll
       for (int k = 0; k < K; ++k) {
         // dL/dl_k = (kappa/tau) G s dw~/dl_k
-        const float2 dl = mul2(A, rx.dsoft(k));
+        float2 dl = mul2(A, rx.dsoft(k));
+        if (kAcc) {  // gradient accumulation: (this micro-batch + earlier ones) * scale
+          const float2 a = reinterpret_cast<const float2*>(P.acc_in_l + k * P.n)[2 * qc + pr];
+          dl = mul2(add2(dl, a), f2(P.acc_scale));
+        }
         if (kExport) {
           m[k][2 * pr] = dl.x;
           m[k][2 * pr + 1] = dl.y;
@@ -603,9 +607,11 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(c
         }
       }
     }
-    const float ds = group_sum(ds2.x + ds2.y, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
+    float ds = group_sum(ds2.x + ds2.y, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
+    if (kAcc && P.acc_in_s) ds = (ds + P.acc_in_s[gidx]) * P.acc_scale;
 
     if (kExport) {
+      if (kAcc) __syncwarp();  // every lane has read acc_in_s before its group leader rewrites it
       if (active) {
         if (P.grad_logits) {
 #pragma unroll
@@ -615,28 +621,30 @@ __global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(c
         }
         if (P.grad_scales && !P.scales_frozen && (lane & (seg - 1)) == 0) P.grad_scales[gidx] = ds;
       }
-      continue;
-    }
-
-    if (!P.scales_frozen) {
-      const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
-      s = fmaf(-P.lrwd_s, s, s) - lr_sign(P.lr_s, c);
-      ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
+    } else {
+      if (!P.scales_frozen) {
+        const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
+        s = fmaf(-P.lrwd_s, s, s) - lr_sign(P.lr_s, c);
+        ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
+      }
+      if (active) {
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+          __stcs(reinterpret_cast<float4*>(P.logits + k * P.n) + qi,
+                 make_float4(l[k][0], l[k][1], l[k][2], l[k][3]));
+          __stcs(reinterpret_cast<float4*>(P.m_logits + k * P.n) + qi,
+                 make_float4(m[k][0], m[k][1], m[k][2], m[k][3]));
+        }
+        if (!P.scales_frozen && (lane & (seg - 1)) == 0) {
+          P.scales[gidx] = s;
+          P.m_scales[gidx] = ms;
+        }
+      }
     }
     if (active) {
-#pragma unroll
-      for (int k = 0; k < K; ++k) {
-        __stcs(reinterpret_cast<float4*>(P.logits + k * P.n) + qi,
-               make_float4(l[k][0], l[k][1], l[k][2], l[k][3]));
-        __stcs(reinterpret_cast<float4*>(P.m_logits + k * P.n) + qi,
-               make_float4(m[k][0], m[k][1], m[k][2], m[k][3]));
-      }
-      if (!P.scales_frozen && (lane & (seg - 1)) == 0) {
-        P.scales[gidx] = s;
-        P.m_scales[gidx] = ms;
-      }
       if (P.lookahead) {
-        // forward of step t+1 from the updated logits and scale (Alg. 1)
+        // forward of the next pass from the (updated, or in export mode unchanged)
+        // logits and scale (Alg. 1)
         float d[4];
 #pragma unroll
         for (int pr = 0; pr < 2; ++pr) {
@@ -1068,11 +1076,12 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
 
 template <class Rx, bool kShift>
 void set_max_smem_carveout() {
-  cudaFuncSetAttribute(k_forward<Rx, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
-  cudaFuncSetAttribute(k_backward<Rx, false, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                       0);
-  cudaFuncSetAttribute(k_backward<Rx, true, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                       0);
+  const auto attr = cudaFuncAttributePreferredSharedMemoryCarveout;
+  cudaFuncSetAttribute(k_forward<Rx, kShift>, attr, 0);
+  cudaFuncSetAttribute(k_backward<Rx, false, kShift, false>, attr, 0);
+  cudaFuncSetAttribute(k_backward<Rx, true, kShift, false>, attr, 0);
+  cudaFuncSetAttribute(k_backward<Rx, false, kShift, true>, attr, 0);
+  cudaFuncSetAttribute(k_backward<Rx, true, kShift, true>, attr, 0);
 }
 
 int grid_for(const void* fn, int num_sms, int threads) {
@@ -1127,7 +1136,7 @@ int ew_grid_size(int K, int which, int num_sms, int mode) {
     constexpr bool SH = decltype(sh)::value;
     set_max_smem_carveout<Rx, SH>();
     g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<Rx, SH>), num_sms, kEwThreads)
-                   : grid_for(reinterpret_cast<const void*>(k_backward<Rx, false, SH>), num_sms,
+                   : grid_for(reinterpret_cast<const void*>(k_backward<Rx, false, SH, false>), num_sms,
                               kEwThreads);
   });
   return g;
@@ -1143,13 +1152,16 @@ cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s) {
 
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
   const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
+  const bool acc = p.acc_in_l != nullptr;
   const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
     using Rx = typename decltype(rx)::type;
     constexpr bool SH = decltype(sh)::value;
     if (export_mode)
-      k_backward<Rx, true, SH><<<grid, kEwThreads, 0, s>>>(p);
+      acc ? k_backward<Rx, true, SH, true><<<grid, kEwThreads, 0, s>>>(p)
+          : k_backward<Rx, true, SH, false><<<grid, kEwThreads, 0, s>>>(p);
     else
-      k_backward<Rx, false, SH><<<grid, kEwThreads, 0, s>>>(p);
+      acc ? k_backward<Rx, false, SH, true><<<grid, kEwThreads, 0, s>>>(p)
+          : k_backward<Rx, false, SH, false><<<grid, kEwThreads, 0, s>>>(p);
   });
   return e != cudaSuccess ? e : cudaGetLastError();
 }

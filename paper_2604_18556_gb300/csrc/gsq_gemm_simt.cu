@@ -98,7 +98,45 @@ __global__ void k_symmetrize(const float* H, void* out, int C) {
   }
 }
 
+// Tokens of one micro-batch to the tensor-core operands: Xb[e][t][c] and
+// Xt[e][c][t] = bf16(X[e][t][c]), through a 32 x 32 shared tile so both writes
+// are coalesced.  T and C are the micro-batch's tokens and the input width;
+// ldt is the row length of Xt (the workspace's maximum token count).
+__global__ void k_tokens_bf16(const float* X, __nv_bfloat16* Xb, __nv_bfloat16* Xt, int T, int C,
+                              int ldt) {
+  __shared__ __nv_bfloat16 tile[32][34];
+  const int e = blockIdx.z;
+  const int t0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  const float* Xe = X + static_cast<int64_t>(e) * T * C;
+  __nv_bfloat16* Xbe = Xb + static_cast<int64_t>(e) * T * C;
+  __nv_bfloat16* Xte = Xt + static_cast<int64_t>(e) * C * ldt;
+  for (int r = ty; r < 32; r += 8) {
+    const int t = t0 + r, c = c0 + tx;
+    __nv_bfloat16 v = __float2bfloat16_rn(0.0f);
+    if (t < T && c < C) {
+      v = __float2bfloat16_rn(Xe[static_cast<int64_t>(t) * C + c]);
+      Xbe[static_cast<int64_t>(t) * C + c] = v;
+    }
+    tile[r][tx] = v;
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int c = c0 + r, t = t0 + tx;
+    if (t < T && c < C) Xte[static_cast<int64_t>(c) * ldt + t] = tile[tx][r];
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
+                               cudaStream_t s) {
+  if (E <= 0 || T <= 0 || C <= 0) return cudaSuccess;
+  dim3 grid((C + 31) / 32, (T + 31) / 32, E), block(32, 8);
+  k_tokens_bf16<<<grid, block, 0, s>>>(X, static_cast<__nv_bfloat16*>(Xb),
+                                       static_cast<__nv_bfloat16*>(Xt), T, C, ldt);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_simt_gemm(const SimtGemm& g, cudaStream_t s) {
   dim3 grid((g.N + BN - 1) / BN, (g.M + BM - 1) / BM, g.batch);

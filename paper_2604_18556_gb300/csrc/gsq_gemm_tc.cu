@@ -18,6 +18,7 @@
 // workspace flags, waits (bounded) for its own in-flight copies, frees its TMEM
 // and returns.
 #include <cuda.h>
+#include <cuda_bf16.h>
 
 #include "gsq_internal.h"
 
@@ -45,8 +46,9 @@ struct TcCfg {
 };
 
 struct TcArgs {
-  int E, R, C;
-  float* G;
+  int E, M, N, K;
+  void* out;      // [E][M][N], fp32 or bf16
+  int out_bf16;
   float alpha;
   DevFlags* flags;
 };
@@ -212,9 +214,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int Mt = (args.R + TC_BM - 1) / TC_BM;
-  const int Nt = (args.C + TC_BN - 1) / TC_BN;
-  const int KB = (args.C + TC_BK - 1) / TC_BK;
+  const int Mt = (args.M + TC_BM - 1) / TC_BM;
+  const int Nt = (args.N + TC_BN - 1) / TC_BN;
+  const int KB = (args.K + TC_BK - 1) / TC_BK;
   static_assert(TC_STAGES >= 2, "pipeline depth");
   const int tiles = args.E * Mt * Nt;
 
@@ -230,8 +232,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
         int e, m, n;
         tile_coords(tile, Mt, Nt, e, m, n);
-        const int arow = e * args.R + m * TC_BM;
-        const int brow = e * args.C + n * TC_BN;
+        const int arow = e * args.M + m * TC_BM;
+        const int brow = e * args.N + n * TC_BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(empty_bar + stage, phase ^ 1u, abort_flag)) {
             ok = false;
@@ -306,21 +308,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       tile_coords(tile, Mt, Nt, e, m, n);
       const int row = m * TC_BM + quarter * 32 + lane;
       const int col0 = n * TC_BN;
-      float* grow = args.G + (static_cast<int64_t>(e) * args.R + row) * args.C;
+      const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
       const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * TC_BN) +
                              (static_cast<uint32_t>(quarter * 32) << 16);
 #pragma unroll 1
       for (int c = 0; c < TC_BN; c += 16) {
         float v[16];
         tmem_ld16(taddr + c, v);
-        if (row < args.R) {
+        if (row < args.M) {
 #pragma unroll
           for (int j = 0; j < 16; j += 4) {
             const int col = col0 + c + j;
-            if (col < args.C)
-              *reinterpret_cast<float4*>(grow + col) =
-                  make_float4(args.alpha * v[j], args.alpha * v[j + 1], args.alpha * v[j + 2],
-                              args.alpha * v[j + 3]);
+            if (col < args.N) {
+              const float4 o = make_float4(args.alpha * v[j], args.alpha * v[j + 1],
+                                           args.alpha * v[j + 2], args.alpha * v[j + 3]);
+              if (args.out_bf16) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(o.x, o.y);
+                const __nv_bfloat162 hi = __floats2bfloat162_rn(o.z, o.w);
+                uint2 raw;
+                raw.x = *reinterpret_cast<const uint32_t*>(&lo);
+                raw.y = *reinterpret_cast<const uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(args.out) + obase + col) = raw;
+              } else {
+                *reinterpret_cast<float4*>(static_cast<float*>(args.out) + obase + col) = o;
+              }
+            }
           }
         }
       }
@@ -396,19 +408,22 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
     attr_done = true;
   }
   CUtensorMap ta, tb;
-  if (!encode_kmajor_bf16(&ta, g.D, static_cast<uint64_t>(g.C),
-                          static_cast<uint64_t>(g.E) * g.R, TC_BM) ||
-      !encode_kmajor_bf16(&tb, g.H, static_cast<uint64_t>(g.C),
-                          static_cast<uint64_t>(g.E) * g.C, BN))
+  if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;  // 16-B rows; 8/16-B stores
+  if (!encode_kmajor_bf16(&ta, g.A, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.M, TC_BM) ||
+      !encode_kmajor_bf16(&tb, g.B, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.N, BN))
     return cudaErrorInvalidValue;
   TcArgs a;
   a.E = g.E;
-  a.R = g.R;
-  a.C = g.C;
-  a.G = g.G;
+  a.M = g.M;
+  a.N = g.N;
+  a.K = g.K;
+  a.out = g.out;
+  a.out_bf16 = g.out_bf16;
   a.alpha = g.alpha;
   a.flags = g.flags;
-  const int Mt = (g.R + TC_BM - 1) / TC_BM, Nt = (g.C + BN - 1) / BN;
+  const int Mt = (g.M + TC_BM - 1) / TC_BM, Nt = (g.N + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
   k_tc_gemm<BN><<<grid, TC_THREADS, TcCfg<BN>::kSmemBytes, s>>>(ta, tb, a);
@@ -419,13 +434,13 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
 
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
 
-int tc_gemm_tile_n(int E, int R, int C, int num_sms) {
+int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
   // 128 x 256 tiles unless their last wave leaves many SMs idle and 128 x 128
   // tiles balance clearly better (e.g. a 4096 x 4096 layer: 3.37 waves of 256-wide
   // tiles on 152 SMs, 6.74 waves of 128-wide ones).
-  const int64_t mt = (R + TC_BM - 1) / TC_BM;
-  const double b256 = wave_balance(static_cast<int64_t>(E) * mt * ((C + 255) / 256), num_sms);
-  const double b128 = wave_balance(static_cast<int64_t>(E) * mt * ((C + 127) / 128), num_sms);
+  const int64_t mt = (M + TC_BM - 1) / TC_BM;
+  const double b256 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 255) / 256), num_sms);
+  const double b128 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 127) / 128), num_sms);
   // Measured on GB300: 128-wide tiles lose more to the narrower MMA than they
   // gain in balance (4096 x 4096 layer: 142 us vs 114 us), so 256 stays the
   // choice unless the balance gap is extreme.
@@ -433,7 +448,7 @@ int tc_gemm_tile_n(int E, int R, int C, int num_sms) {
 }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
-  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.R, g.C, num_sms);
+  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms);
   return bn == 128 ? launch_tc_gemm_bn<128>(g, num_sms, s) : launch_tc_gemm_bn<256>(g, num_sms, s);
 }
 

@@ -66,6 +66,11 @@ struct EwParams {
   // outputs
   float* grad_logits;  // export mode: [K][n]
   float* grad_scales;  // export mode: [n/group]
+  // gradient accumulation over micro-batches: when set, every gradient becomes
+  // (this pass's + acc_in) * acc_scale before export or the Lion update
+  const float* acc_in_l;  // [K][n] or null
+  const float* acc_in_s;  // [n/group] or null
+  float acc_scale;
   float* what;         // forward: optional W^ export [n]
   double* loss_partials;
   DevFlags* flags;
@@ -163,20 +168,27 @@ cudaError_t launch_simt_gemm(const SimtGemm& g, cudaStream_t s);
 // H_out[e] = (H[e] + H[e]^T) / 2 converted to bf16 (out_bf16=1) or fp32.
 cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_bf16,
                               cudaStream_t s);
+// Xb[e] = bf16(X[e]) ([T][C]) and Xt[e] = bf16(X[e])^T ([C][ldt], first T columns).
+cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
+                               cudaStream_t s);
 
 // tcgen05 / TMA bf16 GEMM: G[e] = alpha * D[e] (R x C, bf16, row-major) *
 // H[e]^T (C x C, bf16, row-major; symmetric so H^T = H), fp32 out.
+// out[e][m][n] = alpha * sum_k A[e][m][k] * B[e][n][k], bf16 operands (both
+// K-major, rows of K elements), fp32 accumulation, fp32 or bf16 output.
+// Needs K % 8 == 0 and N % 4 == 0.
 struct TcGemm {
-  int E, R, C;
-  const void* D;
-  const void* H;
-  float* G;
+  int E, M, N, K;
+  const void* A;   // [E*M][K] bf16
+  const void* B;   // [E*N][K] bf16
+  void* out;       // [E][M][N]
+  int out_bf16;
   float alpha;
   DevFlags* flags;
   int tile_n;  // 0: choose 128 or 256 by wave balance
 };
 bool tc_gemm_supported(int device);
-int tc_gemm_tile_n(int E, int R, int C, int num_sms);
+int tc_gemm_tile_n(int E, int M, int N, int num_sms);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 
 }  // namespace gsq

@@ -25,7 +25,7 @@ GSQ_OK, GSQ_ERR_INVALID_ARG, GSQ_ERR_SHAPE, GSQ_ERR_WORKSPACE, GSQ_ERR_CUDA = 0,
 GSQ_ERR_NONFINITE, GSQ_ERR_STATE, GSQ_ERR_TIMEOUT, GSQ_ERR_INJECTED, GSQ_ERR_UNSUPPORTED = 5, 6, 7, 8, 9
 GSQ_MAX_LEVELS = 8
 GSQ_DTYPE_F32, GSQ_DTYPE_BF16 = 0, 1
-GSQ_CALIB_H, GSQ_CALIB_X = 0, 1
+GSQ_CALIB_H, GSQ_CALIB_X, GSQ_CALIB_BATCHES = 0, 1, 2
 GSQ_SCALE_GROUP, GSQ_SCALE_KQUANT2 = 0, 1
 GSQ_GEMM_BF16, GSQ_GEMM_F32 = 0, 1
 GSQ_FLAG_NO_NOISE = 1
@@ -34,13 +34,14 @@ PARAM_MODES = {"full": GSQ_PARAM_FULL, "shift5": GSQ_PARAM_SHIFT5, "mask_sign": 
 (GSQ_T_LOGITS, GSQ_T_SCALES, GSQ_T_MOM_LOGITS, GSQ_T_MOM_SCALES, GSQ_T_D, GSQ_T_G, GSQ_T_W,
  GSQ_T_H, GSQ_T_KQ_D, GSQ_T_KQ_SC, GSQ_T_J0) = range(11)
 (GSQ_K_FORWARD, GSQ_K_GEMM, GSQ_K_BACKWARD, GSQ_K_PROJECT, GSQ_K_PACK, GSQ_K_INIT) = range(6)
-GSQ_K_COUNT = 6
-KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init"]
+GSQ_K_COUNT = 7
+KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init", "tokens"]
 
 EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "gsq_project",
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
             "gsq_sync_status", "gsq_profile_enable", "gsq_profile_read", "gsq_destroy",
-            "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc", "gsq_init_logits"]
+            "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc", "gsq_init_logits",
+            "gsq_step_tokens"]
 
 
 class gsq_layer_desc(Structure):
@@ -101,6 +102,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "gsq_version": (c_char_p, []),
         "gsq_backward_update_noalloc": (c_int32, [POINTER(gsq_backward_args), P]),
         "gsq_init_logits": (c_int32, [P, P, P, c_float, c_float, P]),
+        "gsq_step_tokens": (c_int32, [P, c_uint64, c_uint32, c_uint32, c_float, c_float, c_float,
+                                      c_float, P, c_int64, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -142,6 +145,13 @@ def gsq_step(handle: int, step: int, tau: float, kappa: float, next_tau: float, 
 
 def gsq_forward(handle: int, step: int, tau: float, kappa: float, stream: int, what_ptr=None) -> None:
     _check(_lib.gsq_forward(handle, step, tau, kappa, stream, what_ptr))
+
+
+def gsq_step_tokens(handle: int, step: int, micro: int, n_micro: int, tau: float, kappa: float,
+                    next_tau: float, next_kappa: float, X_ptr, n_tokens: int, stream: int,
+                    loss_ptr=None) -> None:
+    _check(_lib.gsq_step_tokens(handle, step, micro, n_micro, tau, kappa, next_tau, next_kappa,
+                                X_ptr, n_tokens, stream, loss_ptr))
 
 
 def gsq_init_logits(handle: int, codes_ptr, eps_ptr, alpha: float, sigma: float, stream: int) -> None:
@@ -247,12 +257,17 @@ class Layer:
 
     def __init__(self, W, calib, grid: Sequence[float], group_size: int, *, calib_kind: str = "H",
                  scale_mode: str = "group", gemm: str = "bf16", param: str = "full", stream=None,
-                 **hyper):
+                 tokens_per_batch: int = 0, **hyper):
+        """calib_kind "batches": no calibration at init (calib may be None); every
+        micro-batch brings up to tokens_per_batch tokens through step_tokens."""
         import torch
         self._torch = torch
-        assert W.is_cuda and calib.is_cuda and W.dim() == 3 and calib.dim() == 3
+        batches = calib_kind == "batches"
+        assert W.is_cuda and W.dim() == 3
+        if not batches:
+            assert calib is not None and calib.is_cuda and calib.dim() == 3
+            calib = calib.contiguous().float()
         W = W.contiguous()
-        calib = calib.contiguous().float()
         E, R, C = W.shape
         self.shape = (E, R, C)
         self.K = len(grid)
@@ -263,9 +278,9 @@ class Layer:
         self.desc = make_desc(
             experts=E, rows=R, cols=C, grid=grid, group_size=group_size,
             w_dtype=GSQ_DTYPE_BF16 if W.dtype == torch.bfloat16 else GSQ_DTYPE_F32,
-            W_ptr=_ptr(W), calib_ptr=_ptr(calib),
-            calib_kind=GSQ_CALIB_X if calib_kind == "X" else GSQ_CALIB_H,
-            n_tokens=calib.shape[1] if calib_kind == "X" else 0,
+            W_ptr=_ptr(W), calib_ptr=_ptr(calib) if not batches else 0,
+            calib_kind={"X": GSQ_CALIB_X, "batches": GSQ_CALIB_BATCHES}.get(calib_kind, GSQ_CALIB_H),
+            n_tokens=calib.shape[1] if calib_kind == "X" else (tokens_per_batch if batches else 0),
             scale_mode=GSQ_SCALE_KQUANT2 if scale_mode == "kquant2" else GSQ_SCALE_GROUP,
             gemm=GSQ_GEMM_F32 if gemm == "f32" else GSQ_GEMM_BF16,
             param_mode=PARAM_MODES[param], **hyper)
@@ -286,6 +301,14 @@ class Layer:
              next_kappa: float = 1.0, loss=None, grad_logits=None, grad_scales=None) -> None:
         gsq_step(self.handle, t, tau, kappa, next_tau, next_kappa, self._stream(), _ptr(loss),
                  _ptr(grad_logits), _ptr(grad_scales))
+
+    def step_tokens(self, step: int, micro: int, n_micro: int, tau: float, X, kappa: float = 1.0,
+                    next_tau: float = 0.0, next_kappa: float = 1.0, loss=None) -> None:
+        """One micro-batch (tokens X: fp32 [E, T, C] on the device) of a step with
+        gradient accumulation; the update follows the last micro-batch."""
+        X = X.contiguous()
+        gsq_step_tokens(self.handle, step, micro, n_micro, tau, kappa, next_tau, next_kappa,
+                        _ptr(X), X.shape[1], self._stream(), _ptr(loss))
 
     def forward(self, t: int, tau: float, kappa: float = 1.0, what=None) -> None:
         gsq_forward(self.handle, t, tau, kappa, self._stream(), _ptr(what))

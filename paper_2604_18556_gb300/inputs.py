@@ -80,6 +80,20 @@ def make_tokens(w: Workload, device="cpu") -> torch.Tensor:
     return X
 
 
+def make_token_batch(w: Workload, step: int, micro: int, device="cpu") -> torch.Tensor:
+    """Tokens of micro-batch `micro` of step `step` for a per-step-batch workload:
+    [E, w.tokens, C] fp32, with the layer's outlier channels."""
+    X = torch.empty((w.experts, w.tokens, w.cols), dtype=torch.float32, device=device)
+    for e in range(w.experts):
+        g = _gen(device, w.data_seed + _X_ID + 17 * e + 7919 * (step * max(w.micro, 1) + micro + 1))
+        x = _token_chunk(w, g, w.tokens, device)
+        if w.outliers:
+            ch = _outlier_channels(w, e, device)
+            x[:, ch] *= w.outlier_scale
+        X[e] = x
+    return X
+
+
 def make_gram(w: Workload, device="cpu", chunk: int = 8192) -> torch.Tensor:
     """H = X^T X as [E, C, C] fp32, built chunk by chunk with TF32 off."""
     prev = torch.backends.cuda.matmul.allow_tf32

@@ -147,20 +147,23 @@ class Case:
         self.W = inputs.make_weight(w, device=device)
         if w.calib == "X":
             self.calib = inputs.make_tokens(w, device=device)
+        elif w.calib == "batches":
+            self.calib = None                      # tokens arrive with every micro-batch
         else:
             self.calib = inputs.make_gram(w, device=device)
         hyper = dict(init_bias=w.init_bias, seed=w.seed if seed is None else seed,
                      lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise)
         self.layer = g.Layer(self.W, self.calib, w.grid, w.group, calib_kind=w.calib,
-                             scale_mode=w.scale_mode, gemm=gemm, param=w.param, **hyper)
+                             scale_mode=w.scale_mode, gemm=gemm, param=w.param,
+                             tokens_per_batch=w.tokens if w.calib == "batches" else 0, **hyper)
         self.prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float),
                               group=w.group, seed=hyper["seed"], scale_mode=w.scale_mode,
                               lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1,
                               beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
                               noise=noise, shift=w.param == "shift5",
                               mask_sign=w.param == "mask_sign")
-        if keep_calib_host:
+        if keep_calib_host and self.calib is not None:
             host = self.calib.double().cpu().numpy()
             if w.calib == "X":
                 self.prob.X = host

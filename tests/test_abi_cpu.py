@@ -79,20 +79,26 @@ def test_workspace_size_formula(lib):
     for w in WORKLOADS.values():
         d = lib.make_desc(experts=w.experts, rows=w.rows, cols=w.cols, grid=w.grid,
                           group_size=w.group, w_dtype=lib.GSQ_DTYPE_F32 if w.w_dtype == "f32" else lib.GSQ_DTYPE_BF16,
-                          calib_kind=lib.GSQ_CALIB_X if w.calib == "X" else lib.GSQ_CALIB_H,
-                          n_tokens=w.tokens if w.calib == "X" else 0,
+                          calib_kind={"X": lib.GSQ_CALIB_X, "batches": lib.GSQ_CALIB_BATCHES}.get(
+                              w.calib, lib.GSQ_CALIB_H),
+                          n_tokens=w.tokens if w.calib in ("X", "batches") else 0,
                           scale_mode=lib.GSQ_SCALE_KQUANT2 if w.scale_mode == "kquant2" else lib.GSQ_SCALE_GROUP,
                           lr_scales=w.lr_scales,
                           param_mode=lib.PARAM_MODES[w.param])
         n, L = w.n, w.L
         expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * L * n) + 2 * _align(4 * n // w.group)
-        expect += _align(n * w.w_bytes()) + _align(w.experts * w.cols ** 2 * 2) + _align(2 * n) + _align(4 * n)
+        H = 0 if w.calib == "batches" else _align(w.experts * w.cols ** 2 * 2)
+        expect += _align(n * w.w_bytes()) + H + _align(2 * n) + _align(4 * n)
         if w.scale_mode == "kquant2":
             expect += _align(2 * n // 256) + _align(n // 16)
         if w.calib == "X":
             expect += _align(4 * w.experts * w.cols ** 2)
         if w.param == "shift5":
             expect += _align(n)                                    # j0, one byte per weight
+        if w.calib == "batches":                                   # bf16 X, X^T, Y; accumulators
+            et = w.experts * w.tokens
+            expect += 2 * _align(2 * et * w.cols) + _align(2 * et * w.rows)
+            expect += _align(4 * L * n) + _align(4 * n // w.group)
         assert lib.gsq_workspace_size(d) == expect, w.name
     # the largest workload fits comfortably in one GB300's HBM
     big = WORKLOADS["moe64_kquant3"]
@@ -117,6 +123,9 @@ def test_workspace_size_formula(lib):
     (dict(calib_kind=1, n_tokens=0), 1),
     (dict(gemm=5), 1),
     (dict(beta1=1.5), 1),
+    (dict(calib_kind=2, n_tokens=0), 1),         # per-step batches need a token bound
+    (dict(calib_kind=2, n_tokens=12), 1),        # ... that is a multiple of 8
+    (dict(calib_kind=3), 1),
     (dict(param_mode=3), 1),                     # unknown parameterisation
     (dict(param_mode=2), 1),                     # mask x sign needs {-a, 0, a}
     (dict(param_mode=2, grid=(-1.0, 0.0, 2.0)), 1),

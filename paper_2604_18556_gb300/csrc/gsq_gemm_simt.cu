@@ -99,31 +99,48 @@ __global__ void k_symmetrize(const float* H, void* out, int C) {
 }
 
 // Tokens of one micro-batch to the tensor-core operands: Xb[e][t][c] and
-// Xt[e][c][t] = bf16(X[e][t][c]), through a 32 x 32 shared tile so both writes
-// are coalesced.  T and C are the micro-batch's tokens and the input width;
-// ldt is the row length of Xt (the workspace's maximum token count).
-__global__ void k_tokens_bf16(const float* X, __nv_bfloat16* Xb, __nv_bfloat16* Xt, int T, int C,
-                              int ldt) {
-  __shared__ __nv_bfloat16 tile[32][34];
+// Xt[e][c][t] = bf16(X[e][t][c]).  One 64 x 64 tile per block of 256 threads:
+// 16-byte loads along c, 8-byte stores of four bf16 to Xb, the tile through
+// shared memory, then 8-byte stores of four tokens to Xt.  T and C are
+// multiples of 8, so a group of four never straddles an edge.  ldt is the row
+// length of Xt.
+__global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat16* Xb,
+                                                     __nv_bfloat16* Xt, int T, int C, int ldt) {
+  __shared__ __nv_bfloat16 tile[64][68];
   const int e = blockIdx.z;
-  const int t0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
-  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  const int t0 = blockIdx.y * 64, c0 = blockIdx.x * 64;
+  const int tid = threadIdx.x;
+  const int q = (tid & 15) * 4, r0 = tid >> 4;  // 16 groups of four along the tile row
   const float* Xe = X + static_cast<int64_t>(e) * T * C;
   __nv_bfloat16* Xbe = Xb + static_cast<int64_t>(e) * T * C;
   __nv_bfloat16* Xte = Xt + static_cast<int64_t>(e) * C * ldt;
-  for (int r = ty; r < 32; r += 8) {
-    const int t = t0 + r, c = c0 + tx;
-    __nv_bfloat16 v = __float2bfloat16_rn(0.0f);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = r0 + 16 * i, t = t0 + r, c = c0 + q;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (t < T && c < C) v = __ldcs(reinterpret_cast<const float4*>(Xe + static_cast<int64_t>(t) * C + c));
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
     if (t < T && c < C) {
-      v = __float2bfloat16_rn(Xe[static_cast<int64_t>(t) * C + c]);
-      Xbe[static_cast<int64_t>(t) * C + c] = v;
+      uint2 raw;
+      raw.x = *reinterpret_cast<const uint32_t*>(&lo);
+      raw.y = *reinterpret_cast<const uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(Xbe + static_cast<int64_t>(t) * C + c) = raw;
     }
-    tile[r][tx] = v;
+    *reinterpret_cast<__nv_bfloat162*>(&tile[r][q]) = lo;
+    *reinterpret_cast<__nv_bfloat162*>(&tile[r][q + 2]) = hi;
   }
   __syncthreads();
-  for (int r = ty; r < 32; r += 8) {
-    const int c = c0 + r, t = t0 + tx;
-    if (t < T && c < C) Xte[static_cast<int64_t>(c) * ldt + t] = tile[tx][r];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int cr = r0 + 16 * i, c = c0 + cr, t = t0 + q;
+    if (c < C && t < T) {
+      const __nv_bfloat162 lo = __halves2bfloat162(tile[q][cr], tile[q + 1][cr]);
+      const __nv_bfloat162 hi = __halves2bfloat162(tile[q + 2][cr], tile[q + 3][cr]);
+      uint2 raw;
+      raw.x = *reinterpret_cast<const uint32_t*>(&lo);
+      raw.y = *reinterpret_cast<const uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(Xte + static_cast<int64_t>(c) * ldt + t) = raw;
+    }
   }
 }
 
@@ -132,9 +149,10 @@ __global__ void k_tokens_bf16(const float* X, __nv_bfloat16* Xb, __nv_bfloat16* 
 cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
                                cudaStream_t s) {
   if (E <= 0 || T <= 0 || C <= 0) return cudaSuccess;
-  dim3 grid((C + 31) / 32, (T + 31) / 32, E), block(32, 8);
-  k_tokens_bf16<<<grid, block, 0, s>>>(X, static_cast<__nv_bfloat16*>(Xb),
-                                       static_cast<__nv_bfloat16*>(Xt), T, C, ldt);
+  if (T % 8 != 0 || C % 8 != 0 || ldt % 4 != 0) return cudaErrorInvalidValue;
+  dim3 grid((C + 63) / 64, (T + 63) / 64, E);
+  k_tokens_bf16<<<grid, 256, 0, s>>>(X, static_cast<__nv_bfloat16*>(Xb),
+                                     static_cast<__nv_bfloat16*>(Xt), T, C, ldt);
   return cudaGetLastError();
 }
 

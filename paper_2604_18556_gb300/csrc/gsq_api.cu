@@ -24,6 +24,7 @@ namespace {
 constexpr uint64_t kMagic = 0x6773715f6c617972ull;  // "gsq_layr"
 constexpr int kMaxPartials = 16384;
 constexpr int kMaxProfileEvents = 8192;
+constexpr int kGemmGroupN = 8;  // GEMM tile order: 8 output-tile columns per group
 constexpr double kLog2e = 1.4426950408889634;
 
 thread_local std::string g_last_error;
@@ -237,6 +238,7 @@ struct gsq_layer {
   int grid_fwd, grid_bwd;
   bool tc;
   int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
+  int group_n; // column group of the GEMM's tile order
   // pending forward (D valid for these arguments)
   bool d_ready;
   uint64_t d_step;
@@ -387,6 +389,7 @@ gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
     g.alpha = 2.0f;
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = L->tile_n;
+    g.group_n = L->group_n;
     e = launch_tc_gemm(g, L->num_sms, s);
   } else {
     SimtGemm g;
@@ -535,6 +538,11 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128 or 256: override the choice
     const int v = std::atoi(tn);
     if (v == 128 || v == 256) L->tile_n = v;
+  }
+  L->group_n = kGemmGroupN;
+  if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)
+    const int v = std::atoi(gn);
+    if (v >= 0 && v <= 1024) L->group_n = v;
   }
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -720,6 +728,7 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
     TcGemm g;
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = 0;
+    g.group_n = L->group_n;
     g.E = E;
     if (e == cudaSuccess) {  // Y[e] = D[e] X[e]^T  (N = T, K = C), bf16 out
       g.M = R; g.N = T; g.K = C;

@@ -47,6 +47,7 @@ struct TcCfg {
 
 struct TcArgs {
   int E, M, N, K;
+  int group_n;    // tile-order column group (tile_coords)
   void* out;      // [E][M][N], fp32 or bf16
   int out_bf16;
   float alpha;
@@ -161,12 +162,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int Mt, int Nt, int& e, int& m, int& n) {
+// Tile order: per expert, column groups of GN output tiles; within a group n
+// fastest, then m.  The tiles running at the same time then cover a compact
+// block of about (CTAs / GN) rows x GN columns, so both operands are reused from
+// L2: A (the rows) is streamed from HBM once per column group instead of once
+// per column, B (the columns) stays resident while its group runs.
+__device__ __forceinline__ void tile_coords(int tile, int Mt, int Nt, int GN, int& e, int& m,
+                                            int& n) {
   const int per_e = Mt * Nt;
   e = tile / per_e;
   const int r = tile - e * per_e;
-  n = r / Mt;  // m fastest: CTAs running together share the same H rows
-  m = r - n * Mt;
+  const int g = r / (Mt * GN);
+  const int n0 = g * GN;
+  const int gw = min(GN, Nt - n0);
+  const int rr = r - g * Mt * GN;
+  m = rr / gw;
+  n = n0 + (rr - m * gw);
 }
 
 template <int BN>
@@ -231,7 +242,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
         int e, m, n;
-        tile_coords(tile, Mt, Nt, e, m, n);
+        tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
         const int arow = e * args.M + m * TC_BM;
         const int brow = e * args.N + n * TC_BN;
         for (int kb = 0; kb < KB; ++kb) {
@@ -305,7 +316,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
       tc_fence_after();
       int e, m, n;
-      tile_coords(tile, Mt, Nt, e, m, n);
+      tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
       const int row = m * TC_BM + quarter * 32 + lane;
       const int col0 = n * TC_BN;
       const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
@@ -419,6 +430,7 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   a.M = g.M;
   a.N = g.N;
   a.K = g.K;
+  a.group_n = g.group_n > 0 ? g.group_n : (g.N + BN - 1) / BN;
   a.out = g.out;
   a.out_bf16 = g.out_bf16;
   a.alpha = g.alpha;

@@ -185,7 +185,8 @@ struct TcGemm {
   int out_bf16;
   float alpha;
   DevFlags* flags;
-  int tile_n;  // 0: choose 128 or 256 by wave balance
+  int tile_n;   // 0: choose 128 or 256 by wave balance
+  int group_n;  // tile-order column group; <= 0: one group (m fastest across all columns)
 };
 bool tc_gemm_supported(int device);
 int tc_gemm_tile_n(int E, int M, int N, int num_sms);

@@ -535,9 +535,9 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   L->grid_bwd = clamp_grid(ew_grid_size(sh.L, 1, L->num_sms, sh.mode));
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
                              L->num_sms);
-  if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128 or 256: override the choice
+  if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128, 224 or 256: override the choice
     const int v = std::atoi(tn);
-    if (v == 128 || v == 256) L->tile_n = v;
+    if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
   L->group_n = kGemmGroupN;
   if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)

@@ -30,13 +30,15 @@ constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;
 constexpr int TC_THREADS = 192;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
-// Tile shape M = 128 x N = BN (256 or 128) x 64; the pipeline depth fills ~192 KiB.
+// Tile shape M = 128 x N = BN (256, 224 or 128) x 64; the pipeline depth fills ~192 KiB.
 template <int BN>
 struct TcCfg {
   static constexpr int kBBytes = BN * TC_BK * 2;
   static constexpr int kStageBytes = TC_A_BYTES + kBBytes;
   static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
-  static constexpr int kTmemCols = 2 * BN;  // double-buffered fp32 accumulator
+  // double-buffered fp32 accumulator (2 BN columns), allocated as a power of two
+  static constexpr int kTmemCols = 2 * BN <= 256 ? 256 : 512;
+  static constexpr int kAccStride = kTmemCols / 2;  // column offset of the second buffer
   static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
   // kind::f16 instruction descriptor: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1),
   // B bf16 (10-12 = 1), both K-major (bits 15, 16 = 0), N>>3 at 17-22, M>>4 at 24-28.
@@ -280,7 +282,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
         if (!mbar_wait(tempty_bar + acc, acc_phase ^ 1u, abort_flag)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * TC_BN);
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * TcCfg<BN>::kAccStride);
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(full_bar + stage, phase, abort_flag)) {
             ok = false;
@@ -320,7 +322,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int row = m * TC_BM + quarter * 32 + lane;
       const int col0 = n * TC_BN;
       const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
-      const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * TC_BN) +
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * TcCfg<BN>::kAccStride) +
                              (static_cast<uint32_t>(quarter * 32) << 16);
 #pragma unroll 1
       for (int c = 0; c < TC_BN; c += 16) {
@@ -447,21 +449,28 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
 
 int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
-  // 128 x 256 tiles unless their last wave leaves many SMs idle and 128 x 128
-  // tiles balance clearly better (e.g. a 4096 x 4096 layer: 3.37 waves of 256-wide
-  // tiles on 152 SMs, 6.74 waves of 128-wide ones).
+  // Time ~ waves x tile width: 256-wide tiles unless 224-wide ones fill their
+  // waves enough better (a 4096 x 4096 layer: 512 tiles of 256 = 3.37 waves,
+  // rounded up to 4 x 256; 608 tiles of 224 = exactly 4 waves x 224), or unless
+  // 256-wide tiles leave many SMs idle and 128-wide ones balance clearly better.
+  // Measured on GB300: 128-wide tiles lose more to the narrower MMA than they gain
+  // in balance on the 4096 x 4096 layer (142 us vs 114 us).
   const int64_t mt = (M + TC_BM - 1) / TC_BM;
+  auto cost = [&](int bn) {
+    const int64_t tiles = static_cast<int64_t>(E) * mt * ((N + bn - 1) / bn);
+    return static_cast<double>((tiles + num_sms - 1) / num_sms) * bn;
+  };
   const double b256 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 255) / 256), num_sms);
   const double b128 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 127) / 128), num_sms);
-  // Measured on GB300: 128-wide tiles lose more to the narrower MMA than they
-  // gain in balance (4096 x 4096 layer: 142 us vs 114 us), so 256 stays the
-  // choice unless the balance gap is extreme.
-  return (b256 < 0.6 && b128 > b256 + 0.25) ? 128 : 256;
+  if (b256 < 0.6 && b128 > b256 + 0.25) return 128;
+  return cost(224) < 0.95 * cost(256) ? 224 : 256;
 }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
   const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms);
-  return bn == 128 ? launch_tc_gemm_bn<128>(g, num_sms, s) : launch_tc_gemm_bn<256>(g, num_sms, s);
+  if (bn == 128) return launch_tc_gemm_bn<128>(g, num_sms, s);
+  if (bn == 224) return launch_tc_gemm_bn<224>(g, num_sms, s);
+  return launch_tc_gemm_bn<256>(g, num_sms, s);
 }
 
 }  // namespace gsq

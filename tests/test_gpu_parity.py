@@ -232,10 +232,10 @@ def test_trajectory_ternary_full_run():
     assert_close(gpu.scales, st.scales, TOL_F32, "scales after 50 steps")
 
 
-@pytest.mark.parametrize("tile_n", ["128", "256"])
+@pytest.mark.parametrize("tile_n", ["128", "224", "256"])
 @pytest.mark.parametrize("name", ["q_proj", "gate_proj", "moe_kquant"])
 def test_tc_gemm_tile_widths(name, tile_n, monkeypatch):
-    """Both tensor-core tile widths (chosen per layer by wave balance) on ragged
+    """Every tensor-core tile width (chosen per layer by wave balance) on ragged
     shapes, against exact products of the kernel's own bf16 operands."""
     monkeypatch.setenv("GSQ_GEMM_TILE_N", tile_n)
     w = SMALL[name]

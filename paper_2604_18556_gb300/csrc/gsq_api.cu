@@ -324,6 +324,16 @@ EwParams base_params(gsq_layer* L) {
   return p;
 }
 
+// Profiling events; in a stream being captured into a CUDA graph they become
+// event-record nodes, so every replay of the graph re-times its kernels.
+void prof_record(cudaEvent_t ev, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+    cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal);
+  else
+    cudaEventRecord(ev, s);
+}
+
 void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
   slot = -1;
   if (!L->profiling || L->ev_used >= kMaxProfileEvents) return;
@@ -340,14 +350,14 @@ void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
     L->ev_kind.push_back(kind);
   }
   L->ev_kind[i] = kind;
-  cudaEventRecord(L->ev[2 * i], s);
+  prof_record(L->ev[2 * i], s);
   slot = i;
   L->ev_used = i + 1;
 }
 
 void prof_end(gsq_layer* L, int slot, cudaStream_t s) {
   if (slot < 0) return;
-  cudaEventRecord(L->ev[2 * slot + 1], s);
+  prof_record(L->ev[2 * slot + 1], s);
   L->last_stream = s;
 }
 

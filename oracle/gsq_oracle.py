@@ -582,6 +582,41 @@ def project(logits32: np.ndarray, j0=None, levels: int = 0, mask_sign: bool = Fa
 
 
 # ----------------------------------------------------------------------------
+# diagnostics (not part of the step): displacement, saturation, margins
+# ----------------------------------------------------------------------------
+MARGIN_EDGES = np.float32([1e-6, 1e-5, 1e-4, 1e-3, 1e-2, 1e-1, 1.0, 10.0])   # 9 bins
+SHIFT_BINS = 8
+
+
+def diagnostics(prob: Problem, st: RowState, code0, tau: float, kappa: float):
+    """Three diagnostics of the current logits (no noise):
+      * displacement: histogram of |projected code - initial code| in grid steps
+        (App. L's local-shift statistic, measured on the full parameterisation);
+      * saturation: mean over weights of max_k p_k with p = softmax(kappa l / tau)
+        (for mask x sign, of the three-value distribution the two binary instances
+        define), the regime where the logit gradients vanish (App. B);
+      * margins: histogram of the top-two logit gap of the projection (bins split
+        at MARGIN_EDGES, compared in fp32).
+    Returns (displacement counts [8], mean max-probability, margin counts [9])."""
+    codes, margin = project(st.logits, j0=st.j0, levels=prob.levels, mask_sign=prob.mask_sign)
+    disp = np.abs(codes.astype(np.int64) - np.asarray(code0, dtype=np.int64))
+    disp_hist = np.bincount(np.minimum(disp, SHIFT_BINS - 1).reshape(-1), minlength=SHIFT_BINS)
+    l = st.logits.astype(np.float64)
+    if prob.mask_sign:
+        pm = 1.0 / (1.0 + np.exp(-2.0 * kappa * l[0] / tau))
+        pb = 1.0 / (1.0 + np.exp(-2.0 * kappa * l[1] / tau))
+        pmax = np.maximum(np.maximum(pm * (1 - pb), 1 - pm), pm * pb)
+    else:
+        pmax = relax(st.logits, 0.0, tau, kappa).max(axis=0)
+    m = np.asarray(margin, dtype=np.float32).reshape(-1)
+    bins = np.zeros(m.shape, dtype=np.int64)
+    for e in MARGIN_EDGES:
+        bins += (m >= e)
+    margin_hist = np.bincount(bins, minlength=len(MARGIN_EDGES) + 1)
+    return disp_hist, float(pmax.mean()), margin_hist
+
+
+# ----------------------------------------------------------------------------
 # packing (§4.1 symmetric group-wise codes + fp16 scale; §4.4 / App. E K-Quant)
 # ----------------------------------------------------------------------------
 def code_bits(K: int) -> int:

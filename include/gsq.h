@@ -158,6 +158,31 @@ GSQ_API gsq_status gsq_workspace_size(const gsq_layer_desc* desc, size_t* bytes)
 GSQ_API gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t bytes,
                           void* stream, gsq_layer** out);
 
+/* Diagnostics of the current logits (no noise), for monitoring a run; the paper
+ * has no entry point for them but uses the first as the evidence for the local
+ * shift (App. L) and relates the second to vanishing gradients (App. B):
+ *   displacement[d]  number of weights whose projected code is d grid steps
+ *                    from the initial code (RTN, or the codes of
+ *                    gsq_init_logits); d = 7 counts 7 and more;
+ *   margin[b]        number of weights whose top-two logit margin (as
+ *                    gsq_project reports it) falls in bin b: [0, 1e-6),
+ *                    [1e-6, 1e-5), ..., [1, 10), [10, inf);
+ *   mean_max_prob    mean over weights of max_k p_k, p = softmax(kappa l / tau)
+ *                    (mask x sign: the three-value distribution of the two
+ *                    binary instances); near 1 means saturated.
+ * Uses the loss-reduction scratch of the workspace, so it must not overlap a
+ * step of the same layer.  Synchronises `stream`.  Errors: GSQ_ERR_INVALID_ARG,
+ * GSQ_ERR_CUDA. */
+#define GSQ_DIAG_SHIFT_BINS 8
+#define GSQ_DIAG_MARGIN_BINS 9
+typedef struct gsq_diagnostics {
+  int64_t displacement[GSQ_DIAG_SHIFT_BINS];
+  int64_t margin[GSQ_DIAG_MARGIN_BINS];
+  double mean_max_prob;
+} gsq_diagnostics;
+GSQ_API gsq_status gsq_diagnose(gsq_layer* layer, float tau, float kappa, void* stream,
+                        gsq_diagnostics* out);
+
 /* Warm start from a supplied solution (§3.1 "Initialization", Eq. 3-4; App. A),
  * on `stream`, replacing the logits of gsq_init_layer:
  *   l = sigma * (eps + alpha * l_prior), logit momenta = 0, where l_prior is,

@@ -3,6 +3,7 @@
 // the caller's stream and keeps the per-layer bookkeeping (pending look-ahead
 // forward, profiling events).  Never allocates device memory.
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <cmath>
 #include <cstdarg>
@@ -25,6 +26,9 @@ constexpr uint64_t kMagic = 0x6773715f6c617972ull;  // "gsq_layr"
 constexpr int kMaxPartials = 16384;
 constexpr int kMaxProfileEvents = 8192;
 constexpr int kGemmGroupN = 8;  // GEMM tile order: 8 output-tile columns per group
+constexpr size_t kCanaryBytes = 256;
+static_assert(GSQ_DIAG_SHIFT_BINS == kDiagShiftBins && GSQ_DIAG_MARGIN_BINS == kDiagMarginBins,
+              "diagnostics bins");
 constexpr double kLog2e = 1.4426950408889634;
 
 thread_local std::string g_last_error;
@@ -82,7 +86,12 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 struct Layout {
   size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch, j0;
   size_t tok_b, tok_t, Y, acc_l, acc_s;  // per-step token batches (GSQ_CALIB_BATCHES)
+  size_t code0, diag;                     // initial codes and diagnostics counters
   size_t total;
+  // 256 canary bytes after every buffer (written at init, checked by gsq_sync_status)
+  int ncanary;
+  size_t canary[kMaxCanaries];
+  const char* canary_of[kMaxCanaries];
 };
 
 struct Shape {
@@ -119,34 +128,48 @@ Shape shape_of(const gsq_layer_desc& d) {
 Layout layout_of(const Shape& s) {
   Layout L;
   size_t off = 0;
-  auto take = [&](size_t bytes) {
+  L.ncanary = 0;
+  auto take = [&](size_t bytes, const char* name) {
     const size_t o = off;
     off += align256(bytes);
+    L.canary_of[L.ncanary] = name;
+    L.canary[L.ncanary++] = off;
+    off += kCanaryBytes;
     return o;
   };
   const size_t n = static_cast<size_t>(s.n), ng = static_cast<size_t>(s.ng);
-  L.flags = take(sizeof(DevFlags));
-  L.partials = take(sizeof(double) * kMaxPartials);
-  L.logits = take(4 * n * s.L);
-  L.m_logits = take(4 * n * s.L);
-  L.scales = take(4 * ng);
-  L.m_scales = take(4 * ng);
-  L.W = take(n * (s.w_bf16 ? 2 : 4));
-  L.H = s.batches ? off : take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4));
-  L.D = take(n * (s.d_bf16 ? 2 : 4));
-  L.G = take(4 * n);
-  L.kq_d = s.kquant ? take(2 * (n / kSuperBlock)) : off;
-  L.kq_sc = s.kquant ? take(n / kSubBlock) : off;
-  L.hscratch = s.x_mode ? take(static_cast<size_t>(s.E) * s.C * s.C * 4) : off;
-  L.j0 = s.shift ? take(n) : off;
+  L.flags = take(sizeof(DevFlags), "flags");
+  L.partials = take(sizeof(double) * kMaxPartials, "partials");
+  L.logits = take(4 * n * s.L, "logits");
+  L.m_logits = take(4 * n * s.L, "m_logits");
+  L.scales = take(4 * ng, "scales");
+  L.m_scales = take(4 * ng, "m_scales");
+  L.W = take(n * (s.w_bf16 ? 2 : 4), "W");
+  L.H = s.batches ? off
+                  : take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4), "H");
+  L.D = take(n * (s.d_bf16 ? 2 : 4), "D");
+  L.G = take(4 * n, "G");
+  L.kq_d = s.kquant ? take(2 * (n / kSuperBlock), "kq_d") : off;
+  L.kq_sc = s.kquant ? take(n / kSubBlock, "kq_sc") : off;
+  L.hscratch = s.x_mode ? take(static_cast<size_t>(s.E) * s.C * s.C * 4, "hscratch") : off;
+  L.j0 = s.shift ? take(n, "j0") : off;
   const size_t et = static_cast<size_t>(s.E) * static_cast<size_t>(s.T);
-  L.tok_b = s.batches && s.d_bf16 ? take(2 * et * s.C) : off;
-  L.tok_t = s.batches && s.d_bf16 ? take(2 * et * s.C) : off;
-  L.Y = s.batches ? take((s.d_bf16 ? 2 : 4) * et * s.R) : off;
-  L.acc_l = s.batches ? take(4 * n * s.L) : off;
-  L.acc_s = s.batches ? take(4 * ng) : off;
+  L.tok_b = s.batches && s.d_bf16 ? take(2 * et * s.C, "tok_b") : off;
+  L.tok_t = s.batches && s.d_bf16 ? take(2 * et * s.C, "tok_t") : off;
+  L.Y = s.batches ? take((s.d_bf16 ? 2 : 4) * et * s.R, "Y") : off;
+  L.acc_l = s.batches ? take(4 * n * s.L, "acc_l") : off;
+  L.acc_s = s.batches ? take(4 * ng, "acc_s") : off;
+  L.code0 = take(n, "code0");
+  L.diag = take(8 * (kDiagShiftBins + kDiagMarginBins), "diag");
   L.total = off;
   return L;
+}
+
+CanaryList canary_list(const Layout& lay) {
+  CanaryList c;
+  c.count = lay.ncanary;
+  for (int i = 0; i < lay.ncanary; ++i) c.off[i] = lay.canary[i];
+  return c;
 }
 
 bool is_pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
@@ -334,7 +357,13 @@ void prof_record(cudaEvent_t ev, cudaStream_t s) {
     cudaEventRecord(ev, s);
 }
 
+// NVTX range names per kernel kind (visible in nsys / ncu timelines).
+const char* const kKindName[GSQ_K_COUNT] = {"gsq:forward", "gsq:gemm",  "gsq:backward",
+                                            "gsq:project", "gsq:pack",  "gsq:init",
+                                            "gsq:tokens"};
+
 void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
+  nvtxRangePushA(kKindName[kind]);
   slot = -1;
   if (!L->profiling || L->ev_used >= kMaxProfileEvents) return;
   const int i = L->ev_used;
@@ -356,6 +385,7 @@ void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
 }
 
 void prof_end(gsq_layer* L, int slot, cudaStream_t s) {
+  nvtxRangePop();
   if (slot < 0) return;
   prof_record(L->ev[2 * slot + 1], s);
   L->last_stream = s;
@@ -563,6 +593,8 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   };
   if ((e = cudaMemsetAsync(flags, 0, sizeof(DevFlags), s)) != cudaSuccess)
     return bail(cuda_fail(e, "clear flags"));
+  if ((e = launch_canaries(L->ws, canary_list(lay), 1, flags, s)) != cudaSuccess)
+    return bail(cuda_fail(e, "write canaries"));
   const size_t wbytes = static_cast<size_t>(sh.n) * (sh.w_bf16 ? 2 : 4);
   if ((e = cudaMemcpyAsync(L->ws + lay.W, desc->W, wbytes, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
     return bail(cuda_fail(e, "copy W"));
@@ -621,6 +653,7 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   ip.kq_d = sh.kquant ? reinterpret_cast<uint16_t*>(L->ws + lay.kq_d) : nullptr;
   ip.kq_sc = sh.kquant ? reinterpret_cast<int8_t*>(L->ws + lay.kq_sc) : nullptr;
   ip.j0 = sh.shift ? L->ws + lay.j0 : nullptr;
+  ip.code0 = L->ws + lay.code0;
   ip.mask_sign = sh.mask_sign;
   if ((e = launch_init_state(ip, L->num_sms, s)) != cudaSuccess) return bail(cuda_fail(e, "init state"));
   prof_end(L, slot, s);
@@ -856,12 +889,52 @@ gsq_status gsq_init_logits(gsq_layer* L, const uint8_t* codes_dev, const float* 
   p.logits = fptr(L, L->lay.logits);
   p.m_logits = fptr(L, L->lay.m_logits);
   p.j0 = sh.shift ? L->ws + L->lay.j0 : nullptr;
+  p.code0 = L->ws + L->lay.code0;
   int slot;
   prof_begin(L, GSQ_K_INIT, s, slot);
   const cudaError_t e = launch_init_from_codes(p, L->num_sms, s);
   prof_end(L, slot, s);
   if (e != cudaSuccess) return cuda_fail(e, "init from codes");
   L->d_ready = false;
+  return GSQ_OK;
+}
+
+gsq_status gsq_diagnose(gsq_layer* L, float tau, float kappa, void* stream, gsq_diagnostics* out) {
+  GSQ_INJECT("gsq_diagnose");
+  if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (!out) return fail(GSQ_ERR_INVALID_ARG, "out is NULL");
+  if (!(tau > 0.f) || !std::isfinite(tau) || !std::isfinite(kappa))
+    return fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");
+  DeviceGuard guard(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Shape& sh = L->shape;
+  DiagParams p;
+  p.n = sh.n;
+  p.K = sh.L;
+  p.nlev = sh.K;
+  p.mask_sign = sh.mask_sign;
+  p.j0 = sh.shift ? L->ws + L->lay.j0 : nullptr;
+  p.logits = fptr(L, L->lay.logits);
+  p.code0 = L->ws + L->lay.code0;
+  p.kappa_over_tau = static_cast<double>(kappa) / tau;
+  p.hist = reinterpret_cast<unsigned long long*>(L->ws + L->lay.diag);
+  p.partials = reinterpret_cast<double*>(L->ws + L->lay.partials);
+  const int grid = L->grid_fwd;
+  unsigned long long hist[kDiagShiftBins + kDiagMarginBins];
+  std::vector<double> parts(static_cast<size_t>(grid));
+  cudaError_t e = cudaMemsetAsync(p.hist, 0, sizeof(hist), s);
+  if (e == cudaSuccess) e = launch_diagnose(p, grid, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(hist, p.hist, sizeof(hist), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(parts.data(), p.partials, sizeof(double) * grid, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "diagnostics");
+  for (int i = 0; i < kDiagShiftBins; ++i) out->displacement[i] = static_cast<int64_t>(hist[i]);
+  for (int i = 0; i < kDiagMarginBins; ++i)
+    out->margin[i] = static_cast<int64_t>(hist[kDiagShiftBins + i]);
+  double sum = 0.0;
+  for (int b = 0; b < grid; ++b) sum += parts[b];
+  out->mean_max_prob = sum / static_cast<double>(sh.n);
   return GSQ_OK;
 }
 
@@ -970,7 +1043,10 @@ gsq_status gsq_sync_status(gsq_layer* L, void* stream) {
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
   DeviceGuard guard(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e = cudaStreamSynchronize(s);
+  DevFlags* cflags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+  cudaError_t e = launch_canaries(L->ws, canary_list(L->lay), 0, cflags, s);
+  if (e != cudaSuccess) return cuda_fail(e, "check canaries");
+  e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "gsq_sync_status");
   DevFlags* flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
   unsigned int err = 0;
@@ -978,6 +1054,11 @@ gsq_status gsq_sync_status(gsq_layer* L, void* stream) {
   if (e != cudaSuccess) return cuda_fail(e, "read error word");
   if (err) {
     cudaMemset(&flags->error, 0, sizeof(err));
+    if ((err & 0xFFFF0000u) == kCanaryError) {
+      const unsigned int i = err & 0xFFFFu;
+      return fail(GSQ_ERR_STATE, "workspace canary after buffer '%s' was overwritten",
+                  i < static_cast<unsigned int>(L->lay.ncanary) ? L->lay.canary_of[i] : "?");
+    }
     return fail(GSQ_ERR_TIMEOUT, "a bounded device-side wait gave up (code 0x%x)", err);
   }
   return GSQ_OK;

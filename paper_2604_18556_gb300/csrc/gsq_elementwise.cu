@@ -711,11 +711,10 @@ __device__ __forceinline__ InitConsts init_consts(const InitParams& P) {
 // Logits of a quad: init_bias on the RTN level (or, with local shift, on the
 // delta = 0 logit, with the RTN index stored as j0); momenta 0.
 __device__ __forceinline__ void write_init_quad(const InitParams& P, int64_t qi, const int (&code)[4]) {
-  if (P.j0) {
-    reinterpret_cast<uint32_t*>(P.j0)[qi] =
-        static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
-        (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
-  }
+  const uint32_t c4 = static_cast<uint32_t>(code[0]) | (static_cast<uint32_t>(code[1]) << 8) |
+                      (static_cast<uint32_t>(code[2]) << 16) | (static_cast<uint32_t>(code[3]) << 24);
+  if (P.j0) reinterpret_cast<uint32_t*>(P.j0)[qi] = c4;
+  if (P.code0) reinterpret_cast<uint32_t*>(P.code0)[qi] = c4;
   if (P.mask_sign) {
     // Eq. 3 on the RTN code (0, 1, 2 for -a, 0, a), times init_bias:
     // l_m = +b if the code is nonzero else -b; l_b = +b, -b or 0 by its sign
@@ -864,6 +863,7 @@ __global__ void __launch_bounds__(kEwThreads) k_init_from_codes(const InitCodesP
       clamped |= static_cast<uint32_t>(c[j]) << (8 * j);
     }
     if (P.j0) reinterpret_cast<uint32_t*>(P.j0)[qi] = clamped;
+    if (P.code0) reinterpret_cast<uint32_t*>(P.code0)[qi] = clamped;
     for (int k = 0; k < L; ++k) {
       float4 e = make_float4(0.f, 0.f, 0.f, 0.f);
       if (P.eps) e = __ldcs(reinterpret_cast<const float4*>(P.eps + k * P.n) + qi);
@@ -1074,6 +1074,58 @@ __global__ void __launch_bounds__(kEwThreads) k_pack_kquant(const PackParams P) 
   }
 }
 
+// ---------------------------------------------------------------------------
+// Diagnostics of the current logits (no noise): histogram of |code - initial
+// code|, histogram of top-two margins (bins split at 1e-6 ... 10, compared in
+// fp32), and per-block sums of the max probability of softmax(kappa l / tau)
+// (of the three-value distribution for mask x sign).  Counts are integers, so
+// their atomics commute; the probability sums go out per block.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kEwThreads) k_diagnose(const DiagParams P) {
+  __shared__ unsigned int hist[kDiagShiftBins + kDiagMarginBins];
+  __shared__ double red[kEwThreads / 32];
+  for (int i = threadIdx.x; i < kDiagShiftBins + kDiagMarginBins; i += blockDim.x) hist[i] = 0u;
+  __syncthreads();
+  const float edges[kDiagMarginBins - 1] = {1e-6f, 1e-5f, 1e-4f, 1e-3f, 1e-2f, 1e-1f, 1.0f, 10.0f};
+  double acc = 0.0;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < P.n; i += stride) {
+    int code;
+    float mg;
+    decide(P, i, code, mg);
+    const int d = abs(code - static_cast<int>(P.code0[i]));
+    atomicAdd(&hist[d < kDiagShiftBins ? d : kDiagShiftBins - 1], 1u);
+    int b = 0;
+#pragma unroll
+    for (int e = 0; e < kDiagMarginBins - 1; ++e) b += mg >= edges[e] ? 1 : 0;
+    atomicAdd(&hist[kDiagShiftBins + b], 1u);
+    double pmax;
+    if (P.mask_sign) {
+      const double pm = 1.0 / (1.0 + exp(-2.0 * P.kappa_over_tau * P.logits[i]));
+      const double pb = 1.0 / (1.0 + exp(-2.0 * P.kappa_over_tau * P.logits[P.n + i]));
+      pmax = fmax(fmax(pm * (1.0 - pb), 1.0 - pm), pm * pb);
+    } else {
+      float lmax = P.logits[i];
+      for (int k = 1; k < P.K; ++k) lmax = fmaxf(lmax, P.logits[k * P.n + i]);
+      double sum = 0.0;
+      for (int k = 0; k < P.K; ++k) sum += exp(P.kappa_over_tau * (P.logits[k * P.n + i] - lmax));
+      pmax = 1.0 / sum;
+    }
+    acc += pmax;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
+    P.partials[blockIdx.x] = s;
+  }
+  for (int i = threadIdx.x; i < kDiagShiftBins + kDiagMarginBins; i += blockDim.x)
+    if (hist[i]) atomicAdd(P.hist + i, static_cast<unsigned long long>(hist[i]));
+}
+
 template <class Rx, bool kShift>
 void set_max_smem_carveout() {
   const auto attr = cudaFuncAttributePreferredSharedMemoryCarveout;
@@ -1193,6 +1245,11 @@ cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16, uns
   const int64_t blocks = (count + 255) / 256;
   const int grid = static_cast<int>(blocks < 4096 ? blocks : 4096);
   k_nonfinite<<<grid, 256, 0, s>>>(x, count, is_bf16, counter);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_diagnose(const DiagParams& p, int grid, cudaStream_t s) {
+  k_diagnose<<<grid, kEwThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

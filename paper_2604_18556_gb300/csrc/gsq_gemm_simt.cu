@@ -144,7 +144,26 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
   }
 }
 
+// One block per canary (256 bytes = 64 words): write the pattern, or compare.
+__global__ void k_canaries(uint8_t* ws, const CanaryList list, int write, DevFlags* flags) {
+  const int i = blockIdx.x;
+  uint32_t* c = reinterpret_cast<uint32_t*>(ws + list.off[i]);
+  const uint32_t pattern = 0x5EED0000u ^ static_cast<uint32_t>(i) * 0x9E3779B1u;
+  if (write) {
+    c[threadIdx.x] = pattern ^ threadIdx.x;
+  } else if (c[threadIdx.x] != (pattern ^ threadIdx.x)) {
+    atomicCAS(&flags->error, 0u, kCanaryError | static_cast<unsigned int>(i));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_canaries(uint8_t* ws, const CanaryList& list, int write, DevFlags* flags,
+                            cudaStream_t s) {
+  if (list.count <= 0) return cudaSuccess;
+  k_canaries<<<list.count, 64, 0, s>>>(ws, list, write, flags);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
                                cudaStream_t s) {

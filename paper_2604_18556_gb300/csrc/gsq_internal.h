@@ -90,6 +90,7 @@ struct InitParams {
   int K;               // grid levels
   int mask_sign;       // logits are the (mask, sign) planes, Eq. 3 from the RTN code
   uint8_t* j0;         // local shift: receives the RTN index; logits then hold 5 planes
+  uint8_t* code0;      // receives the initial grid code of every weight (diagnostics)
   int group;
   int kquant;
   int w_bf16;
@@ -105,6 +106,17 @@ struct InitParams {
 };
 cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s);
 
+// Workspace canaries: 256 bytes after every buffer, written with a fixed word at
+// init and checked later; a mismatch stores kCanaryError | index in flags->error.
+constexpr int kMaxCanaries = 32;
+constexpr unsigned int kCanaryError = 0xCA000000u;
+struct CanaryList {
+  int count;
+  uint64_t off[kMaxCanaries];
+};
+cudaError_t launch_canaries(uint8_t* ws, const CanaryList& list, int write, DevFlags* flags,
+                            cudaStream_t s);
+
 struct InitCodesParams {
   int64_t n;
   int K;               // grid levels
@@ -116,6 +128,7 @@ struct InitCodesParams {
   float* logits;       // [L][n]
   float* m_logits;     // [L][n]
   uint8_t* j0;         // local shift: receives the codes
+  uint8_t* code0;      // receives the codes (initial codes for the diagnostics)
 };
 cudaError_t launch_init_from_codes(const InitCodesParams& p, int num_sms, cudaStream_t s);
 cudaError_t launch_nonfinite_scan(const void* x, int64_t count, int is_bf16,
@@ -132,6 +145,22 @@ struct ProjectParams {
   float* margin;
 };
 cudaError_t launch_project(const ProjectParams& p, int num_sms, cudaStream_t s);
+
+constexpr int kDiagShiftBins = 8;   // |code - initial code| = 0..6, >= 7
+constexpr int kDiagMarginBins = 9;  // margins split at 1e-6, 1e-5, ..., 1, 10
+struct DiagParams {
+  int64_t n;
+  int K;               // logits per weight
+  int nlev;            // grid levels
+  int mask_sign;
+  const uint8_t* j0;   // local shift (null otherwise)
+  const float* logits;
+  const uint8_t* code0;
+  double kappa_over_tau;
+  unsigned long long* hist;  // [kDiagShiftBins + kDiagMarginBins], zeroed by the caller
+  double* partials;          // [grid] sums of the max probability
+};
+cudaError_t launch_diagnose(const DiagParams& p, int grid, cudaStream_t s);
 
 struct PackParams {
   int64_t n;

@@ -12,8 +12,8 @@ from __future__ import annotations
 
 import ctypes
 import os
-from ctypes import (POINTER, Structure, byref, c_char_p, c_float, c_int32, c_int64, c_size_t,
-                    c_uint32, c_uint64, c_void_p)
+from ctypes import (POINTER, Structure, byref, c_char_p, c_double, c_float, c_int32, c_int64,
+                    c_size_t, c_uint32, c_uint64, c_void_p)
 from typing import Optional, Sequence
 
 # GSQ_LIBRARY, if set, names a libgsq.so built elsewhere (same ABI).
@@ -41,7 +41,15 @@ EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
             "gsq_sync_status", "gsq_profile_enable", "gsq_profile_read", "gsq_destroy",
             "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc", "gsq_init_logits",
-            "gsq_step_tokens"]
+            "gsq_step_tokens", "gsq_diagnose"]
+
+
+GSQ_DIAG_SHIFT_BINS, GSQ_DIAG_MARGIN_BINS = 8, 9
+
+
+class gsq_diagnostics(Structure):
+    _fields_ = [("displacement", c_int64 * GSQ_DIAG_SHIFT_BINS),
+                ("margin", c_int64 * GSQ_DIAG_MARGIN_BINS), ("mean_max_prob", c_double)]
 
 
 class gsq_layer_desc(Structure):
@@ -102,6 +110,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "gsq_version": (c_char_p, []),
         "gsq_backward_update_noalloc": (c_int32, [POINTER(gsq_backward_args), P]),
         "gsq_init_logits": (c_int32, [P, P, P, c_float, c_float, P]),
+        "gsq_diagnose": (c_int32, [P, c_float, c_float, P, POINTER(gsq_diagnostics)]),
         "gsq_step_tokens": (c_int32, [P, c_uint64, c_uint32, c_uint32, c_float, c_float, c_float,
                                       c_float, P, c_int64, P, P]),
     }
@@ -152,6 +161,13 @@ def gsq_step_tokens(handle: int, step: int, micro: int, n_micro: int, tau: float
                     loss_ptr=None) -> None:
     _check(_lib.gsq_step_tokens(handle, step, micro, n_micro, tau, kappa, next_tau, next_kappa,
                                 X_ptr, n_tokens, stream, loss_ptr))
+
+
+def gsq_diagnose(handle: int, tau: float, kappa: float, stream: int) -> dict:
+    out = gsq_diagnostics()
+    _check(_lib.gsq_diagnose(handle, tau, kappa, stream, byref(out)))
+    return {"displacement": list(out.displacement), "margin": list(out.margin),
+            "mean_max_prob": out.mean_max_prob}
 
 
 def gsq_init_logits(handle: int, codes_ptr, eps_ptr, alpha: float, sigma: float, stream: int) -> None:
@@ -318,6 +334,10 @@ class Layer:
         codes = codes.contiguous()
         eps = None if eps is None else eps.contiguous()
         gsq_init_logits(self.handle, _ptr(codes), _ptr(eps), alpha, sigma, self._stream())
+
+    def diagnose(self, tau: float, kappa: float = 1.0) -> dict:
+        """Displacement and margin histograms and the mean max-probability (see gsq.h)."""
+        return gsq_diagnose(self.handle, tau, kappa, self._stream())
 
     def project(self, codes=None, margin=None) -> None:
         gsq_project(self.handle, self._stream(), _ptr(codes), _ptr(margin))

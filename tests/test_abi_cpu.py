@@ -44,7 +44,8 @@ def test_every_declared_symbol_is_exported(lib):
         assert getattr(cdll, n) is not None
 
 
-@pytest.mark.parametrize("struct", ["gsq_layer_desc", "gsq_profile", "gsq_backward_args"])
+@pytest.mark.parametrize("struct", ["gsq_layer_desc", "gsq_profile", "gsq_backward_args",
+                                    "gsq_diagnostics"])
 def test_struct_layout_matches_c(lib, tmp_path, struct):
     cls = getattr(lib, struct)
     fields = [f for f, _ in cls._fields_]
@@ -86,19 +87,22 @@ def test_workspace_size_formula(lib):
                           lr_scales=w.lr_scales,
                           param_mode=lib.PARAM_MODES[w.param])
         n, L = w.n, w.L
-        expect = _align(256) + _align(8 * 16384) + 2 * _align(4 * L * n) + 2 * _align(4 * n // w.group)
-        H = 0 if w.calib == "batches" else _align(w.experts * w.cols ** 2 * 2)
-        expect += _align(n * w.w_bytes()) + H + _align(2 * n) + _align(4 * n)
+        # every buffer is 256-byte aligned and followed by a 256-byte canary
+        bufs = [256, 8 * 16384, 4 * L * n, 4 * L * n, 4 * n // w.group, 4 * n // w.group,
+                n * w.w_bytes(), 2 * n, 4 * n]
+        if w.calib != "batches":
+            bufs.append(w.experts * w.cols ** 2 * 2)               # H (bf16)
         if w.scale_mode == "kquant2":
-            expect += _align(2 * n // 256) + _align(n // 16)
+            bufs += [2 * n // 256, n // 16]
         if w.calib == "X":
-            expect += _align(4 * w.experts * w.cols ** 2)
+            bufs.append(4 * w.experts * w.cols ** 2)
         if w.param == "shift5":
-            expect += _align(n)                                    # j0, one byte per weight
+            bufs.append(n)                                         # j0, one byte per weight
         if w.calib == "batches":                                   # bf16 X, X^T, Y; accumulators
             et = w.experts * w.tokens
-            expect += 2 * _align(2 * et * w.cols) + _align(2 * et * w.rows)
-            expect += _align(4 * L * n) + _align(4 * n // w.group)
+            bufs += [2 * et * w.cols, 2 * et * w.cols, 2 * et * w.rows, 4 * L * n, 4 * n // w.group]
+        bufs += [n, 8 * 17]                                        # initial codes; diagnostics
+        expect = sum(_align(b) + 256 for b in bufs)
         assert lib.gsq_workspace_size(d) == expect, w.name
     # the largest workload fits comfortably in one GB300's HBM
     big = WORKLOADS["moe64_kquant3"]
@@ -150,7 +154,7 @@ def test_parameterisations_size_their_logit_planes(lib):
     sh = lib.gsq_workspace_size(_desc(lib, grid=(-1.0, 0.0, 1.0), param_mode=1))
     n = 64 * 256
     assert base - ms == 2 * 4 * n            # logits + momenta, one plane fewer
-    assert sh - base == 2 * 2 * 4 * n + n    # two planes more, plus j0
+    assert sh - base == 2 * 2 * 4 * n + n + 256   # two planes more, plus j0 and its canary
 
 
 def test_init_rejects_bad_buffers_before_cuda(lib):
@@ -179,7 +183,8 @@ def test_handle_checks(lib):
                      (lib._lib.gsq_destroy, (987654321,)),
                      (lib._lib.gsq_sync_status, (None, None)),
                      (lib._lib.gsq_init_logits, (None, 4096, None, 1.0, 1.0, None)),
-                     (lib._lib.gsq_init_logits, (24681357, 4096, None, 1.0, 1.0, None))]:
+                     (lib._lib.gsq_init_logits, (24681357, 4096, None, 1.0, 1.0, None)),
+                     (lib._lib.gsq_diagnose, (None, 1.0, 1.0, None, None))]:
         assert fn(*args) == lib.GSQ_ERR_INVALID_ARG
     assert lib.gsq_version().count(".") == 2
 

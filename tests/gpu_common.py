@@ -98,6 +98,26 @@ def assert_grad_close(got_l, got_s, ref, prob, tau, kappa, tol, what="", q=None)
         assert not bad.any(), (what + " dL/dscales", int(bad.sum()))
 
 
+def mask_sign_grad_factors(ref, prob, tau, kappa):
+    """|dL/dl| / |G| for both planes: (kappa/tau) s a |b~ dm~| and (kappa/tau) s a |m~ db~|."""
+    fw = ref.fw
+    a = float(prob.grid[2])
+    gm = O.binary_gs_grad(fw.p[0], fw.soft[0], O.BINARY_VALUES[0], tau, kappa)
+    gb = O.binary_gs_grad(fw.p[1], fw.soft[1], O.BINARY_VALUES[1], tau, kappa)
+    return np.abs(np.stack([fw.s * a * fw.soft[1] * gm, fw.s * a * fw.soft[0] * gb]))
+
+
+def mask_sign_grad_bounds(ref, prob, tau, kappa, tol):
+    """Gradients are linear in G; with G the only reduced-precision input (bf16
+    GEMM) its tolerance carries through the factors above."""
+    G = ref.G
+    gscale = tol * (np.abs(G) + np.sqrt(np.mean(G * G)))
+    bl = mask_sign_grad_factors(ref, prob, tau, kappa) * gscale[None] + tol * np.abs(ref.d_logits)
+    nr, Cc = G.shape
+    bs = (np.abs(ref.fw.wtil) * gscale).reshape(nr, Cc // prob.group, prob.group).sum(2)
+    return bl, bs + (0 if ref.d_scales is None else tol * np.abs(ref.d_scales))
+
+
 def check_lion(gpu, orc, theta_in, c_orc, lr, flip_frac, what):
     """Lion results agree to rounding except where the sign of the momentum mix
     c is decided by a difference below the path's tolerance; such flips move a

@@ -7,13 +7,15 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_common import TOL_BF16, Case, assert_close, assert_gemm_bound, assert_grad_close, gsq
+from gpu_common import (TOL_BF16, Case, assert_close, assert_gemm_bound, assert_grad_close, gsq,
+                        mask_sign_grad_bounds)
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
 pytestmark = pytest.mark.gpu
 
-FULL = ["llama8b_q_proj", "llama8b_down_proj", "llama70b_gate_proj", "moe64_kquant3"]
+FULL = ["llama8b_q_proj", "llama8b_down_proj", "llama70b_gate_proj", "moe64_kquant3",
+        "llama8b_down_proj_shift5", "llama8b_q_proj_mask_sign"]
 
 
 def _rows_view(t, K, nr, C_):
@@ -31,15 +33,18 @@ def _sample_rows(w, k=6):
 def _gather_state(case, rows):
     g = gsq()
     w = case.w
-    nr, K, Cc = w.experts * w.rows, w.K, w.cols
+    nr, K, Cc = w.experts * w.rows, w.L, w.cols
     idx = torch.from_numpy(rows).cuda()
     f = lambda which: case.layer.get_tensor(which, torch.float32)
+    j0 = None
+    if w.param == "shift5":
+        j0 = case.layer.get_tensor(g.GSQ_T_J0, torch.uint8).view(nr, Cc)[idx].cpu().numpy()
     L = f(g.GSQ_T_LOGITS).view(K, nr, Cc)[:, idx].cpu().numpy()
     M = f(g.GSQ_T_MOM_LOGITS).view(K, nr, Cc)[:, idx].cpu().numpy()
     S = f(g.GSQ_T_SCALES).view(nr, Cc // w.group)[idx].cpu().numpy()
     MS = f(g.GSQ_T_MOM_SCALES).view(nr, Cc // w.group)[idx].cpu().numpy()
     return O.RowState(row_ids=rows, W=case.W.view(nr, Cc)[idx].float().cpu().double().numpy(),
-                      logits=L, scales=S, m_logits=M, m_scales=MS)
+                      logits=L, scales=S, m_logits=M, m_scales=MS, j0=j0)
 
 
 @pytest.mark.parametrize("name", FULL)
@@ -58,7 +63,7 @@ def test_full_size_step_sampled_rows(name):
         def __getitem__(self, e):
             return Hs[int(e)]
     case.prob.H = _H()
-    nr, K, Cc = w.experts * w.rows, w.K, w.cols
+    nr, K, Cc = w.experts * w.rows, w.L, w.cols
     tau0, tau1 = w.tau(0), w.tau(1)
 
     # (a) gradient export at t = 0 (no update): G, D, loss property, sampled rows
@@ -89,8 +94,14 @@ def test_full_size_step_sampled_rows(name):
                           f"tcgen05 GEMM rows, expert {e}")
     del Hb
     torch.cuda.empty_cache()
-    assert_grad_close(glr, gsr if ref.d_scales is not None else None, ref, case.prob, tau0,
-                      w.kappa, TOL_BF16, "rows")
+    if w.param == "mask_sign":
+        bl, bs = mask_sign_grad_bounds(ref, case.prob, tau0, w.kappa, TOL_BF16)
+        assert np.all(np.abs(glr - ref.d_logits) <= bl * 1.0001 + 1e-30), "dL/dlogits rows"
+        assert np.all(np.abs(gsr - ref.d_scales) <= bs * 1.0001 + 1e-30), "dL/dscales rows"
+    else:
+        q = O.level_values(case.prob, st0) if w.param == "shift5" else None
+        assert_grad_close(glr, gsr if ref.d_scales is not None else None, ref, case.prob, tau0,
+                          w.kappa, TOL_BF16, "rows", q=q)
 
     # (b) the benchmark's step: update with look-ahead, state-synced on the rows
     case.layer.step(0, tau0, w.kappa, next_tau=tau1, next_kappa=w.kappa, loss=loss)
@@ -109,5 +120,45 @@ def test_full_size_step_sampled_rows(name):
     D1 = case.layer.get_tensor(g.GSQ_T_D, torch.bfloat16).view(nr, Cc)[idx].double().cpu().numpy()
     fw1 = O.forward(case.prob, st1, 1, tau1, w.kappa)
     assert_close(D1, fw1.D, 2 ** -8, "look-ahead D rows (bf16 storage)")
+    case.layer.sync_status()
+    case.layer.close()
+
+
+def test_full_size_token_microbatch_sampled_rows():
+    """The per-step token workload at full size (4096 x 4096 layer, one micro-batch of
+    32,768 tokens): D and G on sampled rows against the oracle (G = 2 (D X^T) X taken
+    in float64 over the same fp32 tokens), the loss property, and the state untouched
+    before the last micro-batch."""
+    from paper_2604_18556_gb300 import inputs
+    g = gsq()
+    w = C.WORKLOADS["llama8b_q_proj_tokens"]
+    case = Case(w, gemm="bf16", keep_calib_host=False)
+    rows = _sample_rows(w)
+    nr, Cc = w.experts * w.rows, w.cols
+    X = inputs.make_token_batch(w, 0, 0, device="cuda")
+    st0 = _gather_state(case, rows)
+    loss = torch.zeros(1, device="cuda")
+    # the forward of micro-batch 0 first, so its D can be read: the step's own kernel
+    # ends by writing the next micro-batch's D (and skips the forward done here)
+    case.layer.forward(0, w.tau(0), w.kappa)
+    Dd = case.layer.get_tensor(g.GSQ_T_D, torch.bfloat16).view(nr, Cc).clone()
+    case.layer.step_tokens(0, 0, 2, w.tau(0), X, loss=loss)      # micro-batch 0 of 2
+    torch.cuda.synchronize()
+    Gd = case.layer.get_tensor(g.GSQ_T_G, torch.float32).view(nr, Cc)
+    half_DG = 0.5 * torch.sum(Dd.double() * Gd.double()).item()
+    assert abs(loss.item() - half_DG) <= 1e-5 * abs(half_DG), (loss.item(), half_DG)
+    idx = torch.from_numpy(rows).cuda()
+    Gs, Ds = Gd[idx].double().cpu().numpy(), Dd[idx].double().cpu().numpy()
+    del Gd, Dd
+    fw = O.forward(case.prob, st0, 0, w.tau(0), w.kappa)
+    assert_close(Ds, fw.D, 2 ** -8, "D rows (bf16 storage)")
+    Xh = X[0].cpu().numpy()
+    Gref = np.zeros_like(fw.D)
+    for t0 in range(0, Xh.shape[0], 4096):
+        Xc = Xh[t0:t0 + 4096].astype(np.float64)
+        Gref += 2.0 * (fw.D @ Xc.T) @ Xc
+    assert_close(Gs, Gref, TOL_BF16, "G rows vs float64 token products")
+    st1 = _gather_state(case, rows)                              # no update before the last micro-batch
+    assert np.array_equal(st1.logits, st0.logits) and np.array_equal(st1.scales, st0.scales)
     case.layer.sync_status()
     case.layer.close()

@@ -13,7 +13,7 @@ import pytest
 import torch
 
 from gpu_common import (TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound, check_lion,
-                        check_momentum, gsq)
+                        check_momentum, gsq, mask_sign_grad_bounds)
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -41,26 +41,6 @@ def _randomise(case, seed):
     L = rng.standard_normal((2, w.experts * w.rows, w.cols)).astype(np.float32)
     case.layer.set_tensor(g.GSQ_T_LOGITS, torch.from_numpy(L).cuda())
     return case.state()
-
-
-def _grad_factors(ref, prob, tau, kappa):
-    """|dL/dl| / |G| for both planes: (kappa/tau) s a |b~ dm~| and (kappa/tau) s a |m~ db~|."""
-    fw = ref.fw
-    a = float(prob.grid[2])
-    gm = O.binary_gs_grad(fw.p[0], fw.soft[0], O.BINARY_VALUES[0], tau, kappa)
-    gb = O.binary_gs_grad(fw.p[1], fw.soft[1], O.BINARY_VALUES[1], tau, kappa)
-    return np.abs(np.stack([fw.s * a * fw.soft[1] * gm, fw.s * a * fw.soft[0] * gb]))
-
-
-def _grad_bounds(ref, prob, tau, kappa, tol):
-    """Gradients are linear in G; with G the only reduced-precision input (bf16
-    GEMM) its tolerance carries through the factors above."""
-    G = ref.G
-    gscale = tol * (np.abs(G) + np.sqrt(np.mean(G * G)))
-    bl = _grad_factors(ref, prob, tau, kappa) * gscale[None] + tol * np.abs(ref.d_logits)
-    nr, Cc = G.shape
-    bs = (np.abs(ref.fw.wtil) * gscale).reshape(nr, Cc // prob.group, prob.group).sum(2)
-    return bl, bs + (0 if ref.d_scales is None else tol * np.abs(ref.d_scales))
 
 
 @pytest.mark.parametrize("name", list(SMALL))
@@ -110,7 +90,7 @@ def test_mask_sign_step_loss_and_gradients(name, gemm):
         if ref.d_scales is not None:
             assert_close(gs.cpu().numpy(), ref.d_scales, tol, "dL/dscales")
     else:
-        bl, bs = _grad_bounds(ref, case.prob, TAU[name], 1.0, tol)
+        bl, bs = mask_sign_grad_bounds(ref, case.prob, TAU[name], 1.0, tol)
         assert np.all(np.abs(got_l - ref.d_logits) <= bl * 1.0001 + 1e-30), "dL/dlogits"
         if ref.d_scales is not None:
             err = np.abs(gs.cpu().numpy().astype(np.float64).reshape(ref.d_scales.shape) - ref.d_scales)
@@ -145,7 +125,7 @@ def test_mask_sign_step_update(name, gemm):
             gb_s = None if res.d_scales is None else \
                 tol * (np.abs(res.d_scales) + np.sqrt(np.mean(res.d_scales ** 2)))
         else:
-            gb_l, gb_s = _grad_bounds(res, case.prob, TAU[name], 1.0, tol)
+            gb_l, gb_s = mask_sign_grad_bounds(res, case.prob, TAU[name], 1.0, tol)
         check_momentum(gpu.m_logits, st_sync.m_logits, gb_l, w.beta2, "logit momentum")
         if res.d_scales is not None:
             c_s = w.beta1 * before.m_scales.astype(np.float64) + (1 - w.beta1) * res.d_scales

@@ -431,6 +431,9 @@ def gpu_arm(args, rank, world, local):
                      "peak_source": f"{peak_src} bf16_tflops_sustained"}
     launches = bwd_n + gemm_n + fwd_n
 
+    # method diagnostics of the state after the timed steps (not timed)
+    diag = layer.diagnose(sched(t), w.kappa)
+    diag["after_step"] = t
     e2e = None
     if not args.no_e2e:
         e2e = e2e_run(args, w, W, H, gsq, torch, rank, world)
@@ -449,6 +452,7 @@ def gpu_arm(args, rank, world, local):
                                              "replayed once before the timed region)")
                                   if graph is not None else "eager launches"}),
             "roofline": roofline, "roofline_gemm": roofline_gemm, "clocks": clocks,
+            "diagnostics": diag,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
             "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
                                    "forward": fwd_ms / args.steps},

@@ -30,12 +30,15 @@ constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;
 constexpr int TC_THREADS = 192;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
-// Tile shape M = 128 x N = BN (256, 224 or 128) x 64; the pipeline depth fills ~192 KiB.
+// Tile shape M = 128 x N = BN (256, 224 or 128) x 64; the pipeline fills the shared memory.
 template <int BN>
 struct TcCfg {
   static constexpr int kBBytes = BN * TC_BK * 2;
   static constexpr int kStageBytes = TC_A_BYTES + kBBytes;
-  static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
+  // as many stages as the 227 KiB of shared memory per CTA hold (barriers + 1 KiB
+  // alignment slack beside them), at most 8
+  static constexpr int kStages =
+      ((232448 - 2048) / kStageBytes) < 8 ? ((232448 - 2048) / kStageBytes) : 8;
   // double-buffered fp32 accumulator (2 BN columns), allocated as a power of two
   static constexpr int kTmemCols = 2 * BN <= 256 ? 256 : 512;
   static constexpr int kAccStride = kTmemCols / 2;  // column offset of the second buffer

@@ -452,12 +452,12 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
 
 int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
-  // Time ~ waves x tile width: 256-wide tiles unless 224-wide ones fill their
-  // waves enough better (a 4096 x 4096 layer: 512 tiles of 256 = 3.37 waves,
-  // rounded up to 4 x 256; 608 tiles of 224 = exactly 4 waves x 224), or unless
-  // 256-wide tiles leave many SMs idle and 128-wide ones balance clearly better.
-  // Measured on GB300: 128-wide tiles lose more to the narrower MMA than they gain
-  // in balance on the 4096 x 4096 layer (142 us vs 114 us).
+  // 224-wide tiles by default: their 44 KiB stages give a 5-deep ring against 4 for
+  // 256-wide ones, which measured faster on GB300 on every layer shape here (4096 x
+  // 4096: 99 vs 111 us; 4096 x 14336: 1.00 vs 1.03 ms; 64 experts 2048 x 7168: 8.26
+  // vs 8.58 ms), unless the wave count (waves x width) makes them clearly worse.
+  // 128-wide tiles only when 256-wide ones leave many SMs idle and 128 balances far
+  // better (on the 4096 x 4096 layer they lose: 140 us).
   const int64_t mt = (M + TC_BM - 1) / TC_BM;
   auto cost = [&](int bn) {
     const int64_t tiles = static_cast<int64_t>(E) * mt * ((N + bn - 1) / bn);
@@ -466,7 +466,7 @@ int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
   const double b256 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 255) / 256), num_sms);
   const double b128 = wave_balance(static_cast<int64_t>(E) * mt * ((N + 127) / 128), num_sms);
   if (b256 < 0.6 && b128 > b256 + 0.25) return 128;
-  return cost(224) < 0.95 * cost(256) ? 224 : 256;
+  return cost(224) <= 1.1 * cost(256) ? 224 : 256;
 }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {

@@ -230,11 +230,13 @@ def run_oracle_sample(w, step_budget_s: float, n_steps: int, n_warm: int, Wt=Non
     if Wt is None:
         Wt, H = _cpu_inputs(w, min(w.rows, 256))
     prob = _oracle_problem(w, H[None] if H.ndim == 2 else H, None)
-    # probe one row to size the sample
-    st = O.init_state(prob, Wt[:1], np.arange(1), init_bias=w.init_bias)
+    # size the sample from a probe of 16 rows (after one untimed call)
+    probe = min(16, Wt.shape[0])
+    st = O.init_state(prob, Wt[:probe], np.arange(probe), init_bias=w.init_bias)
+    O.step(prob, st.copy(), 0, w.tau(0), w.kappa)
     t0 = time.perf_counter()
     O.step(prob, st, 0, w.tau(0), w.kappa)
-    t_row = time.perf_counter() - t0
+    t_row = (time.perf_counter() - t0) / probe
     rows = min(Wt.shape[0], _oracle_rows_for(step_budget_s, t_row))
     st = O.init_state(prob, Wt[:rows], np.arange(rows), init_bias=w.init_bias)
     for t in range(n_warm):
@@ -668,7 +670,7 @@ def cpu_baseline(args, w, W, H_host):
     """Oracle step on a bounded row sample, in a single-threaded child process."""
     import numpy as np
     import tempfile
-    rows = min(w.rows, 256)
+    rows = min(w.rows, 1024)
     with tempfile.TemporaryDirectory() as td:
         np.save(os.path.join(td, "W.npy"), W[0, :rows].float().cpu().numpy())
         np.save(os.path.join(td, "H.npy"), H_host)
@@ -678,10 +680,10 @@ def cpu_baseline(args, w, W, H_host):
             "from paper_2604_18556_gb300 import configs as C\n"
             "w = C.WORKLOADS[%r]\n"
             "Wt = np.load(%r); H = np.load(%r)\n"
-            "per, rows, meas = bench.run_oracle_sample(w, %f, 3, 1, Wt, H)\n"
+            "per, rows, meas = bench.run_oracle_sample(w, %f, 6, 1, Wt, H)\n"
             "print(json.dumps([per, rows, meas]))\n"
         ) % (ROOT, w.name, os.path.join(td, "W.npy"), os.path.join(td, "H.npy"),
-             args.cpu_sample_seconds / 4)
+             args.cpu_sample_seconds / 7)
         env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
         r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
                            cwd=ROOT, timeout=600)
@@ -690,7 +692,7 @@ def cpu_baseline(args, w, W, H_host):
                     "sample": f"failed: {r.stderr[-300:]}"}
         per, srows, meas = json.loads(r.stdout.strip().splitlines()[-1])
     return {"value": 1.0 / per, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{srows} of {w.rows} rows, 3 timed steps + 1 warm-up ({meas:.1f} s "
+            "sample": f"{srows} of {w.rows} rows, 6 timed steps + 1 warm-up ({meas:.1f} s "
                       f"measured); full-layer step = sample x {w.rows}/{srows}"}
 
 

@@ -1099,19 +1099,21 @@ __global__ void __launch_bounds__(kEwThreads) k_diagnose(const DiagParams P) {
 #pragma unroll
     for (int e = 0; e < kDiagMarginBins - 1; ++e) b += mg >= edges[e] ? 1 : 0;
     atomicAdd(&hist[kDiagShiftBins + b], 1u);
-    double pmax;
+    // fp32 arithmetic (a monitoring statistic), double accumulation
+    const float kot = static_cast<float>(P.kappa_over_tau);
+    float pmax;
     if (P.mask_sign) {
-      const double pm = 1.0 / (1.0 + exp(-2.0 * P.kappa_over_tau * P.logits[i]));
-      const double pb = 1.0 / (1.0 + exp(-2.0 * P.kappa_over_tau * P.logits[P.n + i]));
-      pmax = fmax(fmax(pm * (1.0 - pb), 1.0 - pm), pm * pb);
+      const float pm = 1.0f / (1.0f + expf(-2.0f * kot * P.logits[i]));
+      const float pb = 1.0f / (1.0f + expf(-2.0f * kot * P.logits[P.n + i]));
+      pmax = fmaxf(fmaxf(pm * (1.0f - pb), 1.0f - pm), pm * pb);
     } else {
       float lmax = P.logits[i];
       for (int k = 1; k < P.K; ++k) lmax = fmaxf(lmax, P.logits[k * P.n + i]);
-      double sum = 0.0;
-      for (int k = 0; k < P.K; ++k) sum += exp(P.kappa_over_tau * (P.logits[k * P.n + i] - lmax));
-      pmax = 1.0 / sum;
+      float sum = 0.0f;
+      for (int k = 0; k < P.K; ++k) sum += expf(kot * (P.logits[k * P.n + i] - lmax));
+      pmax = 1.0f / sum;
     }
-    acc += pmax;
+    acc += static_cast<double>(pmax);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);

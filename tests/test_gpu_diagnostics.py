@@ -1,6 +1,6 @@
 """GPU parity of gsq_diagnose against the oracle's diagnostics: displacement and
 margin histograms bit-exact (integer results of fp32 decisions), mean noise-free
-max-probability to double rounding, for every parameterisation and both scale
+max-probability to fp32 rounding, for every parameterisation and both scale
 modes, after a few steps and after a warm start from supplied codes."""
 import dataclasses
 
@@ -31,7 +31,9 @@ def _check(case, code0, tau, kappa):
                                      float(np.float32(kappa)))
     assert got["displacement"] == disp.tolist()
     assert got["margin"] == marg.tolist()
-    assert abs(got["mean_max_prob"] - pmax) <= 1e-9 * pmax
+    # the kernel evaluates each max-probability in fp32 (a few ulp), then averages
+    # in double: the mean agrees to about the fp32 unit roundoff
+    assert abs(got["mean_max_prob"] - pmax) <= 1e-6 * pmax
     return got
 
 

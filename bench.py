@@ -343,7 +343,7 @@ def gpu_arm(args, rank, world, local):
     w = rank_workload(_workload(args.workload), rank, world)
     W = inputs.make_weight(w, device="cuda")
     H = inputs.make_gram(w, device="cuda")
-    H_host = H[0].double().cpu().numpy() if rank == 0 and not args.no_cpu_baseline else None
+    H_host = H[0].double().cpu().numpy() if world == 1 and not args.no_cpu_baseline else None
     layer = gsq.Layer(W, H, w.grid, w.group, calib_kind="H", scale_mode=w.scale_mode, gemm="bf16",
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
@@ -440,7 +440,7 @@ def gpu_arm(args, rank, world, local):
     if not args.no_e2e:
         e2e = e2e_run(args, w, W, H, gsq, torch, rank, world)
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline:     # the oracle baseline: N = 1 only
         cpu = cpu_baseline(args, w, W, H_host)
 
     if rank == 0:
@@ -552,7 +552,7 @@ def gpu_arm_tokens(args, rank, world, local):
     if not args.no_e2e:
         e2e = e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step)
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline:     # the oracle baseline: N = 1 only
         cpu = cpu_baseline_tokens(args, w)
     if rank == 0:
         print(json.dumps({

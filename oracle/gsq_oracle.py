@@ -280,12 +280,27 @@ def loss_bruteforce(W: np.ndarray, What: np.ndarray, X: np.ndarray) -> float:
 # ----------------------------------------------------------------------------
 # backward (App. B softmax Jacobian) and Lion (§3.3, App. B)
 # ----------------------------------------------------------------------------
+def centred_values(p, values):
+    """d_k - w~ for every k, with w~ = sum_j p_j d_j, written as
+    sum_j p_j (d_k - d_j) (equal because sum_j p_j = 1).  The direct difference
+    cancels catastrophically when p is nearly one-hot (d_m - w~ is then tiny);
+    this form keeps full relative accuracy in float64.  p: [K, ...]; values
+    broadcastable against p."""
+    p = np.asarray(p, dtype=np.float64)
+    d = np.broadcast_to(np.asarray(values, dtype=np.float64), p.shape)
+    out = np.zeros(p.shape)
+    for k in range(p.shape[0]):
+        out[k] = np.sum(p * (d[k][None] - d), axis=0)
+    return out
+
+
 def binary_gs_grad(p, soft, values, tau: float, kappa: float):
     """d(soft value)/dl of a binary instance: the softmax Jacobian (App. B)
     d w~/d l_k = (kappa/tau) p_k (d_k - w~), chained through the tied logits
     l_1 = l, l_0 = -l."""
-    d0, d1 = values
-    return (kappa / tau) * (p[1] * (d1 - soft) - p[0] * (d0 - soft))
+    vals = np.asarray(values, dtype=np.float64).reshape((2,) + (1,) * (np.ndim(p) - 1))
+    c = centred_values(p, vals)
+    return (kappa / tau) * (p[1] * c[1] - p[0] * c[0])
 
 
 def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float, q=None):
@@ -302,7 +317,8 @@ def backward(prob: Problem, fw: Forward, G: np.ndarray, tau: float, kappa: float
         return d_logits, d_scales
     if q is None:
         q = np.asarray(prob.grid, dtype=np.float64)[:, None, None]
-    d_logits = (kappa / tau) * (G * fw.s)[None] * fw.p * (q - fw.wtil[None])
+    # softmax Jacobian (App. B): dL/dl_k = (kappa/tau) G s p_k (q_k - w~)
+    d_logits = (kappa / tau) * (G * fw.s)[None] * fw.p * centred_values(fw.p, q)
     d_scales = (G * fw.wtil).reshape(nr, C // prob.group, prob.group).sum(axis=2)
     return d_logits, d_scales
 

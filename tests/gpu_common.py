@@ -78,7 +78,7 @@ def grad_bounds(ref, prob, tol, q=None):
     fw = ref.fw
     if q is None:
         q = np.asarray(prob.grid, np.float64)[:, None, None]
-    f = np.abs(fw.s[None] * fw.p * (q - fw.wtil[None]))        # |f_k| / (kappa/tau)
+    f = np.abs(fw.s[None] * fw.p * O.centred_values(fw.p, q))   # |f_k| / (kappa/tau)
     bl = None
     nr, C = G.shape
     bs = (np.abs(fw.wtil) * gscale).reshape(nr, C // prob.group, prob.group).sum(2)

@@ -43,6 +43,8 @@ def _args():
     ap.add_argument("--no-graph", action="store_true",
                     help="time eager launches instead of one CUDA-graph replay of the timed steps")
     ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
+    ap.add_argument("--fused", action="store_true",
+                    help="time the fused step kernel (GSQ_FLAG_FUSED) instead of GEMM + backward")
     return ap.parse_args()
 
 
@@ -54,26 +56,34 @@ def _dist():
 
 
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
-ELEMENTWISE_SRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc", "gsq_elementwise.cu")
+CSRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc")
+# the source files each profiled kernel is compiled from
+KERNEL_SOURCES = {
+    "k_backward": ["gsq_elementwise.cu", "gsq_relax.cuh"],
+    "k_step_fused": ["gsq_fused.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
+}
 
 
-def source_sha256(path: str = ELEMENTWISE_SRC) -> str:
+def source_sha256(kernel: str = "k_backward") -> str:
     import hashlib
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
-def committed_traffic(workload: str):
-    """DRAM bytes (read + write) per k_backward launch from the committed ncu
-    capture, or None when there is none for this workload or the kernel source
-    has changed since it was taken."""
+def committed_traffic(workload: str, kernel: str = "k_backward"):
+    """DRAM bytes (read + write) per launch of `kernel` from the committed ncu
+    capture, or None when there is none for this workload or the kernel's
+    sources have changed since it was taken."""
     if not os.path.exists(TRAFFIC_FILE):
         return None
     with open(TRAFFIC_FILE) as f:
-        d = json.load(f)
-    if d.get("source_sha256") != source_sha256():
+        d = json.load(f).get("kernels", {}).get(kernel)
+    if not d or d.get("source_sha256") != source_sha256(kernel):
         return None
-    return d.get("workloads", {}).get(workload, {}).get("k_backward_dram_bytes_per_launch")
+    return d.get("workloads", {}).get(workload, {}).get("dram_bytes_per_launch")
 
 
 def rank_workload(w, rank: int, world: int):
@@ -347,7 +357,8 @@ def gpu_arm(args, rank, world, local):
     layer = gsq.Layer(W, H, w.grid, w.group, calib_kind="H", scale_mode=w.scale_mode, gemm="bf16",
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param)
+                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param,
+                      fused=args.fused)
     stream = torch.cuda.current_stream()
     loss = torch.zeros(1, device="cuda")
     T = w.steps
@@ -414,24 +425,43 @@ def gpu_arm(args, rank, world, local):
     bwd_n, bwd_ms = prof["backward"]
     gemm_n, gemm_ms = prof["gemm"]
     fwd_n, fwd_ms = prof["forward"]
-    bwd_avg = bwd_ms / max(bwd_n, 1)
-    gemm_avg = gemm_ms / max(gemm_n, 1)
-    bytes_bwd = w.elementwise_bytes_per_weight() * n
+    step_n, step_ms = prof["step"]
     flops = w.gemm_flops_per_step()
-    bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
-    gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
-    traffic = committed_traffic(w.name)
-    roofline = {"kernel": "k_backward (fused backward + Lion + next forward)", "bound": "hbm",
-                "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
-                "traffic": traffic, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
-                "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
-                "frac_of_8TBps": bwd_gbs / 8000.0}
-    roofline_gemm = {"kernel": "k_tc_gemm (tcgen05 loss contraction)", "bound": "tensor",
-                     "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
-                     "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
-                     "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
-                     "peak_source": f"{peak_src} bf16_tflops_sustained"}
-    launches = bwd_n + gemm_n + fwd_n
+    if step_n > 0:
+        # one fused kernel per step: the contraction on the tensor cores with the
+        # backward, Lion and next forward as its epilogue (G never leaves the SM)
+        avg = step_ms / step_n
+        nbytes = w.fused_step_bytes()
+        gbs = nbytes / (avg * 1e-3) / 1e9
+        tfs = flops / (avg * 1e-3) / 1e12
+        roofline = {"kernel": "k_step_fused (tcgen05 contraction + backward + Lion + next forward)",
+                    "bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
+                    "traffic": committed_traffic(w.name, "k_step_fused"),
+                    "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
+                    "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": avg,
+                    "frac_of_8TBps": gbs / 8000.0}
+        roofline_gemm = {"kernel": "k_step_fused contraction (its flops over the fused kernel's time)",
+                         "bound": "tensor", "achieved": tfs, "peak": tf_sust, "unit": "TFLOP/s",
+                         "frac": tfs / tf_sust, "flops_per_launch": flops, "avg_launch_ms": avg,
+                         "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    else:
+        bwd_avg = bwd_ms / max(bwd_n, 1)
+        gemm_avg = gemm_ms / max(gemm_n, 1)
+        bytes_bwd = w.elementwise_bytes_per_weight() * n
+        bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
+        gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
+        roofline = {"kernel": "k_backward (fused backward + Lion + next forward)", "bound": "hbm",
+                    "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
+                    "traffic": committed_traffic(w.name),
+                    "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
+                    "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
+                    "frac_of_8TBps": bwd_gbs / 8000.0}
+        roofline_gemm = {"kernel": "k_tc_gemm (tcgen05 loss contraction)", "bound": "tensor",
+                         "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
+                         "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
+                         "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
+                         "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    launches = bwd_n + gemm_n + fwd_n + step_n
 
     # method diagnostics of the state after the timed steps (not timed)
     diag = layer.diagnose(sched(t), w.kappa)
@@ -457,7 +487,7 @@ def gpu_arm(args, rank, world, local):
             "diagnostics": diag,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
             "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
-                                   "forward": fwd_ms / args.steps},
+                                   "forward": fwd_ms / args.steps, "step": step_ms / args.steps},
         }
         print(json.dumps(line), flush=True)
     del graph

@@ -71,7 +71,15 @@ enum { GSQ_DTYPE_F32 = 0, GSQ_DTYPE_BF16 = 1 };
 enum { GSQ_CALIB_H = 0, GSQ_CALIB_X = 1, GSQ_CALIB_BATCHES = 2 };
 enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
 enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
-enum { GSQ_FLAG_NO_NOISE = 1u }; /* g = 0: plain tempered softmax, no Gumbel draw */
+enum {
+  GSQ_FLAG_NO_NOISE = 1u, /* g = 0: plain tempered softmax, no Gumbel draw             */
+  GSQ_FLAG_KEEP_G = 2u,   /* with GSQ_FLAG_FUSED: the fused step also stores G, so
+                             GSQ_T_G reads back the last step's dL/dW^                 */
+  GSQ_FLAG_FUSED = 4u     /* bf16 layers: gsq_step runs one fused kernel (contraction
+                             with the backward, Lion and look-ahead as its epilogue)
+                             instead of two; the same results to rounding.  Measured
+                             slower than the two kernels on GB300, hence opt-in.       */
+};
 enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1, GSQ_PARAM_MASK_SIGN = 2 };
 
 /* Layer problem (Eq. 1 with a linear f; §3.2; §4.1; Table 5 for the defaults).
@@ -221,6 +229,12 @@ GSQ_API gsq_status gsq_init_logits(gsq_layer* layer, const uint8_t* codes_dev, c
  *              the step runs in gradient-export mode: it writes the raw
  *              gradients ([L][E][R][C] fp32, L logits per weight, and
  *              [E][R][C/G] fp32), skips the Lion update and ignores next_tau.
+ * Kernels: the contraction and the backward (+ update + look-ahead) are two
+ * kernels; with GSQ_FLAG_FUSED (bf16, not exporting) one fused kernel runs the
+ * contraction with the rest as its epilogue, so G stays on chip (GSQ_T_G then
+ * reads back only with GSQ_FLAG_KEEP_G).  The D of noise counter t lives in one
+ * of two buffers by the parity of t, so a look-ahead never overwrites the D
+ * that its own step's contraction reads.
  * Never synchronises; graph-capturable for a fixed argument list. */
 GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float kappa, float next_tau,
                     float next_kappa, void* stream, float* loss_dev, float* grad_logits_dev,
@@ -323,7 +337,8 @@ enum {
   GSQ_K_PACK = 4,
   GSQ_K_INIT = 5,
   GSQ_K_TOKENS = 6,   /* per-step tokens to the tensor-core operands (bf16, X^T) */
-  GSQ_K_COUNT = 7
+  GSQ_K_STEP = 7,     /* fused step: loss contraction with backward + Lion (+ look-ahead) */
+  GSQ_K_COUNT = 8
 };
 typedef struct gsq_profile {
   int32_t launches[GSQ_K_COUNT];

@@ -85,6 +85,9 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
   size_t flags, partials, logits, m_logits, scales, m_scales, W, H, D, G, kq_d, kq_sc, hscratch, j0;
+  size_t D2;     // second D buffer (bf16 layers stepped with gsq_step): D of step t lives in
+                 // buffer t mod 2, so a step can write the next D while its own is still read
+  bool has_d2;
   size_t tok_b, tok_t, Y, acc_l, acc_s;  // per-step token batches (GSQ_CALIB_BATCHES)
   size_t code0, diag;                     // initial codes and diagnostics counters
   size_t total;
@@ -148,6 +151,8 @@ Layout layout_of(const Shape& s) {
   L.H = s.batches ? off
                   : take(static_cast<size_t>(s.E) * s.C * s.C * (s.d_bf16 ? 2 : 4), "H");
   L.D = take(n * (s.d_bf16 ? 2 : 4), "D");
+  L.has_d2 = s.d_bf16 && !s.batches;
+  L.D2 = L.has_d2 ? take(2 * n, "D2") : off;
   L.G = take(4 * n, "G");
   L.kq_d = s.kquant ? take(2 * (n / kSuperBlock), "kq_d") : off;
   L.kq_sc = s.kquant ? take(n / kSubBlock, "kq_sc") : off;
@@ -217,7 +222,7 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
   }
   if (d->gemm_precision != GSQ_GEMM_BF16 && d->gemm_precision != GSQ_GEMM_F32)
     return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
-  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE))
+  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE | GSQ_FLAG_KEEP_G | GSQ_FLAG_FUSED))
     return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
   if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5 &&
       d->param_mode != GSQ_PARAM_MASK_SIGN)
@@ -262,6 +267,11 @@ struct gsq_layer {
   bool tc;
   int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
   int group_n; // column group of the GEMM's tile order
+  int fused_group_n;  // row-tile group of the fused step's tile order (1: whole rows first)
+  bool fused;   // GSQ_FLAG_FUSED: gsq_step runs the fused step kernel (bf16, not exporting)
+  bool keep_g;  // GSQ_FLAG_KEEP_G: the fused step also stores G
+  bool g_valid; // the G buffer holds the last step's G
+  size_t d_cur; // offset of the buffer holding the latest D written
   // pending forward (D valid for these arguments)
   bool d_ready;
   uint64_t d_step;
@@ -280,6 +290,12 @@ struct gsq_layer {
 namespace {
 
 float* fptr(gsq_layer* L, size_t off) { return reinterpret_cast<float*>(L->ws + off); }
+
+// Offset of the D buffer of noise counter t (forward pass t writes it, its loss
+// contraction reads it).
+size_t d_off(const gsq_layer* L, uint64_t t) {
+  return (L->lay.has_d2 && (t & 1u)) ? L->lay.D2 : L->lay.D;
+}
 
 // Live handles, so a stale or twice-destroyed pointer is rejected without
 // being dereferenced.
@@ -360,7 +376,7 @@ void prof_record(cudaEvent_t ev, cudaStream_t s) {
 // NVTX range names per kernel kind (visible in nsys / ncu timelines).
 const char* const kKindName[GSQ_K_COUNT] = {"gsq:forward", "gsq:gemm",  "gsq:backward",
                                             "gsq:project", "gsq:pack",  "gsq:init",
-                                            "gsq:tokens"};
+                                            "gsq:tokens", "gsq:step"};
 
 void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
   nvtxRangePushA(kKindName[kind]);
@@ -399,11 +415,13 @@ gsq_status launch_fwd(gsq_layer* L, uint64_t step, float tau, float kappa, float
   p.inv_tau = static_cast<float>(1.0 / tau);
   p.kappa_over_tau = static_cast<float>(static_cast<double>(kappa) / tau);
   p.what = what;
+  p.D = L->ws + d_off(L, step);
   int slot;
   prof_begin(L, GSQ_K_FORWARD, s, slot);
   const cudaError_t e = launch_forward(p, L->grid_fwd, s);
   prof_end(L, slot, s);
   if (e != cudaSuccess) return cuda_fail(e, "forward kernel");
+  L->d_cur = d_off(L, step);
   L->d_ready = true;
   L->d_step = step;
   L->d_tau = tau;
@@ -411,7 +429,7 @@ gsq_status launch_fwd(gsq_layer* L, uint64_t step, float tau, float kappa, float
   return GSQ_OK;
 }
 
-gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
+gsq_status launch_gemm(gsq_layer* L, size_t doff, cudaStream_t s) {
   const Shape& sh = L->shape;
   int slot;
   prof_begin(L, GSQ_K_GEMM, s, slot);
@@ -422,7 +440,7 @@ gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
     g.M = static_cast<int>(sh.R);
     g.N = static_cast<int>(sh.C);
     g.K = static_cast<int>(sh.C);
-    g.A = L->ws + L->lay.D;
+    g.A = L->ws + doff;
     g.B = L->ws + L->lay.H;
     g.out = fptr(L, L->lay.G);
     g.out_bf16 = 0;
@@ -437,7 +455,7 @@ gsq_status launch_gemm(gsq_layer* L, cudaStream_t s) {
     g.M = static_cast<int>(sh.R);
     g.N = static_cast<int>(sh.C);
     g.Kd = static_cast<int>(sh.C);
-    g.A = L->ws + L->lay.D;
+    g.A = L->ws + doff;
     g.sam = sh.C;
     g.sak = 1;
     g.sab = sh.R * sh.C;
@@ -482,7 +500,7 @@ size_t tensor_offset(const gsq_layer* L, int which) {
     case GSQ_T_MOM_LOGITS: return L->lay.m_logits;
     case GSQ_T_SCALES: return L->lay.scales;
     case GSQ_T_MOM_SCALES: return L->lay.m_scales;
-    case GSQ_T_D: return L->lay.D;
+    case GSQ_T_D: return L->d_cur;
     case GSQ_T_G: return L->lay.G;
     case GSQ_T_W: return L->lay.W;
     case GSQ_T_H: return L->lay.H;
@@ -558,6 +576,10 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   L->device = dev;
   L->num_sms = prop.multiProcessorCount;
   L->tc = tc;
+  L->keep_g = (desc->flags & GSQ_FLAG_KEEP_G) != 0;
+  L->fused = lay.has_d2 && tc && (desc->flags & GSQ_FLAG_FUSED) != 0;
+  L->g_valid = false;
+  L->d_cur = lay.D;
   L->d_ready = false;
   L->mb_step = 0;
   L->mb_next = 0;
@@ -580,6 +602,9 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
   L->group_n = kGemmGroupN;
+  // the fused step's tile order: groups of row tiles, as for the GEMM (whole rows
+  // first measured no faster)
+  L->fused_group_n = kGemmGroupN;
   if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)
     const int v = std::atoi(gn);
     if (v >= 0 && v <= 1024) L->group_n = v;
@@ -691,7 +716,8 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
   if (!(L->d_ready && L->d_step == step && L->d_tau == tau && L->d_kappa == kappa)) {
     if ((st = launch_fwd(L, step, tau, kappa, nullptr, s)) != GSQ_OK) return st;
   }
-  if ((st = launch_gemm(L, s)) != GSQ_OK) return st;
+  const bool fused = L->fused && !export_mode;
+  if (!fused && (st = launch_gemm(L, d_off(L, step), s)) != GSQ_OK) return st;
 
   EwParams p = base_params(L);
   p.t = static_cast<uint32_t>(step);
@@ -704,15 +730,38 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
     p.kappa_log2_next = static_cast<float>(next_kappa * kLog2e);
     p.inv_tau_next = static_cast<float>(1.0 / next_tau);
   }
+  p.D = L->ws + d_off(L, step + 1);  // the look-ahead's D
   p.grad_logits = grad_logits_dev;
   p.grad_scales = grad_scales_dev;
   p.loss_out = loss_dev;
   int slot;
-  prof_begin(L, GSQ_K_BACKWARD, s, slot);
-  const cudaError_t e = launch_backward(p, L->grid_bwd, s);
-  prof_end(L, slot, s);
-  if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+  cudaError_t e;
+  if (fused) {
+    const Shape& sh = L->shape;
+    FusedStep f;
+    f.P = p;
+    f.H = L->ws + L->lay.H;
+    f.D_t = L->ws + d_off(L, step);
+    f.D_next = L->ws + d_off(L, step + 1);
+    f.G_out = L->keep_g ? fptr(L, L->lay.G) : nullptr;
+    f.E = static_cast<int>(sh.E);
+    f.R = static_cast<int>(sh.R);
+    f.C = static_cast<int>(sh.C);
+    f.group_n = L->fused_group_n;
+    prof_begin(L, GSQ_K_STEP, s, slot);
+    e = launch_step_fused(f, L->num_sms, s);
+    prof_end(L, slot, s);
+    if (e != cudaSuccess) return cuda_fail(e, "fused step kernel");
+    L->g_valid = L->keep_g;
+  } else {
+    prof_begin(L, GSQ_K_BACKWARD, s, slot);
+    e = launch_backward(p, L->grid_bwd, s);
+    prof_end(L, slot, s);
+    if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+    L->g_valid = true;
+  }
   if (lookahead) {
+    L->d_cur = d_off(L, step + 1);
     L->d_ready = true;
     L->d_step = step + 1;
     L->d_tau = next_tau;
@@ -841,6 +890,7 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
   e = launch_backward(p, L->grid_bwd, s);
   prof_end(L, slot, s);
   if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+  L->g_valid = true;
   if (lookahead) {
     L->d_ready = true;
     L->d_step = t + 1;
@@ -1026,6 +1076,9 @@ static gsq_status copy_tensor(gsq_layer* L, int32_t which, void* dst, const void
 gsq_status gsq_get_tensor(gsq_layer* L, int32_t which, void* dst_dev, size_t bytes, void* stream) {
   GSQ_INJECT("gsq_get_tensor");
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
+  if (which == GSQ_T_G && !L->g_valid)
+    return fail(GSQ_ERR_STATE, "G holds no step's gradient: the fused step keeps it on chip unless "
+                               "the layer has GSQ_FLAG_KEEP_G");
   return copy_tensor(L, which, dst_dev, L->ws + tensor_offset(L, which), bytes, stream, "gsq_get_tensor");
 }
 

@@ -218,6 +218,21 @@ struct TcGemm {
   int group_n;  // tile-order column group; <= 0: one group (m fastest across all columns)
 };
 bool tc_gemm_supported(int device);
+
+// Fused step (gsq_fused.cu): the tensor-core loss contraction with the backward,
+// Lion and look-ahead forward as its epilogue; G stays on chip unless G_out is
+// set.  H ([E*C][C]) and D_t ([E*R][C]) are bf16, K-major; D_next receives the
+// bf16 D of step t + 1 (a different buffer from D_t) when P.lookahead.
+struct FusedStep {
+  EwParams P;
+  const void* H;
+  const void* D_t;
+  void* D_next;
+  float* G_out;  // nullable
+  int E, R, C;
+  int group_n;   // tile order: groups of row tiles
+};
+cudaError_t launch_step_fused(const FusedStep& f, int num_sms, cudaStream_t s);
 int tc_gemm_tile_n(int E, int M, int N, int num_sms);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 

@@ -89,9 +89,13 @@ def test_workspace_size_formula(lib):
         n, L = w.n, w.L
         # every buffer is 256-byte aligned and followed by a 256-byte canary
         bufs = [256, 8 * 16384, 4 * L * n, 4 * L * n, 4 * n // w.group, 4 * n // w.group,
-                n * w.w_bytes(), 2 * n, 4 * n]
+                n * w.w_bytes()]
         if w.calib != "batches":
             bufs.append(w.experts * w.cols ** 2 * 2)               # H (bf16)
+        bufs.append(2 * n)                                         # D (bf16)
+        if w.calib != "batches":
+            bufs.append(2 * n)                                     # D of the odd steps
+        bufs.append(4 * n)                                         # G
         if w.scale_mode == "kquant2":
             bufs += [2 * n // 256, n // 16]
         if w.calib == "X":

@@ -43,6 +43,8 @@ def _args():
     ap.add_argument("--no-graph", action="store_true",
                     help="time eager launches instead of one CUDA-graph replay of the timed steps")
     ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
+    ap.add_argument("--unstaged", action="store_true",
+                    help="time the backward with direct global loads (GSQ_FLAG_UNSTAGED)")
     ap.add_argument("--fused", action="store_true",
                     help="time the fused step kernel (GSQ_FLAG_FUSED) instead of GEMM + backward")
     return ap.parse_args()
@@ -59,7 +61,7 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
 CSRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc")
 # the source files each profiled kernel is compiled from
 KERNEL_SOURCES = {
-    "k_backward": ["gsq_elementwise.cu", "gsq_relax.cuh"],
+    "k_backward": ["gsq_elementwise.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
     "k_step_fused": ["gsq_fused.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
 }
 
@@ -358,7 +360,7 @@ def gpu_arm(args, rank, world, local):
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
                       wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param,
-                      fused=args.fused)
+                      fused=args.fused, unstaged=args.unstaged)
     stream = torch.cuda.current_stream()
     loss = torch.zeros(1, device="cuda")
     T = w.steps
@@ -450,7 +452,8 @@ def gpu_arm(args, rank, world, local):
         bytes_bwd = w.elementwise_bytes_per_weight() * n
         bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
         gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
-        roofline = {"kernel": "k_backward (fused backward + Lion + next forward)", "bound": "hbm",
+        kname = "k_backward" if args.unstaged else "k_backward_staged"
+        roofline = {"kernel": f"{kname} (fused backward + Lion + next forward)", "bound": "hbm",
                     "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
                     "traffic": committed_traffic(w.name),
                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",

@@ -75,10 +75,14 @@ enum {
   GSQ_FLAG_NO_NOISE = 1u, /* g = 0: plain tempered softmax, no Gumbel draw             */
   GSQ_FLAG_KEEP_G = 2u,   /* with GSQ_FLAG_FUSED: the fused step also stores G, so
                              GSQ_T_G reads back the last step's dL/dW^                 */
-  GSQ_FLAG_FUSED = 4u     /* bf16 layers: gsq_step runs one fused kernel (contraction
+  GSQ_FLAG_FUSED = 4u,    /* bf16 layers: gsq_step runs one fused kernel (contraction
                              with the backward, Lion and look-ahead as its epilogue)
                              instead of two; the same results to rounding.  Measured
                              slower than the two kernels on GB300, hence opt-in.       */
+  GSQ_FLAG_UNSTAGED = 8u  /* gsq_step's backward reads its input streams with direct
+                             global loads instead of staging them through shared
+                             memory with bulk asynchronous copies; the same kernel
+                             body and the same results bit for bit (for comparison) */
 };
 enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1, GSQ_PARAM_MASK_SIGN = 2 };
 
@@ -232,7 +236,11 @@ GSQ_API gsq_status gsq_init_logits(gsq_layer* layer, const uint8_t* codes_dev, c
  * Kernels: the contraction and the backward (+ update + look-ahead) are two
  * kernels; with GSQ_FLAG_FUSED (bf16, not exporting) one fused kernel runs the
  * contraction with the rest as its epilogue, so G stays on chip (GSQ_T_G then
- * reads back only with GSQ_FLAG_KEEP_G).  The D of noise counter t lives in one
+ * reads back only with GSQ_FLAG_KEEP_G).  Outside export mode the backward
+ * brings its input streams into shared memory with bulk asynchronous copies a
+ * tile of 1,024 weights ahead (unless GSQ_FLAG_UNSTAGED, or the layer is too
+ * small to give each block more than one tile); the results are the same bit
+ * for bit, apart from the summation order of the loss.  The D of noise counter t lives in one
  * of two buffers by the parity of t, so a look-ahead never overwrites the D
  * that its own step's contraction reads.
  * Never synchronises; graph-capturable for a fixed argument list. */

@@ -222,7 +222,8 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
   }
   if (d->gemm_precision != GSQ_GEMM_BF16 && d->gemm_precision != GSQ_GEMM_F32)
     return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
-  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE | GSQ_FLAG_KEEP_G | GSQ_FLAG_FUSED))
+  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE | GSQ_FLAG_KEEP_G | GSQ_FLAG_FUSED |
+                                         GSQ_FLAG_UNSTAGED))
     return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
   if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5 &&
       d->param_mode != GSQ_PARAM_MASK_SIGN)
@@ -264,6 +265,8 @@ struct gsq_layer {
   int device;
   int num_sms;
   int grid_fwd, grid_bwd;
+  int grid_bwd_staged;  // TMA-staged backward (non-export steps); 0: not used
+  int staged_plan;      // its staging plan
   bool tc;
   int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
   int group_n; // column group of the GEMM's tile order
@@ -595,6 +598,22 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   };
   L->grid_fwd = clamp_grid(ew_grid_size(sh.L, 0, L->num_sms, sh.mode));
   L->grid_bwd = clamp_grid(ew_grid_size(sh.L, 1, L->num_sms, sh.mode));
+  {
+    int lg = 0;
+    while ((1 << lg) < sh.group) ++lg;
+    const int frozen = (desc->lr_scales == 0.f && desc->wd_scales == 0.f) ? 1 : 0;
+    L->staged_plan = 0;
+    L->grid_bwd_staged =
+        (desc->flags & GSQ_FLAG_UNSTAGED)
+            ? 0
+            : ew_staged_grid(sh.L, sh.mode, sh.w_bf16, lg, frozen, L->num_sms, &L->staged_plan);
+    // staging pays only where every block gets more than one tile to overlap
+    // (a plan forced through GSQ_STAGED_PLAN applies at any size)
+    const bool forced = std::getenv("GSQ_STAGED_PLAN") != nullptr;
+    if (L->grid_bwd_staged > 0 && !forced && nq_blocks <= L->grid_bwd_staged)
+      L->grid_bwd_staged = 0;
+    if (L->grid_bwd_staged > 0) L->grid_bwd_staged = clamp_grid(L->grid_bwd_staged);
+  }
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
                              L->num_sms);
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128, 224 or 256: override the choice
@@ -755,7 +774,9 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
     L->g_valid = L->keep_g;
   } else {
     prof_begin(L, GSQ_K_BACKWARD, s, slot);
-    e = launch_backward(p, L->grid_bwd, s);
+    e = (!export_mode && L->grid_bwd_staged > 0)
+            ? launch_backward_staged(p, L->grid_bwd_staged, L->staged_plan, s)
+            : launch_backward(p, L->grid_bwd, s);
     prof_end(L, slot, s);
     if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
     L->g_valid = true;

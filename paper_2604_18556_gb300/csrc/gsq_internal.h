@@ -77,12 +77,24 @@ struct EwParams {
   float* loss_out;     // nullable
 };
 
+// Byte offsets of one stage's streams in the staged backward's shared memory
+// (a tile of 1,024 weights); bytes = stage size, tx = bytes the copies deliver.
+struct BwdStage {
+  uint32_t l, m, g, w, s, ms, j, bytes, tx;
+};
+
 // Records `msg` as this thread's gsq_last_error() text and returns `st` (gsq_api.cu).
 gsq_status set_last_error(gsq_status st, const char* msg);
 
 // ---- launchers (gsq_elementwise.cu) ----------------------------------------
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
+// TMA-staged backward for non-export, non-accumulating steps: its grid for a
+// layer (resident blocks x SMs) and staging plan, 0 where it does not apply;
+// and its launch.
+int ew_staged_grid(int K, int mode, int w_bf16, int log2_group, int scales_frozen, int num_sms,
+                   int* plan);
+cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s);
 int ew_grid_size(int K, int which, int num_sms, int mode);  // which: 0 forward, 1 backward
 
 struct InitParams {

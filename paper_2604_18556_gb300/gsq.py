@@ -28,7 +28,7 @@ GSQ_DTYPE_F32, GSQ_DTYPE_BF16 = 0, 1
 GSQ_CALIB_H, GSQ_CALIB_X, GSQ_CALIB_BATCHES = 0, 1, 2
 GSQ_SCALE_GROUP, GSQ_SCALE_KQUANT2 = 0, 1
 GSQ_GEMM_BF16, GSQ_GEMM_F32 = 0, 1
-GSQ_FLAG_NO_NOISE, GSQ_FLAG_KEEP_G, GSQ_FLAG_FUSED = 1, 2, 4
+GSQ_FLAG_NO_NOISE, GSQ_FLAG_KEEP_G, GSQ_FLAG_FUSED, GSQ_FLAG_UNSTAGED = 1, 2, 4, 8
 GSQ_PARAM_FULL, GSQ_PARAM_SHIFT5, GSQ_PARAM_MASK_SIGN = 0, 1, 2
 PARAM_MODES = {"full": GSQ_PARAM_FULL, "shift5": GSQ_PARAM_SHIFT5, "mask_sign": GSQ_PARAM_MASK_SIGN}
 (GSQ_T_LOGITS, GSQ_T_SCALES, GSQ_T_MOM_LOGITS, GSQ_T_MOM_SCALES, GSQ_T_D, GSQ_T_G, GSQ_T_W,
@@ -244,7 +244,8 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
               lr_scales: float = 5e-5, beta1: float = 0.9, beta2: float = 0.95,
               wd_logits: float = 1.0, wd_scales: float = 0.0, gemm: int = GSQ_GEMM_BF16,
               noise: bool = True, param_mode: int = GSQ_PARAM_FULL,
-              keep_g: bool = False, fused: bool = False) -> gsq_layer_desc:
+              keep_g: bool = False, fused: bool = False,
+              unstaged: bool = False) -> gsq_layer_desc:
     d = gsq_layer_desc()
     d.num_experts, d.out_features, d.in_features = experts, rows, cols
     d.w_dtype = w_dtype
@@ -258,7 +259,7 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
     d.scale_mode = scale_mode
     d.init_bias = init_bias
     d.flags = (0 if noise else GSQ_FLAG_NO_NOISE) | (GSQ_FLAG_KEEP_G if keep_g else 0) | \
-        (GSQ_FLAG_FUSED if fused else 0)
+        (GSQ_FLAG_FUSED if fused else 0) | (GSQ_FLAG_UNSTAGED if unstaged else 0)
     d.seed = seed
     d.lr_logits, d.lr_scales = lr_logits, lr_scales
     d.beta1, d.beta2 = beta1, beta2

@@ -207,7 +207,7 @@ class Case:
 
     def __init__(self, w: C.Workload, gemm: str = "f32", noise: bool = True, seed=None,
                  keep_calib_host: bool = True, device="cuda", keep_g: bool = False,
-                 fused: bool = False):
+                 fused: bool = False, unstaged: bool = False):
         g = gsq()
         self.w = w
         self.gemm = gemm
@@ -221,7 +221,7 @@ class Case:
         hyper = dict(init_bias=w.init_bias, seed=w.seed if seed is None else seed,
                      lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise, keep_g=keep_g,
-                     fused=fused)
+                     fused=fused, unstaged=unstaged)
         self.layer = g.Layer(self.W, self.calib, w.grid, w.group, calib_kind=w.calib,
                              scale_mode=w.scale_mode, gemm=gemm, param=w.param,
                              tokens_per_batch=w.tokens if w.calib == "batches" else 0, **hyper)

@@ -452,14 +452,15 @@ def gpu_arm(args, rank, world, local):
         bytes_bwd = w.elementwise_bytes_per_weight() * n
         bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
         gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
-        kname = "k_backward" if args.unstaged else "k_backward_staged"
+        kname = layer.kernel_name(gsq.GSQ_K_BACKWARD)
         roofline = {"kernel": f"{kname} (fused backward + Lion + next forward)", "bound": "hbm",
                     "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
                     "traffic": committed_traffic(w.name),
                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
                     "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
                     "frac_of_8TBps": bwd_gbs / 8000.0}
-        roofline_gemm = {"kernel": "k_tc_gemm (tcgen05 loss contraction)", "bound": "tensor",
+        roofline_gemm = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} (tcgen05 loss contraction)",
+                         "bound": "tensor",
                          "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
                          "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
                          "flops_per_launch": flops, "avg_launch_ms": gemm_avg,

@@ -419,6 +419,14 @@ GSQ_API const char* gsq_last_error(void);
 /* Library version, "major.minor.patch". */
 GSQ_API const char* gsq_version(void);
 
+/* Name of the kernel that gsq_step launches for the part `kind` of a
+ * non-exporting step of this layer (GSQ_K_GEMM: "k_tc_gemm_pair",
+ * "k_tc_gemm", "k_simt_gemm" or "k_step_fused"; GSQ_K_BACKWARD:
+ * "k_backward_staged", "k_backward" or "k_step_fused"), so timings can be
+ * attributed (the paper has no counterpart: a reporting aid).  Static string
+ * owned by the library; NULL for an invalid handle or another kind. */
+GSQ_API const char* gsq_kernel_name(gsq_layer* layer, int32_t kind);
+
 #ifdef __cplusplus
 }
 #endif

@@ -271,6 +271,7 @@ struct gsq_layer {
   int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
   int group_n; // column group of the GEMM's tile order
   int fused_group_n;  // row-tile group of the fused step's tile order (1: whole rows first)
+  int gemm_pair;      // 1: the loss GEMM runs on CTA pairs (cta_group::2)
   bool fused;   // GSQ_FLAG_FUSED: gsq_step runs the fused step kernel (bf16, not exporting)
   bool keep_g;  // GSQ_FLAG_KEEP_G: the fused step also stores G
   bool g_valid; // the G buffer holds the last step's G
@@ -451,6 +452,7 @@ gsq_status launch_gemm(gsq_layer* L, size_t doff, cudaStream_t s) {
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = L->tile_n;
     g.group_n = L->group_n;
+    g.pair = L->gemm_pair;
     e = launch_tc_gemm(g, L->num_sms, s);
   } else {
     SimtGemm g;
@@ -621,6 +623,10 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
   L->group_n = kGemmGroupN;
+  // CTA pairs by default (measured 1-4% faster than single CTAs on the 4096 x 4096,
+  // 4096 x 14336 and 64-expert layers); GSQ_GEMM_PAIR=0 selects single CTAs
+  L->gemm_pair = 1;
+  if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) L->gemm_pair = std::atoi(gp) == 0 ? 0 : 1;
   // the fused step's tile order: groups of row tiles, as for the GEMM (whole rows
   // first measured no faster)
   L->fused_group_n = kGemmGroupN;
@@ -842,6 +848,7 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = 0;
     g.group_n = L->group_n;
+    g.pair = L->gemm_pair;
     g.E = E;
     if (e == cudaSuccess) {  // Y[e] = D[e] X[e]^T  (N = T, K = C), bf16 out
       g.M = R; g.N = T; g.K = C;
@@ -1176,5 +1183,19 @@ gsq_status gsq_destroy(gsq_layer* L) {
 const char* gsq_last_error(void) { return g_last_error.c_str(); }
 
 const char* gsq_version(void) { return "0.1.0"; }
+
+const char* gsq_kernel_name(gsq_layer* L, int32_t kind) {
+  if (!valid(L)) return nullptr;
+  if (kind == GSQ_K_GEMM) {
+    if (L->fused) return "k_step_fused";
+    if (!L->shape.d_bf16) return "k_simt_gemm";
+    return L->gemm_pair ? "k_tc_gemm_pair" : "k_tc_gemm";
+  }
+  if (kind == GSQ_K_BACKWARD) {
+    if (L->fused) return "k_step_fused";
+    return L->grid_bwd_staged > 0 ? "k_backward_staged" : "k_backward";
+  }
+  return nullptr;
+}
 
 }  // extern "C"

@@ -4,15 +4,18 @@
 // "K-major" operands (the contraction index is contiguous) and H^T = H gives
 // G = 2 D H_sym = dL/dW^ of L = tr(D H D^T) (Eq. 1 with a linear layer).
 //
-// Persistent, warp-specialised kernel, one CTA per SM:
-//   warp 0     TMA producer: 128x64 tile of D and 256x64 tile of H per stage,
-//              128-byte swizzle, into a 4-stage shared-memory ring;
+// Two persistent, warp-specialised kernels: k_tc_gemm (one CTA per SM, below)
+// and k_tc_gemm_pair (CTA pairs sharing one cta_group::2 MMA, the default; see
+// its own comment).  k_tc_gemm:
+//   warp 0     TMA producer: 128x64 tile of D and BNx64 tile of H per stage
+//              (BN = 128, 224 or 256), 128-byte swizzle, into a ring of as many
+//              stages as shared memory holds;
 //   warp 1     TMEM allocator and MMA issuer: tcgen05.mma.cta_group::1.kind::f16
-//              M=128 N=256 K=16, four per 64-wide k-block, accumulating in TMEM;
+//              M=128 N=BN K=16, four per 64-wide k-block, accumulating in TMEM;
 //              tcgen05.commit frees a stage / publishes a finished accumulator;
 //   warps 2-5  epilogue: tcgen05.ld 32x32b of the accumulator (each warp owns
 //              the 32 TMEM lanes of its quarter), scale by alpha, store fp32.
-// The accumulator is double-buffered in TMEM (2 x 256 columns) so the epilogue
+// The accumulator is double-buffered in TMEM (2 x BN columns) so the epilogue
 // of tile i overlaps the MMAs of tile i+1.  Every mbarrier wait is bounded
 // (2 s of %globaltimer); on expiry the CTA records an error code in the
 // workspace flags, waits (bounded) for its own in-flight copies, frees its TMEM
@@ -277,6 +280,222 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicExch(&args.flags->error, 0x7C01u);
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair variant: a cluster of two CTAs on neighbouring SMs computes a
+// 256 x BN output tile with tcgen05.mma.cta_group::2.  Each CTA stages its own
+// 128 rows of A and its half (BN/2 rows) of B, so a stage is 16 KiB + BN KiB/8
+// (30 KiB at BN = 224, 7 stages) and every SM streams a third less operand
+// data than a single CTA with the same tile width.  Both CTAs' copies complete
+// on the leader's (rank 0) full barrier; the leader's single MMA thread issues
+// for the pair and its commits arrive on the empty / accumulator barriers of
+// both CTAs.  Each CTA's epilogue drains its own TMEM (its 128 rows) and
+// arrives on the leader's accumulator-empty barrier.  Waits are bounded as in
+// k_tc_gemm; a CTA that gives up records the error, lets its copies in flight
+// land (a bounded pause) and meets its peer at the final cluster barrier.
+// ---------------------------------------------------------------------------
+constexpr int TC2_BM = 256;  // rows per pair tile (128 per CTA)
+
+template <int BN>
+struct Tc2Cfg {
+  static constexpr int kBHalf = BN / 2;
+  static constexpr int kBBytes = kBHalf * TC_BK * 2;
+  static constexpr int kStageBytes = TC_A_BYTES + kBBytes;
+  static constexpr int kStages =
+      ((232448 - 2048) / kStageBytes) < 8 ? ((232448 - 2048) / kStageBytes) : 8;
+  static constexpr int kTmemCols = 2 * BN <= 256 ? 256 : 512;
+  static constexpr int kAccStride = kTmemCols / 2;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
+  static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                                     (static_cast<uint32_t>(BN >> 3) << 17) |
+                                     (static_cast<uint32_t>(TC2_BM >> 4) << 24);
+  static_assert(kBHalf % 8 == 0, "B half must be whole 8-row swizzle atoms");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1 KiB alignment");
+};
+
+template <int BN>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    k_tc_gemm_pair(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const TcArgs args) {
+  using Cfg = Tc2Cfg<BN>;
+  constexpr int STAGES = Cfg::kStages;
+  constexpr int STAGE_BYTES = Cfg::kStageBytes;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty_bar = full_bar + STAGES;
+  uint64_t* tfull_bar = empty_bar + STAGES;
+  uint64_t* tempty_bar = tfull_bar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: leader, 1: peer
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar + s, 1);
+      mbar_init(empty_bar + s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar + a, 1);
+      mbar_init(tempty_bar + a, 8);  // one arrival per epilogue warp of both CTAs
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(Cfg::kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist before any copy or arrival reaches them
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int Mt = (args.M + TC2_BM - 1) / TC2_BM;
+  const int Nt = (args.N + BN - 1) / BN;
+  const int KB = (args.K + TC_BK - 1) / TC_BK;
+  const int tiles = args.E * Mt * Nt;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (both CTAs) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = pair; ok && tile < tiles; tile += npairs) {
+        int e, m, n;
+        tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+        const int arow = e * args.M + m * TC2_BM + static_cast<int>(rank) * TC_BM;
+        const int brow = e * args.N + n * BN + static_cast<int>(rank) * Cfg::kBHalf;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(empty_bar + stage, phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + stage * STAGE_BYTES;
+          uint8_t* sb = sa + TC_A_BYTES;
+          const uint32_t fb = mapa_shared(smem_u32(full_bar + stage), 0);
+          if (rank == 0) mbar_expect_tx(full_bar + stage, 2 * STAGE_BYTES);
+          tma_load_2d_pair(sa, &tmA, fb, kb * TC_BK, arow);
+          tma_load_2d_pair(sb, &tmB, fb, kb * TC_BK, brow);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // copies in flight complete on the leader's barrier: give them time to land
+        const unsigned long long t0 = global_ns();
+        while (global_ns() - t0 < 200000ull) __nanosleep(1000);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (leader only, for the pair) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = pair; ok && tile < tiles; tile += npairs) {
+        if (!mbar_wait(tempty_bar + acc, acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride);
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(full_bar + stage, phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint64_t da = sw128_desc(sa);
+          const uint64_t db = sw128_desc(sa + TC_A_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, Cfg::kIdesc, (kb | k) != 0 ? 1u : 0u);
+          umma_commit_pair(empty_bar + stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit_pair(tfull_bar + acc);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
+    const int quarter = warp & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = pair; tile < tiles; tile += npairs) {
+      if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
+      tc_fence_after();
+      int e, m, n;
+      tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+      const int row = m * TC2_BM + static_cast<int>(rank) * TC_BM + quarter * 32 + lane;
+      const int col0 = n * BN;
+      const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride) +
+                             (static_cast<uint32_t>(quarter * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 16) {
+        float v[16];
+        tmem_ld16(taddr + c, v);
+        if (row < args.M) {
+#pragma unroll
+          for (int j = 0; j < 16; j += 4) {
+            const int col = col0 + c + j;
+            if (col < args.N) {
+              const float4 o = make_float4(args.alpha * v[j], args.alpha * v[j + 1],
+                                           args.alpha * v[j + 2], args.alpha * v[j + 3]);
+              if (args.out_bf16) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(o.x, o.y);
+                const __nv_bfloat162 hi = __floats2bfloat162_rn(o.z, o.w);
+                uint2 raw;
+                raw.x = *reinterpret_cast<const uint32_t*>(&lo);
+                raw.y = *reinterpret_cast<const uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(args.out) + obase + col) = raw;
+              } else {
+                *reinterpret_cast<float4*>(static_cast<float*>(args.out) + obase + col) = o;
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(tempty_bar + acc), 0));
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // neither CTA leaves while the pair's MMAs or arrivals may touch it
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(Cfg::kTmemCols));
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(&args.flags->error, 0x7C04u);
+}
+
 bool tc_supported_impl(int device) {
   cudaDeviceProp prop;
   if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return false;
@@ -322,6 +541,61 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+template <int BN>
+cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
+  using Cfg = Tc2Cfg<BN>;
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm_pair<BN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  CUtensorMap ta, tb;
+  if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;
+  if (!encode_kmajor_bf16(&ta, g.A, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.M, TC_BM) ||
+      !encode_kmajor_bf16(&tb, g.B, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.N, Cfg::kBHalf))
+    return cudaErrorInvalidValue;
+  TcArgs a;
+  a.E = g.E;
+  a.M = g.M;
+  a.N = g.N;
+  a.K = g.K;
+  a.group_n = g.group_n > 0 ? g.group_n : (g.N + BN - 1) / BN;
+  a.out = g.out;
+  a.out_bf16 = g.out_bf16;
+  a.alpha = g.alpha;
+  a.flags = g.flags;
+  const int Mt = (g.M + TC2_BM - 1) / TC2_BM, Nt = (g.N + BN - 1) / BN;
+  const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
+  int pairs = num_sms / 2;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(TC_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
+  int max_clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&max_clusters, k_tc_gemm_pair<BN>, &cfg) != cudaSuccess ||
+      max_clusters < 1) {
+    cudaGetLastError();
+    return launch_tc_gemm_bn<BN>(g, num_sms, s);  // no CTA pair can be resident: single CTAs
+  }
+  if (max_clusters < pairs) pairs = max_clusters;
+  if (tiles < pairs) pairs = static_cast<int>(tiles);
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_pair<BN>, ta, tb, a);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 }  // namespace
 
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
@@ -346,6 +620,11 @@ int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
 
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
   const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms);
+  if (g.pair && num_sms >= 2) {
+    if (bn == 128) return launch_tc_gemm_pair_bn<128>(g, num_sms, s);
+    if (bn == 224) return launch_tc_gemm_pair_bn<224>(g, num_sms, s);
+    return launch_tc_gemm_pair_bn<256>(g, num_sms, s);
+  }
   if (bn == 128) return launch_tc_gemm_bn<128>(g, num_sms, s);
   if (bn == 224) return launch_tc_gemm_bn<224>(g, num_sms, s);
   return launch_tc_gemm_bn<256>(g, num_sms, s);

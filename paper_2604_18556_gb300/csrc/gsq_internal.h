@@ -228,6 +228,7 @@ struct TcGemm {
   DevFlags* flags;
   int tile_n;   // 0: choose 128 or 256 by wave balance
   int group_n;  // tile-order column group; <= 0: one group (m fastest across all columns)
+  int pair;     // 1: CTA pairs (cta_group::2, 256-row tiles over two SMs)
 };
 bool tc_gemm_supported(int device);
 

@@ -42,7 +42,7 @@ EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
             "gsq_sync_status", "gsq_profile_enable", "gsq_profile_read", "gsq_destroy",
             "gsq_last_error", "gsq_version", "gsq_backward_update_noalloc", "gsq_init_logits",
-            "gsq_step_tokens", "gsq_diagnose"]
+            "gsq_step_tokens", "gsq_diagnose", "gsq_kernel_name"]
 
 
 GSQ_DIAG_SHIFT_BINS, GSQ_DIAG_MARGIN_BINS = 8, 9
@@ -109,6 +109,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "gsq_destroy": (c_int32, [P]),
         "gsq_last_error": (c_char_p, []),
         "gsq_version": (c_char_p, []),
+        "gsq_kernel_name": (c_char_p, [P, c_int32]),
         "gsq_backward_update_noalloc": (c_int32, [POINTER(gsq_backward_args), P]),
         "gsq_init_logits": (c_int32, [P, P, P, c_float, c_float, P]),
         "gsq_diagnose": (c_int32, [P, c_float, c_float, P, POINTER(gsq_diagnostics)]),
@@ -231,6 +232,12 @@ def gsq_version() -> str:
     return _lib.gsq_version().decode()
 
 
+def gsq_kernel_name(handle, kind: int):
+    """The kernel gsq_step launches for GSQ_K_GEMM or GSQ_K_BACKWARD, or None."""
+    r = _lib.gsq_kernel_name(handle, kind)
+    return None if r is None else r.decode()
+
+
 def gsq_backward_update_noalloc(args: gsq_backward_args, stream: int) -> None:
     """The allocation-free backward + Lion update (see include/gsq.h)."""
     _check(_lib.gsq_backward_update_noalloc(byref(args), stream))
@@ -338,6 +345,10 @@ class Layer:
         codes = codes.contiguous()
         eps = None if eps is None else eps.contiguous()
         gsq_init_logits(self.handle, _ptr(codes), _ptr(eps), alpha, sigma, self._stream())
+
+    def kernel_name(self, kind: int):
+        """Kernel gsq_step launches for GSQ_K_GEMM or GSQ_K_BACKWARD on this layer."""
+        return gsq_kernel_name(self.handle, kind)
 
     def diagnose(self, tau: float, kappa: float = 1.0) -> dict:
         """Displacement and margin histograms and the mean max-probability (see gsq.h)."""

@@ -235,9 +235,10 @@ def test_trajectory_ternary_full_run():
 @pytest.mark.parametrize("tile_n", ["128", "224", "256"])
 @pytest.mark.parametrize("name", ["q_proj", "gate_proj", "moe_kquant"])
 def test_tc_gemm_tile_widths(name, tile_n, monkeypatch):
-    """Every tensor-core tile width (chosen per layer by wave balance) on ragged
+    """The single-CTA contraction: every tensor-core tile width (chosen per layer by wave balance) on ragged
     shapes, against exact products of the kernel's own bf16 operands."""
     monkeypatch.setenv("GSQ_GEMM_TILE_N", tile_n)
+    monkeypatch.setenv("GSQ_GEMM_PAIR", "0")  # single CTAs (pairs: test_tc_gemm_cta_pairs)
     w = SMALL[name]
     case = Case(w, gemm="bf16")
     loss = torch.zeros(1, device="cuda")
@@ -248,4 +249,34 @@ def test_tc_gemm_tile_widths(name, tile_n, monkeypatch):
     for e in range(w.experts):
         sel = rows // w.rows == e
         assert_gemm_bound(G[sel], D[sel], H[e], f"tile N = {tile_n}, expert {e}")
+    assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())
+
+
+PAIR_CASES = dict(SMALL, **{
+    # 2,000 rows: eight 256-row pair tiles, the last ragged; 2,688 columns: 12 tiles 224
+    # wide, 11 (the last ragged) 256 wide, 21 of 128; 42 k-blocks; more tiles (88 to
+    # 168) than CTA pairs on the GPU, so every pair runs several
+    "q_proj_multi_wave": C.shrunk(W["llama8b_q_proj"], rows=2000, cols=2688, tokens=4096),
+})
+
+
+@pytest.mark.parametrize("tile_n", ["128", "224", "256"])
+@pytest.mark.parametrize("name", ["q_proj", "gate_proj", "moe_kquant", "q_proj_multi_wave"])
+def test_tc_gemm_cta_pairs(name, tile_n, monkeypatch):
+    """The CTA-pair contraction (tcgen05.mma.cta_group::2, 256-row tiles over two SMs)
+    at every tile width on ragged shapes and several experts, against exact products of
+    the kernel's own bf16 operands, and the loss as 1/2 sum D G."""
+    monkeypatch.setenv("GSQ_GEMM_TILE_N", tile_n)
+    monkeypatch.setenv("GSQ_GEMM_PAIR", "1")
+    w = PAIR_CASES[name]
+    case = Case(w, gemm="bf16")
+    loss = torch.zeros(1, device="cuda")
+    case.layer.step(0, TAU.get(name, 0.55), 1.0, loss=loss)
+    torch.cuda.synchronize()
+    case.layer.sync_status()
+    D, H, G = case.D(), case.H_operand(), case.G()
+    rows = np.arange(w.experts * w.rows)
+    for e in range(w.experts):
+        sel = rows // w.rows == e
+        assert_gemm_bound(G[sel], D[sel], H[e], f"pairs, tile N = {tile_n}, expert {e}")
     assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())

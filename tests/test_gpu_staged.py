@@ -83,3 +83,22 @@ def test_staged_backward_is_bit_identical(name, plan, monkeypatch):
                            Db.view(torch.int16 if gemm == "bf16" else torch.int32)), t
     # the steps did update the state
     assert not np.array_equal(staged.logits(), start)
+
+
+def test_kernel_names_follow_the_layer():
+    """gsq_kernel_name reports what gsq_step launches: staged up to 4 logits per weight
+    on layers with more tiles than resident blocks, direct loads with 5 (local shift),
+    on request and on small layers; the CTA-pair contraction by default."""
+    g = gsq()
+    big = C.shrunk(Q, rows=999, cols=1280, tokens=2048)
+    cases = [(big, {}, "k_backward_staged"),
+             (big, {"unstaged": True}, "k_backward"),
+             (CASES["shift5"], {}, "k_backward"),
+             (CASES["k4_below_one_tile"], {}, "k_backward")]
+    for w, kw, want in cases:
+        case = Case(w, gemm="bf16", **kw)
+        assert case.layer.kernel_name(g.GSQ_K_BACKWARD) == want, (w.name, kw)
+        assert case.layer.kernel_name(g.GSQ_K_GEMM) == "k_tc_gemm_pair"
+        assert case.layer.kernel_name(g.GSQ_K_PROJECT) is None
+    f32 = Case(CASES["k3_fp32_w"], gemm="f32")
+    assert f32.layer.kernel_name(g.GSQ_K_GEMM) == "k_simt_gemm"

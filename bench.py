@@ -571,7 +571,8 @@ def gpu_arm_tokens(args, rank, world, local):
     gemm_tfs = flops_per_launch / (gemm_avg * 1e-3) / 1e12
     bytes_step = w.elementwise_bytes_per_step()
     bwd_gbs = bytes_step / (bwd_ms / args.steps * 1e-3) / 1e9
-    roofline = {"kernel": "k_tc_gemm x 2 (Y = D X^T, then G = 2 Y X; tcgen05, bf16 in, fp32 acc)",
+    roofline = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} x 2 (Y = D X^T, then G = 2 Y X; "
+                          "tcgen05, bf16 in, fp32 acc)",
                 "bound": "tensor", "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
                 "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst, "traffic": None,
                 "flops_per_launch": flops_per_launch, "avg_launch_ms": gemm_avg,

@@ -616,17 +616,17 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
       L->grid_bwd_staged = 0;
     if (L->grid_bwd_staged > 0) L->grid_bwd_staged = clamp_grid(L->grid_bwd_staged);
   }
+  // CTA pairs by default (at the same tile width measured 1-4% faster than single CTAs on the 4096 x 4096,
+  // 4096 x 14336 and 64-expert layers); GSQ_GEMM_PAIR=0 selects single CTAs
+  L->gemm_pair = 1;
+  if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) L->gemm_pair = std::atoi(gp) == 0 ? 0 : 1;
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
-                             L->num_sms);
+                             L->num_sms, L->gemm_pair);
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128, 224 or 256: override the choice
     const int v = std::atoi(tn);
     if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
   L->group_n = kGemmGroupN;
-  // CTA pairs by default (measured 1-4% faster than single CTAs on the 4096 x 4096,
-  // 4096 x 14336 and 64-expert layers); GSQ_GEMM_PAIR=0 selects single CTAs
-  L->gemm_pair = 1;
-  if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) L->gemm_pair = std::atoi(gp) == 0 ? 0 : 1;
   // the fused step's tile order: groups of row tiles, as for the GEMM (whole rows
   // first measured no faster)
   L->fused_group_n = kGemmGroupN;

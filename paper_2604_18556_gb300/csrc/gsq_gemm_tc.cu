@@ -600,7 +600,20 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
 
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
 
-int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
+int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair) {
+  if (pair) {
+    // CTA pairs (256-row tiles over two SMs, 7-stage rings at both widths): 256-wide
+    // tiles unless they take more waves x width than 224-wide ones.  Measured on
+    // GB300: 4096 x 14336 886 vs 955 us, 28672 x 8192 2.11 vs 2.21 ms, 64 experts
+    // 2048 x 7168 7.27 vs 7.69 ms; on 4096 x 4096, 224 wide (4 full waves) wins.
+    const int pairs = num_sms / 2 > 0 ? num_sms / 2 : 1;
+    const int64_t mt2 = (M + 255) / 256;
+    auto pcost = [&](int bn) {
+      const int64_t tiles = static_cast<int64_t>(E) * mt2 * ((N + bn - 1) / bn);
+      return static_cast<double>((tiles + pairs - 1) / pairs) * bn;
+    };
+    return pcost(256) <= pcost(224) ? 256 : 224;
+  }
   // 224-wide tiles by default: their 44 KiB stages give a 5-deep ring against 4 for
   // 256-wide ones, which measured faster on GB300 on every layer shape here (4096 x
   // 4096: 99 vs 111 us; 4096 x 14336: 1.00 vs 1.03 ms; 64 experts 2048 x 7168: 8.26
@@ -619,7 +632,7 @@ int tc_gemm_tile_n(int E, int M, int N, int num_sms) {
 }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
-  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms);
+  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms, g.pair);
   if (g.pair && num_sms >= 2) {
     if (bn == 128) return launch_tc_gemm_pair_bn<128>(g, num_sms, s);
     if (bn == 224) return launch_tc_gemm_pair_bn<224>(g, num_sms, s);

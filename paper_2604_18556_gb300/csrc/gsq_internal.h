@@ -246,7 +246,7 @@ struct FusedStep {
   int group_n;   // tile order: groups of row tiles
 };
 cudaError_t launch_step_fused(const FusedStep& f, int num_sms, cudaStream_t s);
-int tc_gemm_tile_n(int E, int M, int N, int num_sms);
+int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 
 }  // namespace gsq

@@ -272,6 +272,7 @@ struct gsq_layer {
   int group_n; // column group of the GEMM's tile order
   int fused_group_n;  // row-tile group of the fused step's tile order (1: whole rows first)
   int gemm_pair;      // 1: the loss GEMM runs on CTA pairs (cta_group::2)
+  int test_stall;     // test hook (GSQ_TEST_STALL): 1 staged backward, 2 tensor-core GEMM
   bool fused;   // GSQ_FLAG_FUSED: gsq_step runs the fused step kernel (bf16, not exporting)
   bool keep_g;  // GSQ_FLAG_KEEP_G: the fused step also stores G
   bool g_valid; // the G buffer holds the last step's G
@@ -364,6 +365,7 @@ EwParams base_params(gsq_layer* L) {
   p.scales_frozen = (d.lr_scales == 0.f && d.wd_scales == 0.f) ? 1 : 0;
   p.loss_partials = reinterpret_cast<double*>(L->ws + L->lay.partials);
   p.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
+  p.stall = L->test_stall == 1 ? 1 : 0;
   return p;
 }
 
@@ -439,7 +441,8 @@ gsq_status launch_gemm(gsq_layer* L, size_t doff, cudaStream_t s) {
   prof_begin(L, GSQ_K_GEMM, s, slot);
   cudaError_t e;
   if (sh.d_bf16) {
-    TcGemm g;  // G = 2 D H (H symmetrised, so its rows are K-major columns)
+    TcGemm g{};  // G = 2 D H (H symmetrised, so its rows are K-major columns)
+    g.stall = L->test_stall == 2 ? 1 : 0;
     g.E = static_cast<int>(sh.E);
     g.M = static_cast<int>(sh.R);
     g.N = static_cast<int>(sh.C);
@@ -620,6 +623,12 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   // 4096 x 14336 and 64-expert layers); GSQ_GEMM_PAIR=0 selects single CTAs
   L->gemm_pair = 1;
   if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) L->gemm_pair = std::atoi(gp) == 0 ? 0 : 1;
+  // Test hook for the bounded device-side waits: GSQ_TEST_STALL=backward makes the staged
+  // backward skip one stage fill, =gemm makes the tensor-core GEMM skip its first k-block;
+  // the waits on it give up after 2 s and gsq_sync_status reports GSQ_ERR_TIMEOUT.
+  L->test_stall = 0;
+  if (const char* ts = std::getenv("GSQ_TEST_STALL"))
+    L->test_stall = std::strcmp(ts, "backward") == 0 ? 1 : (std::strcmp(ts, "gemm") == 0 ? 2 : 0);
   L->tile_n = tc_gemm_tile_n(static_cast<int>(sh.E), static_cast<int>(sh.R), static_cast<int>(sh.C),
                              L->num_sms, L->gemm_pair);
   if (const char* tn = std::getenv("GSQ_GEMM_TILE_N")) {   // 128, 224 or 256: override the choice
@@ -844,7 +853,8 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
   }
   prof_begin(L, GSQ_K_GEMM, s, slot);
   if (sh.d_bf16) {
-    TcGemm g;
+    TcGemm g{};
+    g.stall = L->test_stall == 2 ? 1 : 0;
     g.flags = reinterpret_cast<DevFlags*>(L->ws + L->lay.flags);
     g.tile_n = 0;
     g.group_n = L->group_n;

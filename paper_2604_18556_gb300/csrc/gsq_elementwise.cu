@@ -403,7 +403,7 @@ __global__ void __launch_bounds__(kEwThreads, Plan::kOcc)
   if (tid == 0) {
 #pragma unroll
     for (int b = 0; b < 2; ++b) {
-      if (first + b * stride < ntiles) {
+      if (first + b * stride < ntiles && !(P.stall && b == 1)) {
         stage_issue<K, kShift, kStageM, kStageGW>(P, S, stage_mem + b * S.bytes, &full[b], first + b * stride);
         issued[b] = 1u;
       }

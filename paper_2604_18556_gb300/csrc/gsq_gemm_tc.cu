@@ -86,6 +86,7 @@ struct TcCfg {
 };
 
 struct TcArgs {
+  int stall;      // test hook: skip the first k-block's copies, so the waits on it run out
   int E, M, N, K;
   int group_n;    // tile-order column group (tile_coords)
   void* out;      // [E][M][N], fp32 or bf16
@@ -166,11 +167,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
           uint8_t* sa = smem + stage * TC_STAGE_BYTES;
           uint8_t* sb = sa + TC_A_BYTES;
-          mbar_expect_tx(full_bar + stage, TC_STAGE_BYTES);
-          tma_load_2d(sa, &tmA, full_bar + stage, kb * TC_BK, arow);
-          tma_load_2d(sb, &tmB, full_bar + stage, kb * TC_BK, brow);
-          issued[stage] = true;
-          issued_phase[stage] = phase;
+          if (!(args.stall && tile == static_cast<int>(blockIdx.x) && kb == 0)) {
+            mbar_expect_tx(full_bar + stage, TC_STAGE_BYTES);
+            tma_load_2d(sa, &tmA, full_bar + stage, kb * TC_BK, arow);
+            tma_load_2d(sb, &tmB, full_bar + stage, kb * TC_BK, brow);
+            issued[stage] = true;
+            issued_phase[stage] = phase;
+          }
           if (++stage == TC_STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -382,9 +385,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           uint8_t* sa = smem + stage * STAGE_BYTES;
           uint8_t* sb = sa + TC_A_BYTES;
           const uint32_t fb = mapa_shared(smem_u32(full_bar + stage), 0);
-          if (rank == 0) mbar_expect_tx(full_bar + stage, 2 * STAGE_BYTES);
-          tma_load_2d_pair(sa, &tmA, fb, kb * TC_BK, arow);
-          tma_load_2d_pair(sb, &tmB, fb, kb * TC_BK, brow);
+          if (!(args.stall && tile == pair && kb == 0)) {
+            if (rank == 0) mbar_expect_tx(full_bar + stage, 2 * STAGE_BYTES);
+            tma_load_2d_pair(sa, &tmA, fb, kb * TC_BK, arow);
+            tma_load_2d_pair(sb, &tmB, fb, kb * TC_BK, brow);
+          }
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -534,6 +539,7 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   a.out_bf16 = g.out_bf16;
   a.alpha = g.alpha;
   a.flags = g.flags;
+  a.stall = g.stall;
   const int Mt = (g.M + TC_BM - 1) / TC_BM, Nt = (g.N + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
@@ -568,6 +574,7 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   a.out_bf16 = g.out_bf16;
   a.alpha = g.alpha;
   a.flags = g.flags;
+  a.stall = g.stall;
   const int Mt = (g.M + TC2_BM - 1) / TC2_BM, Nt = (g.N + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   int pairs = num_sms / 2;

@@ -75,6 +75,8 @@ struct EwParams {
   double* loss_partials;
   DevFlags* flags;
   float* loss_out;     // nullable
+  int stall;           // test hook (GSQ_TEST_STALL=backward): the staged backward never fills
+                       // its second stage, so a bounded wait runs out and reports 0x7C03
 };
 
 // Byte offsets of one stage's streams in the staged backward's shared memory
@@ -229,6 +231,7 @@ struct TcGemm {
   int tile_n;   // 0: choose 128 or 256 by wave balance
   int group_n;  // tile-order column group; <= 0: one group (m fastest across all columns)
   int pair;     // 1: CTA pairs (cta_group::2, 256-row tiles over two SMs)
+  int stall;    // test hook (GSQ_TEST_STALL=gemm): the first k-block is never loaded
 };
 bool tc_gemm_supported(int device);
 

@@ -455,13 +455,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
       const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride) +
                              (static_cast<uint32_t>(quarter * 32) << 16);
+      // 32 columns per TMEM load and wait (BN is a multiple of 32)
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 16) {
-        float v[16];
-        tmem_ld16(taddr + c, v);
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld32(taddr + c, v);
         if (row < args.M) {
 #pragma unroll
-          for (int j = 0; j < 16; j += 4) {
+          for (int j = 0; j < 32; j += 4) {
             const int col = col0 + c + j;
             if (col < args.N) {
               const float4 o = make_float4(args.alpha * v[j], args.alpha * v[j + 1],

@@ -61,7 +61,8 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
 CSRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc")
 # the source files each profiled kernel is compiled from
 KERNEL_SOURCES = {
-    "k_backward": ["gsq_elementwise.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
+    "k_backward": ["gsq_backward.cu", "gsq_staged.cu", "gsq_backward.cuh", "gsq_relax.cuh",
+                   "gsq_tc.cuh", "gsq_internal.h"],
     "k_step_fused": ["gsq_fused.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
 }
 

@@ -1,6 +1,7 @@
 // Elementwise kernels of the GSQ step (HBM-bound): initial state, forward
-// (noise + tempered softmax + soft weight, Alg. 1), fused backward + Lion
-// (+ the next step's forward), hard projection and packing.
+// (noise + tempered softmax + soft weight, Alg. 1), hard projection, packing and
+// diagnostics.  The fused backward + Lion (+ the next step's forward) is in
+// gsq_backward.cu and gsq_staged.cu.
 //
 // Data layout in HBM (n = E*R*C, flat index i = (e*R + r)*C + c):
 //   logits, logit momenta : K planes of n fp32 ([K][E][R][C]), so every level is
@@ -12,63 +13,14 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
-#include <cstdlib>
 #include <type_traits>
 
+#include "gsq_backward.cuh"
 #include "gsq_internal.h"
 #include "gsq_relax.cuh"
-#include "gsq_tc.cuh"
 
 namespace gsq {
 namespace {
-
-__device__ __forceinline__ void load_grid(const EwParams& P, float (&q)[kMaxLevels]) {
-#pragma unroll
-  for (int k = 0; k < kMaxLevels; ++k) q[k] = P.grid[k];
-}
-
-// Block-wide shared copy of the grid (local shift reads it with per-lane indices).
-__device__ __forceinline__ void fill_shared_grid(const EwParams& P, float* sgrid) {
-  if (threadIdx.x < kMaxLevels) sgrid[threadIdx.x] = P.grid[threadIdx.x];
-  __syncthreads();
-}
-
-
-// Deterministic loss reduction: per-block double partials, summed in block
-// order by the last block to finish (no device-side wait).
-__device__ __forceinline__ void reduce_loss(float acc, const EwParams& P) {
-  __shared__ double red[kEwThreads / 32];
-  __shared__ bool is_last;
-  double v = static_cast<double>(acc);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    double s = 0.0;
-    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
-    P.loss_partials[blockIdx.x] = s;
-    __threadfence();
-    const unsigned int prev = atomicAdd(&P.flags->blocks_done, 1u);
-    is_last = (prev == gridDim.x - 1);
-  }
-  __syncthreads();
-  if (is_last) {  // the whole last block sums the partials, in a fixed order
-    __threadfence();
-    double s = 0.0;
-    for (unsigned int b = threadIdx.x; b < gridDim.x; b += blockDim.x) s += __ldcg(P.loss_partials + b);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_down_sync(0xffffffffu, s, off);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      double t = 0.0;
-      for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += red[w];
-      if (P.loss_out) *P.loss_out = static_cast<float>(t);
-      P.flags->blocks_done = 0u;
-    }
-  }
-}
 
 // ---------------------------------------------------------------------------
 // Forward: D = s * w~ - W for step (t, tau, kappa); optional W^ export.
@@ -116,382 +68,6 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
     store_d4(P.D, qi, P.d_bf16, d);
     if (P.what) reinterpret_cast<float4*>(P.what)[qi] = make_float4(what[0], what[1], what[2], what[3]);
   }
-}
-
-// ---------------------------------------------------------------------------
-// Fused backward for step t: recompute the noise and the relaxation, loss
-// partial 1/2 D*G, logit gradients (App. B), per-group scale gradient by
-// warp shuffles, Lion in place; then (look-ahead) the forward of step t+1 from
-// the updated registers.  Bytes per weight with look-ahead (L logits per
-// weight): read 8L + 4 + b_W (+1 for j0), write 8L + 2 (D bf16).
-// ---------------------------------------------------------------------------
-// Blocks per SM the register budget aims for (measured best on GB300): two;
-// three for the two-logit relaxations, which fit in 85 registers.
-template <int K>
-struct BwdOcc {
-  static constexpr int value = 2;
-};
-template <>
-struct BwdOcc<2> {
-  static constexpr int value = 3;
-};
-
-// The per-quad body, shared by the kernel that loads its streams directly
-// (k_backward) and the one that stages them through shared memory
-// (k_backward_staged), so both do the same arithmetic.  l, m, gv, w, s, ms, j4
-// hold the quad's inputs (m unused in export mode; gv zero for inactive lanes);
-// l and m are updated in place.  Every lane of the warp calls it (the scale-group
-// sums are shuffles).
-template <class Rx, bool kExport, bool kShift, bool kAcc>
-__device__ __forceinline__ void bwd_quad(const EwParams& P, const float (&q)[kMaxLevels],
-                                         const float* sgrid, int lane, int seg, int64_t qi,
-                                         bool active, float (&l)[Rx::L][4], float (&m)[Rx::L][4],
-                                         float4 gv, const float (&w)[4], float s, float ms,
-                                         uint32_t j4, float2& loss2) {
-  constexpr int K = Rx::L;
-  const PhiloxKeys& keys = P.keys;
-  const int64_t qc = active ? qi : 0;
-  const int64_t gidx = (qc * 4) >> P.log2_group;
-  const float2 Gq[2] = {make_float2(gv.x, gv.y), make_float2(gv.z, gv.w)};
-  float2 ds2 = f2(0.0f);
-#pragma unroll
-  for (int pr = 0; pr < 2; ++pr) {
-    float2 l2[K], h[K];
-#pragma unroll
-    for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
-    Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
-    Rx::noise(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
-    const float2 wt = rx.relax(l2, h, P.kappa_log2, P.inv_tau);
-    const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
-    const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
-    loss2 = fma2(mul2(f2(0.5f), dj), Gq[pr], loss2);
-    ds2 = fma2(Gq[pr], wt, ds2);
-    const float2 A = mul2(f2(P.kappa_over_tau * s), Gq[pr]);
-#pragma unroll
-    for (int k = 0; k < K; ++k) {
-      // dL/dl_k = (kappa/tau) G s dw~/dl_k
-      float2 dl = mul2(A, rx.dsoft(k));
-      if (kAcc) {  // gradient accumulation: (this micro-batch + earlier ones) * scale
-        const float2 a = reinterpret_cast<const float2*>(P.acc_in_l + k * P.n)[2 * qc + pr];
-        dl = mul2(add2(dl, a), f2(P.acc_scale));
-      }
-      if (kExport) {
-        m[k][2 * pr] = dl.x;
-        m[k][2 * pr + 1] = dl.y;
-      } else {
-        // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l - lr wd l - lr sign(c);
-        // m <- b2 m + (1-b2) g.  The decay is one fma on l (no rounded 1 - lr wd).
-        const float2 mo = make_float2(m[k][2 * pr], m[k][2 * pr + 1]);
-        const float2 c = fma2(f2(P.b1), mo, mul2(f2(1.0f - P.b1), dl));
-        const float2 ln = add2(fma2(f2(-P.lrwd_l), l2[k], l2[k]),
-                               make_float2(-lr_sign(P.lr_l, c.x), -lr_sign(P.lr_l, c.y)));
-        const float2 mn = fma2(f2(P.b2), mo, mul2(f2(1.0f - P.b2), dl));
-        l[k][2 * pr] = ln.x; l[k][2 * pr + 1] = ln.y;
-        m[k][2 * pr] = mn.x; m[k][2 * pr + 1] = mn.y;
-      }
-    }
-  }
-  float ds = group_sum(ds2.x + ds2.y, seg);  // dL/ds_g = sum_{c in g} G_c w~_c
-  if (kAcc && P.acc_in_s) ds = (ds + P.acc_in_s[gidx]) * P.acc_scale;
-
-  if (kExport) {
-    if (kAcc) __syncwarp();  // every lane has read acc_in_s before its group leader rewrites it
-    if (active) {
-      if (P.grad_logits) {
-#pragma unroll
-        for (int k = 0; k < K; ++k)
-          reinterpret_cast<float4*>(P.grad_logits + k * P.n)[qi] =
-              make_float4(m[k][0], m[k][1], m[k][2], m[k][3]);
-      }
-      if (P.grad_scales && !P.scales_frozen && (lane & (seg - 1)) == 0) P.grad_scales[gidx] = ds;
-    }
-  } else {
-    if (!P.scales_frozen) {
-      const float c = fmaf(P.b1, ms, (1.0f - P.b1) * ds);
-      s = fmaf(-P.lrwd_s, s, s) - lr_sign(P.lr_s, c);
-      ms = fmaf(P.b2, ms, (1.0f - P.b2) * ds);
-    }
-    if (active) {
-#pragma unroll
-      for (int k = 0; k < K; ++k) {
-        __stcs(reinterpret_cast<float4*>(P.logits + k * P.n) + qi,
-               make_float4(l[k][0], l[k][1], l[k][2], l[k][3]));
-        __stcs(reinterpret_cast<float4*>(P.m_logits + k * P.n) + qi,
-               make_float4(m[k][0], m[k][1], m[k][2], m[k][3]));
-      }
-      if (!P.scales_frozen && (lane & (seg - 1)) == 0) {
-        P.scales[gidx] = s;
-        P.m_scales[gidx] = ms;
-      }
-    }
-  }
-  if (active) {
-    if (P.lookahead) {
-      // forward of the next pass from the (updated, or in export mode unchanged)
-      // logits and scale (Alg. 1)
-      float d[4];
-#pragma unroll
-      for (int pr = 0; pr < 2; ++pr) {
-        float2 l2[K], h[K];
-#pragma unroll
-        for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
-        const Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
-        Rx::noise(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
-        const float2 wt = rx.value(l2, h, P.kappa_log2_next, P.inv_tau_next);
-        const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
-        d[2 * pr] = dd.x;
-        d[2 * pr + 1] = dd.y;
-      }
-      store_d4(P.D, qi, P.d_bf16, d);
-    }
-  }
-}
-
-// Direct loads of quad qi's inputs.  Lanes past the end (only in the last warp)
-// read quad 0 and take G = 0, so every value stays finite and their loss and
-// scale-gradient terms vanish; nothing is stored for them.  A scale group is
-// never split across active and inactive lanes.
-template <int K, bool kExport, bool kShift>
-__device__ __forceinline__ void bwd_load_global(const EwParams& P, int64_t qi, bool active,
-                                                float (&l)[K][4], float (&m)[K][4], float4& gv,
-                                                float (&w)[4], float& s, float& ms, uint32_t& j4) {
-  const int64_t qc = active ? qi : 0;
-  const int64_t gidx = (qc * 4) >> P.log2_group;
-#pragma unroll
-  for (int k = 0; k < K; ++k) {
-    const float4 v = __ldcs(reinterpret_cast<const float4*>(P.logits + k * P.n) + qc);
-    l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
-  }
-  if (!kExport) {
-#pragma unroll
-    for (int k = 0; k < K; ++k) {
-      const float4 v = __ldcs(reinterpret_cast<const float4*>(P.m_logits + k * P.n) + qc);
-      m[k][0] = v.x; m[k][1] = v.y; m[k][2] = v.z; m[k][3] = v.w;
-    }
-  }
-  gv = __ldcs(reinterpret_cast<const float4*>(P.G) + qc);
-  if (!active) gv = make_float4(0.f, 0.f, 0.f, 0.f);
-  load_w4(P.W, qc, P.w_bf16, w);
-  s = __ldg(P.scales + gidx);
-  ms = 0.0f;
-  if (!kExport && !P.scales_frozen) ms = __ldg(P.m_scales + gidx);
-  j4 = kShift ? load_j0(P, qc) : 0u;
-}
-
-template <class Rx, bool kExport, bool kShift, bool kAcc>
-__global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(const EwParams P) {
-  constexpr int K = Rx::L;
-  float q[kMaxLevels];
-  load_grid(P, q);
-  __shared__ float sgrid[kMaxLevels];
-  if (kShift) fill_shared_grid(P, sgrid);
-  const int lane = threadIdx.x & 31;
-  const int seg = P.group >> 2;  // lanes per scale group
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  float2 loss2 = f2(0.0f);
-
-  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
-       base < P.nq; base += stride) {
-    const int64_t qi = base + lane;
-    const bool active = qi < P.nq;
-    float l[K][4], m[K][4], w[4];
-    float4 gv;
-    float s, ms;
-    uint32_t j4;
-    bwd_load_global<K, kExport, kShift>(P, qi, active, l, m, gv, w, s, ms, j4);
-    bwd_quad<Rx, kExport, kShift, kAcc>(P, q, sgrid, lane, seg, qi, active, l, m, gv, w, s, ms,
-                                        j4, loss2);
-  }
-  reduce_loss(loss2.x + loss2.y, P);
-}
-
-// ---------------------------------------------------------------------------
-// TMA-staged fused backward (non-export, non-accumulating steps): the per-quad
-// body of k_backward, with the streams a block reads (logits, their momenta,
-// G, W, scales, scale momenta, j0) brought into shared memory by bulk
-// asynchronous copies (cp.async.bulk, completion counted on an mbarrier) a tile
-// ahead, so the warps read them with shared-memory loads instead of stalling
-// on HBM.  A tile is 256 quads (1,024 weights, one quad per thread); tiles go
-// to blocks round-robin (tile = blockIdx.x + j * gridDim.x) through two stages.
-// The last warp to finish reading a stage (a shared counter) issues the copies
-// of the block's tile two ahead into it, so no warp waits for another.  A
-// partial last tile is read with direct loads by the block whose turn it is.
-// Logit momenta are staged for L <= 5 logits, where two stages of two resident
-// blocks fit in shared memory; otherwise they are loaded directly at the top of
-// the iteration and arrive while the noise is drawn.  Stores stay direct.
-// Every wait is bounded (2 s of %globaltimer); on expiry the block records an
-// error code, waits (bounded) for its own copies in flight and returns.
-// ---------------------------------------------------------------------------
-constexpr int kTileQ = kEwThreads;                 // quads per tile
-constexpr int64_t kTileW = 4 * kTileQ;             // weights per tile
-constexpr uint32_t kPlaneBytes = 4u * kTileW;      // one fp32 plane of a tile
-
-// A staging plan: blocks per SM the registers are budgeted for, and which of the
-// per-weight streams besides the logits go through shared memory (logit
-// momenta; G and W).  Streams not staged are loaded directly at the top of the
-// iteration.  Two stages of every resident block must fit in shared memory.
-template <int kOcc_, bool kStageM_, bool kStageGW_>
-struct StagePlan {
-  static constexpr int kOcc = kOcc_;
-  static constexpr bool kStageM = kStageM_;
-  static constexpr bool kStageGW = kStageGW_;
-};
-
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-
-// Copies of tile `tile` into stage `st`; the byte count the mbarrier expects
-// is S.tx (the sum of the copies below).
-template <int L, bool kShift, bool kStageM, bool kStageGW>
-__device__ __forceinline__ void stage_issue(const EwParams& P, const BwdStage& S, unsigned char* st,
-                                            uint64_t* bar, int64_t tile) {
-  const int64_t w0 = tile * kTileW;
-  mbar_expect_tx(bar, S.tx);
-#pragma unroll
-  for (int k = 0; k < L; ++k) bulk_g2s(st + S.l + k * kPlaneBytes, P.logits + k * P.n + w0, kPlaneBytes, bar);
-  if (kStageM) {
-#pragma unroll
-    for (int k = 0; k < L; ++k)
-      bulk_g2s(st + S.m + k * kPlaneBytes, P.m_logits + k * P.n + w0, kPlaneBytes, bar);
-  }
-  if (kStageGW) {
-    bulk_g2s(st + S.g, P.G + w0, kPlaneBytes, bar);
-    const int wb = P.w_bf16 ? 2 : 4;
-    bulk_g2s(st + S.w, static_cast<const unsigned char*>(P.W) + w0 * wb,
-             static_cast<uint32_t>(kTileW * wb), bar);
-  }
-  const uint32_t sb = kPlaneBytes >> P.log2_group;  // one fp32 per scale group
-  bulk_g2s(st + S.s, P.scales + (w0 >> P.log2_group), sb, bar);
-  if (!P.scales_frozen) bulk_g2s(st + S.ms, P.m_scales + (w0 >> P.log2_group), sb, bar);
-  if (kShift) bulk_g2s(st + S.j, P.j0 + w0, static_cast<uint32_t>(kTileW), bar);
-}
-
-template <class Rx, bool kShift, class Plan>
-__global__ void __launch_bounds__(kEwThreads, Plan::kOcc)
-    k_backward_staged(const EwParams P, const BwdStage S) {
-  constexpr int K = Rx::L;
-  constexpr bool kStageM = Plan::kStageM;
-  constexpr bool kStageGW = Plan::kStageGW;
-  constexpr unsigned int kWarps = kEwThreads / 32;
-  extern __shared__ __align__(128) unsigned char stage_mem[];
-  __shared__ __align__(8) uint64_t full[2];
-  __shared__ unsigned int done[2], issued[2];
-  __shared__ int abort_flag;
-  __shared__ float sgrid[kMaxLevels];
-  float q[kMaxLevels];
-  load_grid(P, q);
-  const int tid = threadIdx.x, lane = tid & 31;
-  const int seg = P.group >> 2;  // lanes per scale group
-  const int64_t ntiles = P.nq / kTileQ;  // full tiles
-  const int64_t first = blockIdx.x, stride = gridDim.x;
-  volatile int* abort_v = &abort_flag;
-  if (tid == 0) {
-    mbar_init(&full[0], 1);
-    mbar_init(&full[1], 1);
-    done[0] = done[1] = 0u;
-    issued[0] = issued[1] = 0u;
-    abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (kShift && tid < kMaxLevels) sgrid[tid] = P.grid[tid];
-  __syncthreads();
-  if (tid == 0) {
-#pragma unroll
-    for (int b = 0; b < 2; ++b) {
-      if (first + b * stride < ntiles && !(P.stall && b == 1)) {
-        stage_issue<K, kShift, kStageM, kStageGW>(P, S, stage_mem + b * S.bytes, &full[b], first + b * stride);
-        issued[b] = 1u;
-      }
-    }
-  }
-  float2 loss2 = f2(0.0f);
-  int64_t j = 0;
-  for (int64_t tile = first; tile < ntiles; tile += stride, ++j) {
-    const int b = static_cast<int>(j & 1);
-    const uint32_t parity = static_cast<uint32_t>((j >> 1) & 1);
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[b], parity, abort_v) ? 1 : 0);
-    if (!ok) break;
-    const unsigned char* st = stage_mem + b * S.bytes;
-    const int64_t qi = tile * kTileQ + tid;
-    float l[K][4], m[K][4], w[4];
-#pragma unroll
-    for (int k = 0; k < K; ++k) {
-      const float4 v = reinterpret_cast<const float4*>(st + S.l + k * kPlaneBytes)[tid];
-      l[k][0] = v.x; l[k][1] = v.y; l[k][2] = v.z; l[k][3] = v.w;
-    }
-#pragma unroll
-    for (int k = 0; k < K; ++k) {
-      const float4 v = kStageM ? reinterpret_cast<const float4*>(st + S.m + k * kPlaneBytes)[tid]
-                               : __ldcs(reinterpret_cast<const float4*>(P.m_logits + k * P.n) + qi);
-      m[k][0] = v.x; m[k][1] = v.y; m[k][2] = v.z; m[k][3] = v.w;
-    }
-    float4 gv;
-    if (!kStageGW) {
-      gv = __ldcs(reinterpret_cast<const float4*>(P.G) + qi);
-      load_w4(P.W, qi, P.w_bf16, w);
-    } else {
-      gv = reinterpret_cast<const float4*>(st + S.g)[tid];
-      if (P.w_bf16) {
-        const uint2 raw = reinterpret_cast<const uint2*>(st + S.w)[tid];
-        const float2 fa = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
-        const float2 fb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
-        w[0] = fa.x; w[1] = fa.y; w[2] = fb.x; w[3] = fb.y;
-      } else {
-        const float4 v = reinterpret_cast<const float4*>(st + S.w)[tid];
-        w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
-      }
-    }
-    const int gl = (tid * 4) >> P.log2_group;  // scale group within the tile
-    const float s = reinterpret_cast<const float*>(st + S.s)[gl];
-    const float ms = P.scales_frozen ? 0.0f : reinterpret_cast<const float*>(st + S.ms)[gl];
-    const uint32_t j4 = kShift ? reinterpret_cast<const uint32_t*>(st + S.j)[tid] : 0u;
-    // Release the stage: the warp that completes the count refills it with this
-    // block's tile two ahead (generic reads ordered before the async-proxy writes).
-    __syncwarp();
-    if (lane == 0) {
-      __threadfence_block();
-      const unsigned int prev = atomicAdd(&done[b], 1u);
-      if ((prev + 1u) % kWarps == 0u) {
-        const int64_t nxt = tile + 2 * stride;
-        if (nxt < ntiles) {
-          __threadfence_block();
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          stage_issue<K, kShift, kStageM, kStageGW>(P, S, stage_mem + b * S.bytes, &full[b], nxt);
-          issued[b] += 1u;
-        }
-      }
-    }
-    bwd_quad<Rx, false, kShift, false>(P, q, sgrid, lane, seg, qi, true, l, m, gv, w, s, ms, j4,
-                                       loss2);
-  }
-  __syncthreads();
-  if (*abort_v) {
-    // wait (bounded, ignoring the abort flag) for the copies still in flight into
-    // this block's stages before the block leaves
-    if (tid == 0) {
-#pragma unroll
-      for (int b = 0; b < 2; ++b)
-        if (issued[b]) mbar_wait(&full[b], (issued[b] - 1u) & 1u, abort_v, false);
-    }
-  } else if (ntiles * kTileQ < P.nq && first == ntiles % stride) {
-    // the partial last tile, with direct loads
-    const int64_t qi = ntiles * kTileQ + tid;
-    const bool active = qi < P.nq;
-    float l[K][4], m[K][4], w[4];
-    float4 gv;
-    float s, ms;
-    uint32_t j4;
-    bwd_load_global<K, false, kShift>(P, qi, active, l, m, gv, w, s, ms, j4);
-    bwd_quad<Rx, false, kShift, false>(P, q, sgrid, lane, seg, qi, active, l, m, gv, w, s, ms, j4,
-                                       loss2);
-  }
-  reduce_loss(loss2.x + loss2.y, P);
-  if (tid == 0 && *abort_v) atomicExch(&P.flags->error, 0x7C03u);
 }
 
 // ---------------------------------------------------------------------------
@@ -958,13 +534,8 @@ __global__ void __launch_bounds__(kEwThreads) k_diagnose(const DiagParams P) {
 }
 
 template <class Rx, bool kShift>
-void set_max_smem_carveout() {
-  const auto attr = cudaFuncAttributePreferredSharedMemoryCarveout;
-  cudaFuncSetAttribute(k_forward<Rx, kShift>, attr, 0);
-  cudaFuncSetAttribute(k_backward<Rx, false, kShift, false>, attr, 0);
-  cudaFuncSetAttribute(k_backward<Rx, true, kShift, false>, attr, 0);
-  cudaFuncSetAttribute(k_backward<Rx, false, kShift, true>, attr, 0);
-  cudaFuncSetAttribute(k_backward<Rx, true, kShift, true>, attr, 0);
+void set_forward_carveout() {
+  cudaFuncSetAttribute(k_forward<Rx, kShift>, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
 }
 
 int grid_for(const void* fn, int num_sms, int threads) {
@@ -979,14 +550,13 @@ int grid_for(const void* fn, int num_sms, int threads) {
 
 
 int ew_grid_size(int K, int which, int num_sms, int mode) {
+  if (which != 0) return ew_backward_grid(K, num_sms, mode);
   int g = num_sms;
   with_relax(K, mode, [&](auto rx, auto sh) {
     using Rx = typename decltype(rx)::type;
     constexpr bool SH = decltype(sh)::value;
-    set_max_smem_carveout<Rx, SH>();
-    g = which == 0 ? grid_for(reinterpret_cast<const void*>(k_forward<Rx, SH>), num_sms, kEwThreads)
-                   : grid_for(reinterpret_cast<const void*>(k_backward<Rx, false, SH, false>), num_sms,
-                              kEwThreads);
+    set_forward_carveout<Rx, SH>();
+    g = grid_for(reinterpret_cast<const void*>(k_forward<Rx, SH>), num_sms, kEwThreads);
   });
   return g;
 }
@@ -997,143 +567,6 @@ cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s) {
     k_forward<Rx, decltype(sh)::value><<<grid, kEwThreads, 0, s>>>(p);
   });
   return e != cudaSuccess ? e : cudaGetLastError();
-}
-
-cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
-  const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
-  const bool acc = p.acc_in_l != nullptr;
-  const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
-    using Rx = typename decltype(rx)::type;
-    constexpr bool SH = decltype(sh)::value;
-    if (export_mode)
-      acc ? k_backward<Rx, true, SH, true><<<grid, kEwThreads, 0, s>>>(p)
-          : k_backward<Rx, true, SH, false><<<grid, kEwThreads, 0, s>>>(p);
-    else
-      acc ? k_backward<Rx, false, SH, true><<<grid, kEwThreads, 0, s>>>(p)
-          : k_backward<Rx, false, SH, false><<<grid, kEwThreads, 0, s>>>(p);
-  });
-  return e != cudaSuccess ? e : cudaGetLastError();
-}
-
-namespace {
-
-BwdStage stage_layout(int L, bool stage_m, bool stage_gw, int w_bf16, int log2_group,
-                      int scales_frozen, int shift) {
-  auto up = [](uint32_t x) { return (x + 127u) & ~127u; };
-  BwdStage S{};
-  const uint32_t sb = kPlaneBytes >> log2_group;
-  const uint32_t wbytes = static_cast<uint32_t>(kTileW) * (w_bf16 ? 2u : 4u);
-  uint32_t off = 0, tx = 0;
-  S.l = off; off += L * kPlaneBytes; tx += L * kPlaneBytes;
-  S.m = off;
-  if (stage_m) { off += L * kPlaneBytes; tx += L * kPlaneBytes; }
-  S.g = off;
-  if (stage_gw) { off += kPlaneBytes; tx += kPlaneBytes; }
-  S.w = off;
-  if (stage_gw) { off += up(wbytes); tx += wbytes; }
-  S.s = off; off += up(sb); tx += sb;
-  S.ms = off;
-  if (!scales_frozen) { off += up(sb); tx += sb; }
-  S.j = off;
-  if (shift) { off += static_cast<uint32_t>(kTileW); tx += static_cast<uint32_t>(kTileW); }
-  S.bytes = (off + 1023u) & ~1023u;
-  S.tx = tx;
-  return S;
-}
-
-// Staging plans (the plan id is kept by the layer), measured on GB300 against
-// each other and against the direct-load kernel:
-//   1: 2 blocks/SM, every stream staged (tuning alternative);
-//   3: 3 blocks/SM (80 registers, up to 4 logits per weight), logits, G, W and
-//      scales staged, logit momenta loaded directly: fastest up to 4 logits;
-//   5: 2 blocks/SM, as 3 with the register budget of 2 blocks: fastest from 6
-//      logits up.
-// With 5 logits (local shift) the direct-load kernel was faster than every
-// plan, so none is chosen there.
-using Plan1 = StagePlan<2, true, true>;
-using Plan3 = StagePlan<3, false, true>;
-using Plan5 = StagePlan<2, false, true>;
-
-int default_plan(int L) { return L <= 4 ? 3 : (L == 5 ? 0 : 5); }
-
-template <int L, class F>
-void with_plan(int plan, F&& f) {
-  switch (plan) {
-    case 1: f(Plan1{}); break;
-    case 3: if constexpr (L <= 4) f(Plan3{}); break;
-    case 5: f(Plan5{}); break;
-    default: break;
-  }
-}
-
-template <class Rx, bool kShift, class Plan>
-int staged_grid_for(const BwdStage& S, int num_sms) {
-  auto* fn = k_backward_staged<Rx, kShift, Plan>;
-  const int dyn = 2 * static_cast<int>(S.bytes);
-  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn) != cudaSuccess ||
-      cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, 100) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reinterpret_cast<const void*>(fn),
-                                                    kEwThreads, dyn) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  // only where the blocks the plan budgets its registers for are resident
-  return per_sm >= Plan::kOcc ? per_sm * num_sms : 0;
-}
-
-}  // namespace
-
-int ew_staged_grid(int K, int mode, int w_bf16, int log2_group, int scales_frozen, int num_sms,
-                   int* plan_out) {
-  *plan_out = 0;
-  if (log2_group < 2 || log2_group > 7) return 0;
-  int g = 0;
-  with_relax(K, mode, [&](auto rx, auto sh) {
-    using Rx = typename decltype(rx)::type;
-    constexpr bool SH = decltype(sh)::value;
-    int plan = default_plan(Rx::L);
-    if (const char* e = std::getenv("GSQ_STAGED_PLAN")) {  // tuning override: 1, 3 or 5
-      const int v = std::atoi(e);
-      if (v == 1 || v == 3 || v == 5) plan = v;
-    }
-    with_plan<Rx::L>(plan, [&](auto pl) {
-      using Plan = decltype(pl);
-      const BwdStage S = stage_layout(Rx::L, Plan::kStageM, Plan::kStageGW, w_bf16, log2_group,
-                                      scales_frozen, SH ? 1 : 0);
-      g = staged_grid_for<Rx, SH, Plan>(S, num_sms);
-      if (g > 0) *plan_out = plan;
-    });
-  });
-  return g;
-}
-
-cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s) {
-  if (p.grad_logits || p.grad_scales || p.acc_in_l || p.acc_in_s) return cudaErrorInvalidValue;
-  if (p.log2_group < 2 || p.log2_group > 7) return cudaErrorInvalidValue;
-  // bulk copies need 16-byte aligned sources (tile offsets are multiples of 16 B)
-  auto a16 = [](const void* x) { return (reinterpret_cast<uintptr_t>(x) & 15u) == 0; };
-  if (!a16(p.logits) || !a16(p.m_logits) || !a16(p.G) || !a16(p.W) || !a16(p.scales) ||
-      !a16(p.m_scales) || (p.j0 && !a16(p.j0)) || ((p.n * 4) & 15))
-    return cudaErrorInvalidValue;
-  bool launched = false;
-  const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
-    using Rx = typename decltype(rx)::type;
-    constexpr bool SH = decltype(sh)::value;
-    with_plan<Rx::L>(plan, [&](auto pl) {
-      using Plan = decltype(pl);
-      const BwdStage S = stage_layout(Rx::L, Plan::kStageM, Plan::kStageGW, p.w_bf16, p.log2_group,
-                                      p.scales_frozen, SH ? 1 : 0);
-      k_backward_staged<Rx, SH, Plan><<<grid, kEwThreads, 2 * S.bytes, s>>>(p, S);
-      launched = true;
-    });
-  });
-  if (e != cudaSuccess) return e;
-  if (!launched) return cudaErrorInvalidValue;
-  return cudaGetLastError();
 }
 
 cudaError_t launch_init_state(const InitParams& p, int num_sms, cudaStream_t s) {

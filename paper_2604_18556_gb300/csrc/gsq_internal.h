@@ -88,7 +88,7 @@ struct BwdStage {
 // Records `msg` as this thread's gsq_last_error() text and returns `st` (gsq_api.cu).
 gsq_status set_last_error(gsq_status st, const char* msg);
 
-// ---- launchers (gsq_elementwise.cu) ----------------------------------------
+// ---- launchers (gsq_elementwise.cu; backward: gsq_backward.cu, gsq_staged.cu) --
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
 cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
 // TMA-staged backward for non-export, non-accumulating steps: its grid for a
@@ -98,6 +98,7 @@ int ew_staged_grid(int K, int mode, int w_bf16, int log2_group, int scales_froze
                    int* plan);
 cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s);
 int ew_grid_size(int K, int which, int num_sms, int mode);  // which: 0 forward, 1 backward
+int ew_backward_grid(int K, int num_sms, int mode);          // gsq_backward.cu
 
 struct InitParams {
   int64_t n;

@@ -59,6 +59,24 @@ bool encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Output of the CTA-pair GEMM as a 3D map [E][M][N] (fp32 or bf16) for TMA
+// stores of 32 x 32 boxes, swizzled 128 B (fp32 rows) or 64 B (bf16 rows).
+static bool encode_out_map(CUtensorMap* map, void* base, int E, int M, int N, int bf16) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  const uint64_t es = bf16 ? 2 : 4;
+  const cuuint64_t dims[3] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(M),
+                              static_cast<cuuint64_t>(E)};
+  const cuuint64_t strides[2] = {static_cast<cuuint64_t>(N) * es,
+                                 static_cast<cuuint64_t>(M) * N * es};
+  const cuuint32_t box[3] = {32u, 32u, 1u};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base,
+            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            bf16 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 namespace {
 
 constexpr int TC_BM = 128, TC_BK = 64;
@@ -303,14 +321,19 @@ struct Tc2Cfg {
   static constexpr int kBHalf = BN / 2;
   static constexpr int kBBytes = kBHalf * TC_BK * 2;
   static constexpr int kStageBytes = TC_A_BYTES + kBBytes;
+  // epilogue staging: two 32 x 32 fp32 chunks per epilogue warp (4 warps)
+  static constexpr int kEpiChunk = 32 * 32 * 4;
+  static constexpr int kEpiBytes = 4 * 2 * kEpiChunk;
   static constexpr int kStages =
-      ((232448 - 2048) / kStageBytes) < 8 ? ((232448 - 2048) / kStageBytes) : 8;
+      ((232448 - 2048 - kEpiBytes) / kStageBytes) < 8 ? ((232448 - 2048 - kEpiBytes) / kStageBytes)
+                                                       : 8;
   static constexpr int kTmemCols = 2 * BN <= 256 ? 256 : 512;
   static constexpr int kAccStride = kTmemCols / 2;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 256 + 1024;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kEpiBytes + 256 + 1024;
   static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
                                      (static_cast<uint32_t>(BN >> 3) << 17) |
                                      (static_cast<uint32_t>(TC2_BM >> 4) << 24);
+  static_assert(BN % 32 == 0, "the epilogue stores 32-column chunks");
   static_assert(kBHalf % 8 == 0, "B half must be whole 8-row swizzle atoms");
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1 KiB alignment");
 };
@@ -318,14 +341,15 @@ struct Tc2Cfg {
 template <int BN>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     k_tc_gemm_pair(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const TcArgs args) {
+                   const __grid_constant__ CUtensorMap tmO, const TcArgs args) {
   using Cfg = Tc2Cfg<BN>;
   constexpr int STAGES = Cfg::kStages;
   constexpr int STAGE_BYTES = Cfg::kStageBytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint8_t* epi = smem + STAGES * STAGE_BYTES;  // epilogue staging (1 KiB aligned)
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(epi + Cfg::kEpiBytes);
   uint64_t* empty_bar = full_bar + STAGES;
   uint64_t* tfull_bar = empty_bar + STAGES;
   uint64_t* tempty_bar = tfull_bar + 2;
@@ -347,6 +371,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmO)) : "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -442,44 +467,67 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
   } else {
     // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
+    // Each warp drains its 32 TMEM lanes (rows) 32 columns at a time into one of
+    // two 32 x 32 staging chunks and writes the chunk with one TMA tensor store
+    // (whole-line writes).  The store map is 3D [E][M][N], so rows past M of an
+    // expert and columns past N are not written.  Staging layout = the map's
+    // swizzle (128 B for fp32 rows, 64 B for bf16 rows): 16-byte piece p of row r
+    // sits at piece p ^ (r % 8) (fp32) or p ^ ((r / 2) % 4) (bf16), so the 32
+    // lanes' writes of one piece spread over all banks.
     const int quarter = warp & 3;
+    uint8_t* wbuf = epi + quarter * 2 * Cfg::kEpiChunk;
     int acc = 0;
     uint32_t acc_phase = 0;
+    int chunks = 0;  // chunks this warp has stored; buffer = chunks & 1
     for (int tile = pair; tile < tiles; tile += npairs) {
       if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
       tc_fence_after();
       int e, m, n;
       tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
-      const int row = m * TC2_BM + static_cast<int>(rank) * TC_BM + quarter * 32 + lane;
+      const int row0 = m * TC2_BM + static_cast<int>(rank) * TC_BM + quarter * 32;
       const int col0 = n * BN;
-      const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
       const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride) +
                              (static_cast<uint32_t>(quarter * 32) << 16);
-      // 32 columns per TMEM load and wait (BN is a multiple of 32)
 #pragma unroll 1
       for (int c = 0; c < BN; c += 32) {
         float v[32];
         tmem_ld32(taddr + c, v);
-        if (row < args.M) {
-#pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            const int col = col0 + c + j;
-            if (col < args.N) {
-              const float4 o = make_float4(args.alpha * v[j], args.alpha * v[j + 1],
-                                           args.alpha * v[j + 2], args.alpha * v[j + 3]);
-              if (args.out_bf16) {
-                const __nv_bfloat162 lo = __floats2bfloat162_rn(o.x, o.y);
-                const __nv_bfloat162 hi = __floats2bfloat162_rn(o.z, o.w);
-                uint2 raw;
-                raw.x = *reinterpret_cast<const uint32_t*>(&lo);
-                raw.y = *reinterpret_cast<const uint32_t*>(&hi);
-                *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(args.out) + obase + col) = raw;
-              } else {
-                *reinterpret_cast<float4*>(static_cast<float*>(args.out) + obase + col) = o;
-              }
-            }
-          }
+        if (row0 >= args.M || col0 + c >= args.N) continue;  // nothing of this chunk is stored
+        uint8_t* buf = wbuf + (chunks & 1) * Cfg::kEpiChunk;
+        if (chunks >= 2) {  // the store that last read this buffer has finished reading it
+          if (lane == 0) bulk_wait_read_1();
+          __syncwarp();
         }
+        if (args.out_bf16) {
+          uint8_t* rowp = buf + lane * 64;
+          const int sw = (lane >> 1) & 3;
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            uint32_t w[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const __nv_bfloat162 b2 = __floats2bfloat162_rn(args.alpha * v[8 * p + 2 * h],
+                                                              args.alpha * v[8 * p + 2 * h + 1]);
+              w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+            }
+            *reinterpret_cast<uint4*>(rowp + 16 * (p ^ sw)) = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        } else {
+          uint8_t* rowp = buf + lane * 128;
+          const int sw = lane & 7;
+#pragma unroll
+          for (int p = 0; p < 8; ++p)
+            *reinterpret_cast<float4*>(rowp + 16 * (p ^ sw)) =
+                make_float4(args.alpha * v[4 * p], args.alpha * v[4 * p + 1],
+                            args.alpha * v[4 * p + 2], args.alpha * v[4 * p + 3]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tmO, buf, col0 + c, row0, e);
+          bulk_commit();
+        }
+        ++chunks;
       }
       tc_fence_before();
       __syncwarp();
@@ -489,6 +537,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         acc_phase ^= 1u;
       }
     }
+    if (lane == 0) bulk_wait_all();  // every store complete before the CTA leaves
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -558,12 +608,15 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, to;
   if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;
+  if (g.out_bf16 && g.N % 8 != 0) return cudaErrorInvalidValue;  // 16-byte row pitch of the store map
+  if ((reinterpret_cast<uintptr_t>(g.out) & 15) != 0) return cudaErrorInvalidValue;
   if (!encode_kmajor_bf16(&ta, g.A, static_cast<uint64_t>(g.K),
                           static_cast<uint64_t>(g.E) * g.M, TC_BM) ||
       !encode_kmajor_bf16(&tb, g.B, static_cast<uint64_t>(g.K),
-                          static_cast<uint64_t>(g.E) * g.N, Cfg::kBHalf))
+                          static_cast<uint64_t>(g.E) * g.N, Cfg::kBHalf) ||
+      !encode_out_map(&to, g.out, g.E, g.M, g.N, g.out_bf16))
     return cudaErrorInvalidValue;
   TcArgs a;
   a.E = g.E;
@@ -600,7 +653,7 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   if (max_clusters < pairs) pairs = max_clusters;
   if (tiles < pairs) pairs = static_cast<int>(tiles);
   cfg.gridDim = dim3(2 * pairs, 1, 1);
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_pair<BN>, ta, tb, a);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_pair<BN>, ta, tb, to, a);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 

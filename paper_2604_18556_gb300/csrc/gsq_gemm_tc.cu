@@ -305,11 +305,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 // CTA-pair variant: a cluster of two CTAs on neighbouring SMs computes a
 // 256 x BN output tile with tcgen05.mma.cta_group::2.  Each CTA stages its own
 // 128 rows of A and its half (BN/2 rows) of B, so a stage is 16 KiB + BN KiB/8
-// (30 KiB at BN = 224, 7 stages) and every SM streams a third less operand
-// data than a single CTA with the same tile width.  Both CTAs' copies complete
-// on the leader's (rank 0) full barrier; the leader's single MMA thread issues
-// for the pair and its commits arrive on the empty / accumulator barriers of
-// both CTAs.  Each CTA's epilogue drains its own TMEM (its 128 rows) and
+// (30 KiB at BN = 224, 6 stages beside 32 KiB of epilogue staging) and every
+// SM streams a third less operand data than a single CTA with the same tile
+// width.  Both CTAs' copies complete on the leader's (rank 0) full barrier; the
+// leader's single MMA thread issues for the pair and its commits arrive on the
+// empty / accumulator barriers of both CTAs.  Each CTA's epilogue drains its
+// own TMEM (its 128 rows) through shared memory into TMA tensor stores and
 // arrives on the leader's accumulator-empty barrier.  Waits are bounded as in
 // k_tc_gemm; a CTA that gives up records the error, lets its copies in flight
 // land (a bounded pause) and meets its peer at the final cluster barrier.
@@ -663,7 +664,7 @@ bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
 
 int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair) {
   if (pair) {
-    // CTA pairs (256-row tiles over two SMs, 7-stage rings at both widths): 256-wide
+    // CTA pairs (256-row tiles over two SMs, 6-stage rings at both widths): 256-wide
     // tiles unless they take more waves x width than 224-wide ones.  Measured on
     // GB300: 4096 x 14336 886 vs 955 us, 28672 x 8192 2.11 vs 2.21 ms, 64 experts
     // 2048 x 7168 7.27 vs 7.69 ms; on 4096 x 4096, 224 wide (4 full waves) wins.

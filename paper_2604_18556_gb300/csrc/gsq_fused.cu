@@ -437,13 +437,10 @@ __global__ void __launch_bounds__(FZ_THREADS, 1)
 template <class Rx, bool kShift>
 cudaError_t launch_fused_impl(const CUtensorMap& tmH, const CUtensorMap& tmD, const FusedArgs& a,
                               int grid, cudaStream_t s) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    const cudaError_t e = cudaFuncSetAttribute(
-        k_step_fused<Rx, kShift>, cudaFuncAttributeMaxDynamicSharedMemorySize, FZ_SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  // set on every launch: the attribute belongs to the current device
+  const cudaError_t e = cudaFuncSetAttribute(
+      k_step_fused<Rx, kShift>, cudaFuncAttributeMaxDynamicSharedMemorySize, FZ_SMEM_BYTES);
+  if (e != cudaSuccess) return e;
   k_step_fused<Rx, kShift><<<grid, FZ_THREADS, FZ_SMEM_BYTES, s>>>(tmH, tmD, a);
   return cudaGetLastError();
 }

@@ -567,13 +567,10 @@ double wave_balance(int64_t tiles, int num_sms) {
 
 template <int BN>
 cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         TcCfg<BN>::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  // set on every launch: the attribute belongs to the current device
+  cudaError_t ea = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        TcCfg<BN>::kSmemBytes);
+  if (ea != cudaSuccess) return ea;
   CUtensorMap ta, tb;
   if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;  // 16-B rows; 8/16-B stores
   if (!encode_kmajor_bf16(&ta, g.A, static_cast<uint64_t>(g.K),
@@ -602,13 +599,10 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
 template <int BN>
 cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   using Cfg = Tc2Cfg<BN>;
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm_pair<BN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  // set on every launch: the attribute belongs to the current device
+  cudaError_t ea = cudaFuncSetAttribute(k_tc_gemm_pair<BN>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  if (ea != cudaSuccess) return ea;
   CUtensorMap ta, tb, to;
   if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;
   if (g.out_bf16 && g.N % 8 != 0) return cudaErrorInvalidValue;  // 16-byte row pitch of the store map

@@ -125,6 +125,8 @@ def test_workspace_size_formula(lib):
     (dict(grid=tuple(range(9))), 1),             # K > 8
     (dict(grid=(0.0, 0.0 + 1e-30)), 1),          # no level of usable magnitude? ascending but tiny ok
     (dict(rows=0), 2),
+    (dict(cols=0), 2),                           # empty layers
+    (dict(experts=0), 2),
     (dict(scale_mode=1, group_size=16), 1),      # KQUANT2 needs frozen scales
     (dict(scale_mode=1, group_size=16, lr_scales=0.0, cols=128), 2),   # C % 256
     (dict(w_dtype=7), 1),
@@ -149,6 +151,21 @@ def test_descriptor_validation(lib, kw, status):
         lib.gsq_workspace_size(d)
     assert ei.value.status == status
     assert lib.gsq_last_error()
+
+
+def test_flags_known_and_unknown(lib):
+    """Every documented flag bit is accepted (the unstaged-backward bit among them);
+    an unknown bit is an argument error."""
+    for f in (lib.GSQ_FLAG_NO_NOISE, lib.GSQ_FLAG_KEEP_G | lib.GSQ_FLAG_FUSED,
+              lib.GSQ_FLAG_UNSTAGED):
+        d = _desc(lib)
+        d.flags = f
+        assert lib.gsq_workspace_size(d) > 0
+    d = _desc(lib)
+    d.flags = 16
+    with pytest.raises(lib.GsqError) as ei:
+        lib.gsq_workspace_size(d)
+    assert ei.value.status == 1 and "flags" in lib.gsq_last_error()
 
 
 def test_parameterisations_size_their_logit_planes(lib):

@@ -45,8 +45,6 @@ def _args():
     ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
     ap.add_argument("--unstaged", action="store_true",
                     help="time the backward with direct global loads (GSQ_FLAG_UNSTAGED)")
-    ap.add_argument("--fused", action="store_true",
-                    help="time the fused step kernel (GSQ_FLAG_FUSED) instead of GEMM + backward")
     return ap.parse_args()
 
 
@@ -63,7 +61,6 @@ CSRC = os.path.join(ROOT, "paper_2604_18556_gb300", "csrc")
 KERNEL_SOURCES = {
     "k_backward": ["gsq_backward.cu", "gsq_staged.cu", "gsq_backward.cuh", "gsq_relax.cuh",
                    "gsq_tc.cuh", "gsq_internal.h"],
-    "k_step_fused": ["gsq_fused.cu", "gsq_relax.cuh", "gsq_tc.cuh"],
 }
 
 
@@ -361,7 +358,7 @@ def gpu_arm(args, rank, world, local):
                       init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
                       lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
                       wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param,
-                      fused=args.fused, unstaged=args.unstaged)
+                      unstaged=args.unstaged)
     stream = torch.cuda.current_stream()
     loss = torch.zeros(1, device="cuda")
     T = w.steps
@@ -428,45 +425,26 @@ def gpu_arm(args, rank, world, local):
     bwd_n, bwd_ms = prof["backward"]
     gemm_n, gemm_ms = prof["gemm"]
     fwd_n, fwd_ms = prof["forward"]
-    step_n, step_ms = prof["step"]
     flops = w.gemm_flops_per_step()
-    if step_n > 0:
-        # one fused kernel per step: the contraction on the tensor cores with the
-        # backward, Lion and next forward as its epilogue (G never leaves the SM)
-        avg = step_ms / step_n
-        nbytes = w.fused_step_bytes()
-        gbs = nbytes / (avg * 1e-3) / 1e9
-        tfs = flops / (avg * 1e-3) / 1e12
-        roofline = {"kernel": "k_step_fused (tcgen05 contraction + backward + Lion + next forward)",
-                    "bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
-                    "traffic": committed_traffic(w.name, "k_step_fused"),
-                    "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
-                    "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": avg,
-                    "frac_of_8TBps": gbs / 8000.0}
-        roofline_gemm = {"kernel": "k_step_fused contraction (its flops over the fused kernel's time)",
-                         "bound": "tensor", "achieved": tfs, "peak": tf_sust, "unit": "TFLOP/s",
-                         "frac": tfs / tf_sust, "flops_per_launch": flops, "avg_launch_ms": avg,
-                         "peak_source": f"{peak_src} bf16_tflops_sustained"}
-    else:
-        bwd_avg = bwd_ms / max(bwd_n, 1)
-        gemm_avg = gemm_ms / max(gemm_n, 1)
-        bytes_bwd = w.elementwise_bytes_per_weight() * n
-        bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
-        gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
-        kname = layer.kernel_name(gsq.GSQ_K_BACKWARD)
-        roofline = {"kernel": f"{kname} (fused backward + Lion + next forward)", "bound": "hbm",
-                    "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
-                    "traffic": committed_traffic(w.name),
-                    "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
-                    "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
-                    "frac_of_8TBps": bwd_gbs / 8000.0}
-        roofline_gemm = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} (tcgen05 loss contraction)",
-                         "bound": "tensor",
-                         "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
-                         "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
-                         "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
-                         "peak_source": f"{peak_src} bf16_tflops_sustained"}
-    launches = bwd_n + gemm_n + fwd_n + step_n
+    bwd_avg = bwd_ms / max(bwd_n, 1)
+    gemm_avg = gemm_ms / max(gemm_n, 1)
+    bytes_bwd = w.elementwise_bytes_per_weight() * n
+    bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
+    gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
+    kname = layer.kernel_name(gsq.GSQ_K_BACKWARD)
+    roofline = {"kernel": f"{kname} (fused backward + Lion + next forward)", "bound": "hbm",
+                "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
+                "traffic": committed_traffic(w.name),
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
+                "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
+                "frac_of_8TBps": bwd_gbs / 8000.0}
+    roofline_gemm = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} (tcgen05 loss contraction)",
+                     "bound": "tensor",
+                     "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
+                     "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
+                     "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
+                     "peak_source": f"{peak_src} bf16_tflops_sustained"}
+    launches = bwd_n + gemm_n + fwd_n
 
     # method diagnostics of the state after the timed steps (not timed)
     diag = layer.diagnose(sched(t), w.kappa)
@@ -492,7 +470,7 @@ def gpu_arm(args, rank, world, local):
             "diagnostics": diag,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
             "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
-                                   "forward": fwd_ms / args.steps, "step": step_ms / args.steps},
+                                   "forward": fwd_ms / args.steps},
         }
         print(json.dumps(line), flush=True)
     del graph

@@ -73,12 +73,7 @@ enum { GSQ_SCALE_GROUP = 0, GSQ_SCALE_KQUANT2 = 1 };
 enum { GSQ_GEMM_BF16 = 0, GSQ_GEMM_F32 = 1 };
 enum {
   GSQ_FLAG_NO_NOISE = 1u, /* g = 0: plain tempered softmax, no Gumbel draw             */
-  GSQ_FLAG_KEEP_G = 2u,   /* with GSQ_FLAG_FUSED: the fused step also stores G, so
-                             GSQ_T_G reads back the last step's dL/dW^                 */
-  GSQ_FLAG_FUSED = 4u,    /* bf16 layers: gsq_step runs one fused kernel (contraction
-                             with the backward, Lion and look-ahead as its epilogue)
-                             instead of two; the same results to rounding.  Measured
-                             slower than the two kernels on GB300, hence opt-in.       */
+                          /* bits 2 and 4 are reserved (rejected)                      */
   GSQ_FLAG_UNSTAGED = 8u  /* gsq_step's backward reads its input streams with direct
                              global loads instead of staging them through shared
                              memory with bulk asynchronous copies; the same kernel
@@ -126,6 +121,16 @@ enum { GSQ_PARAM_FULL = 0, GSQ_PARAM_SHIFT5 = 1, GSQ_PARAM_MASK_SIGN = 2 };
  *              the round-to-nearest code, times init_bias.  Projection:
  *              m = [l_m >= 0], b = 2 [l_b >= 0] - 1; code 0, 1, 2 for -a, 0, a;
  *              margin = 2|l_m|, or min(2|l_m|, 2|l_b|) when m = 1.
+ * index_offset flat index, within a larger layer this one is a shard of, of this
+ *              layer's first weight: weight (e, r, c) draws its noise with the
+ *              counter index index_offset + (e*R + r)*C + c (0 for a whole layer).
+ *              Rows and experts are independent in Eq. 1 with a linear f (the
+ *              loss is a sum over rows, L = sum_r D_r H D_r^T, and Lion acts
+ *              elementwise), so a shard holding rows [r0, r0 + R) of a one-expert
+ *              layer with C inputs (index_offset = r0*C), or experts [e0, e0 + E)
+ *              of a layer with R rows per expert (index_offset = e0*R*C), steps
+ *              its weights exactly as the whole layer would, and the shards'
+ *              losses sum to the layer's.  A multiple of 8.
  * Limits: 1 <= E, 1 <= R, 8 <= C, C % 8 == 0, E*R*C < 2^40, 2 <= K <= 8.
  */
 typedef struct gsq_layer_desc {
@@ -152,6 +157,7 @@ typedef struct gsq_layer_desc {
   float wd_scales;
   int32_t gemm_precision;
   int32_t param_mode;
+  uint64_t index_offset;
 } gsq_layer_desc;
 
 typedef struct gsq_layer gsq_layer; /* opaque handle, host memory owned by libgsq */
@@ -234,9 +240,7 @@ GSQ_API gsq_status gsq_init_logits(gsq_layer* layer, const uint8_t* codes_dev, c
  *              gradients ([L][E][R][C] fp32, L logits per weight, and
  *              [E][R][C/G] fp32), skips the Lion update and ignores next_tau.
  * Kernels: the contraction and the backward (+ update + look-ahead) are two
- * kernels; with GSQ_FLAG_FUSED (bf16, not exporting) one fused kernel runs the
- * contraction with the rest as its epilogue, so G stays on chip (GSQ_T_G then
- * reads back only with GSQ_FLAG_KEEP_G).  Outside export mode the backward
+ * kernels.  Outside export mode the backward
  * brings its input streams into shared memory with bulk asynchronous copies a
  * tile of 1,024 weights ahead (unless GSQ_FLAG_UNSTAGED, or the layer is too
  * small to give each block more than one tile); the results are the same bit
@@ -345,8 +349,7 @@ enum {
   GSQ_K_PACK = 4,
   GSQ_K_INIT = 5,
   GSQ_K_TOKENS = 6,   /* per-step tokens to the tensor-core operands (bf16, X^T) */
-  GSQ_K_STEP = 7,     /* fused step: loss contraction with backward + Lion (+ look-ahead) */
-  GSQ_K_COUNT = 8
+  GSQ_K_COUNT = 7
 };
 typedef struct gsq_profile {
   int32_t launches[GSQ_K_COUNT];
@@ -371,9 +374,12 @@ GSQ_API gsq_status gsq_profile_read(gsq_layer* layer, gsq_profile* out);
  * Its only scratch (a counter and one double per thread block) is a static
  * 131,328-byte device array inside libgsq that every GPU loading the library
  * holds until the process exits; nothing is allocated, so E*R*C is limited to
- * 16,777,216 weights (larger layers return GSQ_ERR_SHAPE).  The first call on a
- * device looks up that array's device address (cudaGetSymbolAddress); make that
- * first call before any stream capture on the device.  All calls on one GPU
+ * 16,777,216 weights (larger layers return GSQ_ERR_SHAPE).  The first call in a
+ * CUDA context looks up that array's device address (cudaGetSymbolAddress) and
+ * caches it under the context's ID; a later call in another context (after
+ * cudaDeviceReset, or with another context current on the device) looks it up
+ * again.  Make the first call in each context before any stream capture.
+ * flags accepts GSQ_FLAG_NO_NOISE only; any other bit is GSQ_ERR_INVALID_ARG.  All calls on one GPU
  * share its copy of the array and it keeps the last call's contents (the call
  * clears the counter before launching): calls that overlap on the same GPU (for
  * instance on two streams) race and corrupt each other's loss value; the state
@@ -421,8 +427,8 @@ GSQ_API const char* gsq_version(void);
 
 /* Name of the kernel that gsq_step launches for the part `kind` of a
  * non-exporting step of this layer (GSQ_K_GEMM: "k_tc_gemm_pair",
- * "k_tc_gemm", "k_simt_gemm" or "k_step_fused"; GSQ_K_BACKWARD:
- * "k_backward_staged", "k_backward" or "k_step_fused"), so timings can be
+ * "k_tc_gemm" or "k_simt_gemm"; GSQ_K_BACKWARD: "k_backward_staged" or
+ * "k_backward"), so timings can be
  * attributed (the paper has no counterpart: a reporting aid).  Static string
  * owned by the library; NULL for an invalid handle or another kind. */
 GSQ_API const char* gsq_kernel_name(gsq_layer* layer, int32_t kind);

@@ -86,15 +86,6 @@ class Workload:
         write logits, logit momentum (4L each), D for the next step (2)."""
         return 16 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
 
-    def fused_step_bytes(self) -> int:
-        """Algorithmic HBM bytes of one launch of the fused step kernel (loss
-        contraction with the backward, Lion and next forward as its epilogue): the
-        elementwise bytes without G, which never leaves the SM, plus the
-        contraction's operands read once, D of this step (2 per weight) and H
-        (2 C^2 per expert)."""
-        return (self.elementwise_bytes_per_weight() - 4 + 2) * self.n + \
-            2 * self.experts * self.cols * self.cols
-
     def gemm_flops_per_step(self) -> int:
         """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or
         per micro-batch Y = D X^T and G = 2 Y X (4 R C T per expert)."""

@@ -222,8 +222,7 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
   }
   if (d->gemm_precision != GSQ_GEMM_BF16 && d->gemm_precision != GSQ_GEMM_F32)
     return fail(GSQ_ERR_INVALID_ARG, "bad gemm_precision %d", d->gemm_precision);
-  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE | GSQ_FLAG_KEEP_G | GSQ_FLAG_FUSED |
-                                         GSQ_FLAG_UNSTAGED))
+  if (d->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE | GSQ_FLAG_UNSTAGED))
     return fail(GSQ_ERR_INVALID_ARG, "unknown flags 0x%x", d->flags);
   if (d->param_mode != GSQ_PARAM_FULL && d->param_mode != GSQ_PARAM_SHIFT5 &&
       d->param_mode != GSQ_PARAM_MASK_SIGN)
@@ -237,6 +236,8 @@ gsq_status validate_desc(const gsq_layer_desc* d) {
   if (d->beta1 < 0.f || d->beta1 > 1.f || d->beta2 < 0.f || d->beta2 > 1.f)
     return fail(GSQ_ERR_INVALID_ARG, "betas must be in [0, 1]");
   if (d->lr_logits < 0.f || d->lr_scales < 0.f) return fail(GSQ_ERR_INVALID_ARG, "negative learning rate");
+  if (d->index_offset % 8 != 0 || d->index_offset > (1ull << 62) - static_cast<uint64_t>(n))
+    return fail(GSQ_ERR_INVALID_ARG, "index_offset must be a multiple of 8 below 2^62 - E*R*C");
   return GSQ_OK;
 }
 
@@ -270,11 +271,8 @@ struct gsq_layer {
   bool tc;
   int tile_n;  // N of the tensor-core GEMM tile (128 or 256)
   int group_n; // column group of the GEMM's tile order
-  int fused_group_n;  // row-tile group of the fused step's tile order (1: whole rows first)
   int gemm_pair;      // 1: the loss GEMM runs on CTA pairs (cta_group::2)
   int test_stall;     // test hook (GSQ_TEST_STALL): 1 staged backward, 2 tensor-core GEMM
-  bool fused;   // GSQ_FLAG_FUSED: gsq_step runs the fused step kernel (bf16, not exporting)
-  bool keep_g;  // GSQ_FLAG_KEEP_G: the fused step also stores G
   bool g_valid; // the G buffer holds the last step's G
   size_t d_cur; // offset of the buffer holding the latest D written
   // pending forward (D valid for these arguments)
@@ -354,6 +352,7 @@ EwParams base_params(gsq_layer* L) {
     p.keys.k1[r] = key1 + r * 0xBB67AE85u;
   }
   p.noise = (d.flags & GSQ_FLAG_NO_NOISE) ? 0 : 1;
+  p.index_base = d.index_offset;
   p.lr_l = d.lr_logits;
   p.lr_s = d.lr_scales;
   p.b1 = d.beta1;
@@ -382,7 +381,7 @@ void prof_record(cudaEvent_t ev, cudaStream_t s) {
 // NVTX range names per kernel kind (visible in nsys / ncu timelines).
 const char* const kKindName[GSQ_K_COUNT] = {"gsq:forward", "gsq:gemm",  "gsq:backward",
                                             "gsq:project", "gsq:pack",  "gsq:init",
-                                            "gsq:tokens", "gsq:step"};
+                                            "gsq:tokens"};
 
 void prof_begin(gsq_layer* L, int kind, cudaStream_t s, int& slot) {
   nvtxRangePushA(kKindName[kind]);
@@ -584,8 +583,6 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   L->device = dev;
   L->num_sms = prop.multiProcessorCount;
   L->tc = tc;
-  L->keep_g = (desc->flags & GSQ_FLAG_KEEP_G) != 0;
-  L->fused = lay.has_d2 && tc && (desc->flags & GSQ_FLAG_FUSED) != 0;
   L->g_valid = false;
   L->d_cur = lay.D;
   L->d_ready = false;
@@ -636,9 +633,6 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
   L->group_n = kGemmGroupN;
-  // the fused step's tile order: groups of row tiles, as for the GEMM (whole rows
-  // first measured no faster)
-  L->fused_group_n = kGemmGroupN;
   if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)
     const int v = std::atoi(gn);
     if (v >= 0 && v <= 1024) L->group_n = v;
@@ -750,8 +744,7 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
   if (!(L->d_ready && L->d_step == step && L->d_tau == tau && L->d_kappa == kappa)) {
     if ((st = launch_fwd(L, step, tau, kappa, nullptr, s)) != GSQ_OK) return st;
   }
-  const bool fused = L->fused && !export_mode;
-  if (!fused && (st = launch_gemm(L, d_off(L, step), s)) != GSQ_OK) return st;
+  if ((st = launch_gemm(L, d_off(L, step), s)) != GSQ_OK) return st;
 
   EwParams p = base_params(L);
   p.t = static_cast<uint32_t>(step);
@@ -770,32 +763,13 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
   p.loss_out = loss_dev;
   int slot;
   cudaError_t e;
-  if (fused) {
-    const Shape& sh = L->shape;
-    FusedStep f;
-    f.P = p;
-    f.H = L->ws + L->lay.H;
-    f.D_t = L->ws + d_off(L, step);
-    f.D_next = L->ws + d_off(L, step + 1);
-    f.G_out = L->keep_g ? fptr(L, L->lay.G) : nullptr;
-    f.E = static_cast<int>(sh.E);
-    f.R = static_cast<int>(sh.R);
-    f.C = static_cast<int>(sh.C);
-    f.group_n = L->fused_group_n;
-    prof_begin(L, GSQ_K_STEP, s, slot);
-    e = launch_step_fused(f, L->num_sms, s);
-    prof_end(L, slot, s);
-    if (e != cudaSuccess) return cuda_fail(e, "fused step kernel");
-    L->g_valid = L->keep_g;
-  } else {
-    prof_begin(L, GSQ_K_BACKWARD, s, slot);
-    e = (!export_mode && L->grid_bwd_staged > 0)
-            ? launch_backward_staged(p, L->grid_bwd_staged, L->staged_plan, s)
-            : launch_backward(p, L->grid_bwd, s);
-    prof_end(L, slot, s);
-    if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
-    L->g_valid = true;
-  }
+  prof_begin(L, GSQ_K_BACKWARD, s, slot);
+  e = (!export_mode && L->grid_bwd_staged > 0)
+          ? launch_backward_staged(p, L->grid_bwd_staged, L->staged_plan, s)
+          : launch_backward(p, L->grid_bwd, s);
+  prof_end(L, slot, s);
+  if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
+  L->g_valid = true;
   if (lookahead) {
     L->d_cur = d_off(L, step + 1);
     L->d_ready = true;
@@ -1115,8 +1089,7 @@ gsq_status gsq_get_tensor(gsq_layer* L, int32_t which, void* dst_dev, size_t byt
   GSQ_INJECT("gsq_get_tensor");
   if (!valid(L)) return fail(GSQ_ERR_INVALID_ARG, "invalid layer handle");
   if (which == GSQ_T_G && !L->g_valid)
-    return fail(GSQ_ERR_STATE, "G holds no step's gradient: the fused step keeps it on chip unless "
-                               "the layer has GSQ_FLAG_KEEP_G");
+    return fail(GSQ_ERR_STATE, "G holds no step's gradient yet (no step has run)");
   return copy_tensor(L, which, dst_dev, L->ws + tensor_offset(L, which), bytes, stream, "gsq_get_tensor");
 }
 
@@ -1197,12 +1170,10 @@ const char* gsq_version(void) { return "0.1.0"; }
 const char* gsq_kernel_name(gsq_layer* L, int32_t kind) {
   if (!valid(L)) return nullptr;
   if (kind == GSQ_K_GEMM) {
-    if (L->fused) return "k_step_fused";
     if (!L->shape.d_bf16) return "k_simt_gemm";
     return L->gemm_pair ? "k_tc_gemm_pair" : "k_tc_gemm";
   }
   if (kind == GSQ_K_BACKWARD) {
-    if (L->fused) return "k_step_fused";
     return L->grid_bwd_staged > 0 ? "k_backward_staged" : "k_backward";
   }
   return nullptr;

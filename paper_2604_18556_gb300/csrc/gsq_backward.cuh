@@ -112,7 +112,7 @@ __device__ __forceinline__ void bwd_quad(const EwParams& P, const float (&q)[kMa
 #pragma unroll
     for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
     Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
-    Rx::noise(keys, P.t, static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
+    Rx::noise(keys, P.t, P.index_base + static_cast<uint64_t>(qc) * 4 + 2 * pr, P.noise, h);
     const float2 wt = rx.relax(l2, h, P.kappa_log2, P.inv_tau);
     const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
     const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
@@ -188,7 +188,7 @@ __device__ __forceinline__ void bwd_quad(const EwParams& P, const float (&q)[kMa
 #pragma unroll
         for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
         const Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
-        Rx::noise(keys, P.t_next, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+        Rx::noise(keys, P.t_next, P.index_base + static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
         const float2 wt = rx.value(l2, h, P.kappa_log2_next, P.inv_tau_next);
         const float2 dd = fma2(f2(s), wt, make_float2(-w[2 * pr], -w[2 * pr + 1]));
         d[2 * pr] = dd.x;

@@ -57,7 +57,7 @@ __global__ void __launch_bounds__(kEwThreads) k_forward(const EwParams P) {
 #pragma unroll
       for (int k = 0; k < K; ++k) l2[k] = make_float2(l[k][2 * pr], l[k][2 * pr + 1]);
       const Rx rx(q, sgrid, P.nlev, (j4 >> (16 * pr)) & 0xFFu, (j4 >> (16 * pr + 8)) & 0xFFu);
-      Rx::noise(keys, P.t, static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
+      Rx::noise(keys, P.t, P.index_base + static_cast<uint64_t>(qi) * 4 + 2 * pr, P.noise, h);
       const float2 wt = rx.value(l2, h, P.kappa_log2, P.inv_tau);
       // D = s w~ - W as one rounding per weight (identical in every kernel that forms D)
       const float2 wh = mul2(f2(s), wt);

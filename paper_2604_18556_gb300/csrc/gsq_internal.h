@@ -52,6 +52,7 @@ struct EwParams {
   // noise
   PhiloxRoundKeys keys;
   int noise;          // 0: g = 0
+  uint64_t index_base;  // noise counter index of weight 0 (a shard's offset in the whole layer)
   // step t (backward / forward)
   uint32_t t;
   float kappa_log2, inv_tau, kappa_over_tau;  // kappa_log2 = kappa * log2(e)
@@ -236,20 +237,6 @@ struct TcGemm {
 };
 bool tc_gemm_supported(int device);
 
-// Fused step (gsq_fused.cu): the tensor-core loss contraction with the backward,
-// Lion and look-ahead forward as its epilogue; G stays on chip unless G_out is
-// set.  H ([E*C][C]) and D_t ([E*R][C]) are bf16, K-major; D_next receives the
-// bf16 D of step t + 1 (a different buffer from D_t) when P.lookahead.
-struct FusedStep {
-  EwParams P;
-  const void* H;
-  const void* D_t;
-  void* D_next;
-  float* G_out;  // nullable
-  int E, R, C;
-  int group_n;   // tile order: groups of row tiles
-};
-cudaError_t launch_step_fused(const FusedStep& f, int num_sms, cudaStream_t s);
 int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 

@@ -5,6 +5,7 @@
 // their own buffers; the kernel's only scratch -- the last-block counter and
 // one double partial loss per thread block -- lives in the file-scope array
 // below, which every GPU that loads this library holds until the process exits.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -35,21 +36,69 @@ gsq_status na_fail(gsq_status st, const char* fmt, ...) {
   return set_last_error(st, buf);  // reported by gsq_last_error()
 }
 
-// Device address of g_noalloc_scratch on each device, looked up once with that
-// device current (the host-side name is only a stand-in, not a device address).
+// Device address of g_noalloc_scratch, cached per device together with the ID of
+// the CUDA context it was looked up in (the host-side name is only a stand-in,
+// not a device address).  A context ID is never reused within a process, so
+// after cudaDeviceReset, or when the caller makes another context current on
+// the same device, the module is loaded anew and the ID no longer matches: the
+// address is then looked up again instead of reusing a stale one.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+struct ScratchSlot {
+  unsigned long long ctx_id;
+  unsigned char* addr;
+};
+
 std::mutex g_addr_mu;
-unsigned char* g_addr[kMaxDevices] = {};
+ScratchSlot g_slot[kMaxDevices] = {};
+CtxGetCurrentFn g_ctx_current = nullptr;
+CtxGetIdFn g_ctx_id = nullptr;
+
+gsq_status driver_fns() {
+  if (g_ctx_current && g_ctx_id) return GSQ_OK;
+  void* a = nullptr;
+  void* b = nullptr;
+  cudaDriverEntryPointQueryResult qa, qb;
+  if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &a, 12000, cudaEnableDefault, &qa) !=
+          cudaSuccess ||
+      qa != cudaDriverEntryPointSuccess ||
+      cudaGetDriverEntryPointByVersion("cuCtxGetId", &b, 12000, cudaEnableDefault, &qb) !=
+          cudaSuccess ||
+      qb != cudaDriverEntryPointSuccess)
+    return na_fail(GSQ_ERR_CUDA, "driver entry points cuCtxGetCurrent / cuCtxGetId not found");
+  g_ctx_current = reinterpret_cast<CtxGetCurrentFn>(a);
+  g_ctx_id = reinterpret_cast<CtxGetIdFn>(b);
+  return GSQ_OK;
+}
+
+gsq_status current_ctx_id(unsigned long long* id) {
+  CUcontext ctx = nullptr;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || !ctx) return GSQ_ERR_CUDA;
+  return g_ctx_id(ctx, id) == CUDA_SUCCESS ? GSQ_OK : GSQ_ERR_CUDA;
+}
 
 gsq_status scratch_address(int dev, unsigned char** out) {
   std::lock_guard<std::mutex> lk(g_addr_mu);
-  if (!g_addr[dev]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess)
-      return na_fail(GSQ_ERR_CUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
-    g_addr[dev] = static_cast<unsigned char*>(p);
+  gsq_status st = driver_fns();
+  if (st != GSQ_OK) return st;
+  unsigned long long id = 0;
+  // No context is current before the first runtime call that needs one: the
+  // lookup below makes the device's primary context current, then it has an ID.
+  const bool have_ctx = current_ctx_id(&id) == GSQ_OK;
+  if (have_ctx && g_slot[dev].addr && g_slot[dev].ctx_id == id) {
+    *out = g_slot[dev].addr;
+    return GSQ_OK;
   }
-  *out = g_addr[dev];
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess)
+    return na_fail(GSQ_ERR_CUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
+  if (!have_ctx && current_ctx_id(&id) != GSQ_OK)
+    return na_fail(GSQ_ERR_CUDA, "no current CUDA context after the scratch lookup");
+  g_slot[dev].ctx_id = id;
+  g_slot[dev].addr = static_cast<unsigned char*>(p);
+  *out = g_slot[dev].addr;
   return GSQ_OK;
 }
 
@@ -80,6 +129,8 @@ extern "C" GSQ_API gsq_status gsq_backward_update_noalloc(const gsq_backward_arg
     return na_fail(GSQ_ERR_INVALID_ARG, "bad w_dtype");
   if (a->d_dtype != GSQ_DTYPE_F32 && a->d_dtype != GSQ_DTYPE_BF16)
     return na_fail(GSQ_ERR_INVALID_ARG, "bad d_dtype");
+  if (a->flags & ~static_cast<uint32_t>(GSQ_FLAG_NO_NOISE))
+    return na_fail(GSQ_ERR_INVALID_ARG, "flags: only GSQ_FLAG_NO_NOISE is accepted");
   if (a->step >= (1ull << 32)) return na_fail(GSQ_ERR_INVALID_ARG, "step must be < 2^32");
   if (!(a->tau > 0.f) || !std::isfinite(a->tau) || !std::isfinite(a->kappa))
     return na_fail(GSQ_ERR_INVALID_ARG, "need tau > 0 and finite kappa");

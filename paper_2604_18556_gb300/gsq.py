@@ -28,15 +28,15 @@ GSQ_DTYPE_F32, GSQ_DTYPE_BF16 = 0, 1
 GSQ_CALIB_H, GSQ_CALIB_X, GSQ_CALIB_BATCHES = 0, 1, 2
 GSQ_SCALE_GROUP, GSQ_SCALE_KQUANT2 = 0, 1
 GSQ_GEMM_BF16, GSQ_GEMM_F32 = 0, 1
-GSQ_FLAG_NO_NOISE, GSQ_FLAG_KEEP_G, GSQ_FLAG_FUSED, GSQ_FLAG_UNSTAGED = 1, 2, 4, 8
+GSQ_FLAG_NO_NOISE, GSQ_FLAG_UNSTAGED = 1, 8
 GSQ_PARAM_FULL, GSQ_PARAM_SHIFT5, GSQ_PARAM_MASK_SIGN = 0, 1, 2
 PARAM_MODES = {"full": GSQ_PARAM_FULL, "shift5": GSQ_PARAM_SHIFT5, "mask_sign": GSQ_PARAM_MASK_SIGN}
 (GSQ_T_LOGITS, GSQ_T_SCALES, GSQ_T_MOM_LOGITS, GSQ_T_MOM_SCALES, GSQ_T_D, GSQ_T_G, GSQ_T_W,
  GSQ_T_H, GSQ_T_KQ_D, GSQ_T_KQ_SC, GSQ_T_J0) = range(11)
-(GSQ_K_FORWARD, GSQ_K_GEMM, GSQ_K_BACKWARD, GSQ_K_PROJECT, GSQ_K_PACK, GSQ_K_INIT, GSQ_K_TOKENS,
- GSQ_K_STEP) = range(8)
-GSQ_K_COUNT = 8
-KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init", "tokens", "step"]
+(GSQ_K_FORWARD, GSQ_K_GEMM, GSQ_K_BACKWARD, GSQ_K_PROJECT, GSQ_K_PACK, GSQ_K_INIT,
+ GSQ_K_TOKENS) = range(7)
+GSQ_K_COUNT = 7
+KERNEL_NAMES = ["forward", "gemm", "backward", "project", "pack", "init", "tokens"]
 
 EXPORTED = ["gsq_workspace_size", "gsq_init_layer", "gsq_step", "gsq_forward", "gsq_project",
             "gsq_packed_size", "gsq_pack", "gsq_tensor_size", "gsq_get_tensor", "gsq_set_tensor",
@@ -61,7 +61,7 @@ class gsq_layer_desc(Structure):
         ("group_size", c_int32), ("scale_mode", c_int32), ("init_bias", c_float),
         ("flags", c_uint32), ("seed", c_uint64), ("lr_logits", c_float), ("lr_scales", c_float),
         ("beta1", c_float), ("beta2", c_float), ("wd_logits", c_float), ("wd_scales", c_float),
-        ("gemm_precision", c_int32), ("param_mode", c_int32),
+        ("gemm_precision", c_int32), ("param_mode", c_int32), ("index_offset", c_uint64),
     ]
 
 
@@ -251,8 +251,7 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
               lr_scales: float = 5e-5, beta1: float = 0.9, beta2: float = 0.95,
               wd_logits: float = 1.0, wd_scales: float = 0.0, gemm: int = GSQ_GEMM_BF16,
               noise: bool = True, param_mode: int = GSQ_PARAM_FULL,
-              keep_g: bool = False, fused: bool = False,
-              unstaged: bool = False) -> gsq_layer_desc:
+              unstaged: bool = False, index_offset: int = 0) -> gsq_layer_desc:
     d = gsq_layer_desc()
     d.num_experts, d.out_features, d.in_features = experts, rows, cols
     d.w_dtype = w_dtype
@@ -265,14 +264,14 @@ def make_desc(*, experts: int, rows: int, cols: int, grid: Sequence[float], grou
     d.group_size = group_size
     d.scale_mode = scale_mode
     d.init_bias = init_bias
-    d.flags = (0 if noise else GSQ_FLAG_NO_NOISE) | (GSQ_FLAG_KEEP_G if keep_g else 0) | \
-        (GSQ_FLAG_FUSED if fused else 0) | (GSQ_FLAG_UNSTAGED if unstaged else 0)
+    d.flags = (0 if noise else GSQ_FLAG_NO_NOISE) | (GSQ_FLAG_UNSTAGED if unstaged else 0)
     d.seed = seed
     d.lr_logits, d.lr_scales = lr_logits, lr_scales
     d.beta1, d.beta2 = beta1, beta2
     d.wd_logits, d.wd_scales = wd_logits, wd_scales
     d.gemm_precision = gemm
     d.param_mode = param_mode
+    d.index_offset = index_offset
     return d
 
 

@@ -206,8 +206,8 @@ class Case:
     """A layer problem on the GPU (through the C ABI) and the same problem for the oracle."""
 
     def __init__(self, w: C.Workload, gemm: str = "f32", noise: bool = True, seed=None,
-                 keep_calib_host: bool = True, device="cuda", keep_g: bool = False,
-                 fused: bool = False, unstaged: bool = False):
+                 keep_calib_host: bool = True, device="cuda", unstaged: bool = False,
+                 index_offset: int = 0):
         g = gsq()
         self.w = w
         self.gemm = gemm
@@ -220,8 +220,8 @@ class Case:
             self.calib = inputs.make_gram(w, device=device)
         hyper = dict(init_bias=w.init_bias, seed=w.seed if seed is None else seed,
                      lr_logits=w.lr_logits, lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                     wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise, keep_g=keep_g,
-                     fused=fused, unstaged=unstaged)
+                     wd_logits=w.wd_logits, wd_scales=w.wd_scales, noise=noise,
+                     unstaged=unstaged, index_offset=index_offset)
         self.layer = g.Layer(self.W, self.calib, w.grid, w.group, calib_kind=w.calib,
                              scale_mode=w.scale_mode, gemm=gemm, param=w.param,
                              tokens_per_batch=w.tokens if w.calib == "batches" else 0, **hyper)

@@ -137,6 +137,8 @@ def test_workspace_size_formula(lib):
     (dict(calib_kind=2, n_tokens=12), 1),        # ... that is a multiple of 8
     (dict(calib_kind=3), 1),
     (dict(param_mode=3), 1),                     # unknown parameterisation
+    (dict(index_offset=4), 1),                   # a shard's noise offset is a multiple of 8
+    (dict(index_offset=1 << 62), 1),             # ... and leaves room for the layer's indices
     (dict(param_mode=2), 1),                     # mask x sign needs {-a, 0, a}
     (dict(param_mode=2, grid=(-1.0, 0.0, 2.0)), 1),
     (dict(param_mode=2, grid=(-1.0, 0.5, 1.0)), 1),
@@ -155,17 +157,26 @@ def test_descriptor_validation(lib, kw, status):
 
 def test_flags_known_and_unknown(lib):
     """Every documented flag bit is accepted (the unstaged-backward bit among them);
-    an unknown bit is an argument error."""
-    for f in (lib.GSQ_FLAG_NO_NOISE, lib.GSQ_FLAG_KEEP_G | lib.GSQ_FLAG_FUSED,
-              lib.GSQ_FLAG_UNSTAGED):
+    a reserved or unknown bit is an argument error."""
+    for f in (lib.GSQ_FLAG_NO_NOISE, lib.GSQ_FLAG_UNSTAGED,
+              lib.GSQ_FLAG_NO_NOISE | lib.GSQ_FLAG_UNSTAGED):
         d = _desc(lib)
         d.flags = f
         assert lib.gsq_workspace_size(d) > 0
-    d = _desc(lib)
-    d.flags = 16
-    with pytest.raises(lib.GsqError) as ei:
-        lib.gsq_workspace_size(d)
-    assert ei.value.status == 1 and "flags" in lib.gsq_last_error()
+    for f in (2, 4, 16):
+        d = _desc(lib)
+        d.flags = f
+        with pytest.raises(lib.GsqError) as ei:
+            lib.gsq_workspace_size(d)
+        assert ei.value.status == 1 and "flags" in lib.gsq_last_error()
+
+
+def test_shard_offsets_accepted(lib):
+    """A row shard (offset r0 * C) and an expert shard (offset e0 * R * C) are valid
+    descriptors of the same size as the whole layer's piece."""
+    base = lib.gsq_workspace_size(_desc(lib))
+    assert lib.gsq_workspace_size(_desc(lib, index_offset=64 * 256)) == base
+    assert lib.gsq_workspace_size(_desc(lib, index_offset=7 * 64 * 256)) == base
 
 
 def test_parameterisations_size_their_logit_planes(lib):
@@ -230,3 +241,59 @@ def test_fault_injection_env(tmp_path):
     code2 = code.replace("gsq.gsq_workspace_size(d)", "gsq.gsq_init_layer(d, 256, 1 << 30, 0)")
     r = subprocess.run([sys.executable, "-c", code2], capture_output=True, text=True, env=env, check=True)
     assert r.stdout.strip() == "[8, 1, 1, 1]"   # injected first, then argument errors
+
+
+def _noalloc_args(lib, **kw):
+    a = lib.gsq_backward_args()
+    a.num_experts, a.out_features, a.in_features = 1, 64, 256
+    a.num_levels, a.group_size = 4, 128
+    for k, q in enumerate((-1.5, -0.5, 0.5, 1.5)):
+        a.grid[k] = q
+    a.w_dtype, a.d_dtype = lib.GSQ_DTYPE_BF16, lib.GSQ_DTYPE_BF16
+    # non-null stand-ins: every case below is rejected before any pointer is used
+    a.W = a.G = a.logits = a.m_logits = a.scales = a.m_scales = 4096
+    a.step, a.tau, a.kappa = 0, 1.0, 1.0
+    for k, v in kw.items():
+        if k == "grid":
+            for i, q in enumerate(v):
+                a.grid[i] = q
+        else:
+            setattr(a, k, v)
+    return a
+
+
+@pytest.mark.parametrize("kw,status,text", [
+    (dict(in_features=260), 2, "C % 8"),
+    (dict(in_features=0), 2, "C >= 8"),
+    (dict(num_experts=0), 2, "E >= 1"),
+    (dict(out_features=0), 2, "R >= 1"),
+    (dict(num_levels=1), 1, "num_levels"),
+    (dict(num_levels=9), 1, "num_levels"),
+    (dict(group_size=96), 2, "group_size"),
+    (dict(group_size=2), 2, "group_size"),
+    (dict(group_size=256, in_features=512), 2, "group_size"),
+    (dict(in_features=192), 2, "group_size"),            # C % G
+    (dict(W=None), 1, "required"),
+    (dict(G=None), 1, "required"),
+    (dict(m_scales=None), 1, "required"),
+    (dict(w_dtype=3), 1, "w_dtype"),
+    (dict(d_dtype=-1), 1, "d_dtype"),
+    (dict(flags=2), 1, "flags"),
+    (dict(flags=8), 1, "flags"),
+    (dict(step=1 << 32), 1, "step"),
+    (dict(tau=0.0), 1, "tau"),
+    (dict(tau=-1.0), 1, "tau"),
+    (dict(tau=float("inf")), 1, "tau"),
+    (dict(kappa=float("nan")), 1, "kappa"),
+    (dict(grid=(-1.5, -0.5, -0.5, 1.5)), 1, "ascend"),
+    (dict(out_features=4097, in_features=4096), 2, "16777216"),
+])
+def test_noalloc_validation_before_cuda(lib, kw, status, text):
+    """gsq_backward_update_noalloc rejects every invalid argument on the host, before
+    any CUDA call, with its status and a message naming the argument."""
+    with pytest.raises(lib.GsqError) as ei:
+        lib.gsq_backward_update_noalloc(_noalloc_args(lib, **kw), 0)
+    assert ei.value.status == status
+    assert text in lib.gsq_last_error(), lib.gsq_last_error()
+    assert lib._lib.gsq_backward_update_noalloc(None, None) == lib.GSQ_ERR_INVALID_ARG
+    assert "NULL" in lib.gsq_last_error()

@@ -7,7 +7,8 @@ is a static array inside libgsq.  Here the state lives in caller-owned torch
 buffers; each step, the handle-based gsq_step runs on a layer with the same
 initial state, and the new entry point, given that step's dL/dW^ (read from the
 layer), must leave the caller's buffers equal to the layer's state and report
-the same loss.  Two calls in a row, in both GEMM precisions.  This file sorts
+the same loss.  Two calls in a row, in both GEMM precisions, and once at the
+largest layer the static scratch serves (4096 x 4096, 2^24 weights).  This file sorts
 last so that a run stopping at the first failure has run every other test."""
 import ctypes
 
@@ -44,10 +45,15 @@ def _args(g, w, W, G, st, loss, t, tau, kappa, d_dtype):
     return a
 
 
-@pytest.mark.parametrize("gemm", ["f32", "bf16"])
-def test_noalloc_update_matches_step(gemm):
+@pytest.mark.parametrize("gemm,rows,cols", [
+    ("f32", 192, 512), ("bf16", 192, 512),
+    # exactly the documented limit of 2^24 weights: the last thread block writes the
+    # last partial slot of the static scratch array
+    ("bf16", 4096, 4096)])
+def test_noalloc_update_matches_step(gemm, rows, cols):
     g = gsq()
-    w = C.shrunk(C.WORKLOADS["llama8b_q_proj"], rows=192, cols=512, tokens=2048)
+    w = C.shrunk(C.WORKLOADS["llama8b_q_proj"], rows=rows, cols=cols,
+                 tokens=2048 if rows * cols < (1 << 24) else None)
     W = inputs.make_weight(w, device="cuda").contiguous()
     H = inputs.make_gram(w, device="cuda")
     layer = g.Layer(W, H, w.grid, w.group, gemm=gemm, seed=w.seed, lr_logits=w.lr_logits,

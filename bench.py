@@ -8,11 +8,18 @@ tau annealed 1.0 -> 0.1 over 500 steps).  Prints one JSON line.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gsq|reference]
                   [--workload NAME]
 
+The K timed steps are captured once as a CUDA graph; the graph is replayed
+until the timed window covers at least --min-window-ms, each replay (exactly K
+steps) bracketed by a synchronize, and the median replay gives ms_per_step.
+
 --impl reference times the CPU oracle (the plain float64 restatement of the
-method) on a row sample of the same layer; rows are independent, so the full
-layer's step time is the sample's time scaled by R / rows.  Under torchrun,
-every rank runs its own independent layer (weak scaling, no collective on the
-data path); rank 0 prints the whole-job throughput.
+method) on the host's cores: one single-threaded process per core, each
+following its own block of rows (rows are independent, Eq. 1 with a linear f),
+all blocks together covering the layer where the time allows it, else a row
+sample scaled by R / rows.  Under torchrun, the layer is split across the ranks
+(rows of a one-expert layer, whole experts of the MoE batch; no collective on
+the data path), so the whole job advances one layer step per step (strong
+scaling); rank 0 prints the whole layer's throughput.
 """
 from __future__ import annotations
 
@@ -42,7 +49,10 @@ def _args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-graph", action="store_true",
                     help="time eager launches instead of one CUDA-graph replay of the timed steps")
-    ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-step-seconds", type=float, default=1.5,
+                    help="oracle baseline: target seconds per timed step of each host core")
+    ap.add_argument("--min-window-ms", type=float, default=500.0,
+                    help="replay the captured K-step graph until the timed window is this long")
     ap.add_argument("--unstaged", action="store_true",
                     help="time the backward with direct global loads (GSQ_FLAG_UNSTAGED)")
     return ap.parse_args()
@@ -86,13 +96,12 @@ def committed_traffic(workload: str, kernel: str = "k_backward"):
     return d.get("workloads", {}).get(workload, {}).get("dram_bytes_per_launch")
 
 
-def rank_workload(w, rank: int, world: int):
-    """Each rank quantizes its own independent layer of the same shape (weak
-    scaling: rows and experts never exchange data, so ranks share nothing)."""
-    if world <= 1:
-        return w
-    import dataclasses
-    return dataclasses.replace(w, seed=w.seed + rank, data_seed=w.data_seed + 100 * rank)
+def rank_shard(w, rank: int, world: int):
+    """This rank's part of the layer: whole experts of a multi-expert layer, or a
+    block of rows of a one-expert layer (rows and experts never exchange data, so
+    the ranks share nothing but a copy of H)."""
+    from paper_2604_18556_gb300 import configs as C
+    return C.shard(w, rank, world)
 
 
 def max_over_ranks(x: float, device) -> float:
@@ -106,9 +115,39 @@ def max_over_ranks(x: float, device) -> float:
     return float(t.item())
 
 
-def whole_job_steps_per_s(ms_per_step: float, world: int) -> float:
-    """All ranks' steps per second: world layers advance one step every ms_per_step."""
-    return world * 1000.0 / ms_per_step
+def sum_over_ranks(x: float, device) -> float:
+    """The whole layer's value of a per-shard sum (the loss: rows add up)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t)
+    return float(t.item())
+
+
+def layer_steps_per_s(ms_per_step: float) -> float:
+    """Whole-layer steps per second: every rank advances its shard of the one
+    layer once per step, so the job advances the layer once every ms_per_step."""
+    return 1000.0 / ms_per_step
+
+
+def replays_for_window(ms_per_replay: float, min_window_ms: float, cap: int = 1000) -> int:
+    """Replays of the K-step graph that cover at least min_window_ms (>= 1)."""
+    if ms_per_replay <= 0:
+        return 1
+    import math
+    return max(1, min(cap, int(math.ceil(min_window_ms / ms_per_replay))))
+
+
+def elementwise_bytes_8d(w) -> int:
+    """Algorithmic HBM bytes of one step's elementwise work as the step is
+    defined (separate forward, backward and Lion passes over the streams):
+    forward reads the logits (4L) and W (b_W) and writes D (2); backward + Lion
+    reads the logits, their momenta (4L each) and G (4) and writes the logits and
+    momenta (4L each); local shift reads its base index j0 in both passes (2):
+    n (20L + b_W + 6 [+ 2]) per step.  Scale terms are O(n / G) and left out."""
+    return w.n * (20 * w.L + w.w_bytes() + 6 + (2 if w.param == "shift5" else 0))
 
 
 def _peaks():
@@ -122,10 +161,12 @@ def _peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms during the timed region."""
+    """nvidia-smi clocks, throttle reasons and utilisation sampled every 100 ms during the
+    timed region; the SM clock reported is the median over samples with the GPU busy."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,"
+              "utilization.gpu")
 
     def __init__(self, device_index: int):
         self.dev = device_index
@@ -136,7 +177,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "200", "-i", str(self.dev)], stdout=subprocess.PIPE,
+                 "-lms", "100", "-i", str(self.dev)], stdout=subprocess.PIPE,
                 stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -156,7 +197,7 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.thread.join(timeout=2)
-        sm, smax, reasons = [], [], set()
+        sm, smax, reasons, busy = [], [], set(), []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for ln in self.lines:
             parts = [p.strip() for p in ln.split(",")]
@@ -170,11 +211,20 @@ class ClockSampler:
             for nm, v in zip(names, parts[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(nm)
+            if len(parts) > 9:
+                try:
+                    if float(parts[9]) >= 50.0:
+                        busy.append(float(parts[1]))
+                except ValueError:
+                    pass
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
         sm.sort()
-        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        busy.sort()
+        med = busy[len(busy) // 2] if busy else sm[len(sm) // 2]
+        return {"sm_mhz": med, "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm), "samples_under_load": len(busy),
+                "sm_mhz_all_samples": sm[len(sm) // 2]}
 
 
 def _workload(name):
@@ -195,9 +245,20 @@ def _config(w, extra=None):
 
 
 # ----------------------------------------------------------------------------
-# CPU oracle on a row sample (baseline / reference arm)
+# CPU oracle on the host cores (baseline / reference arm)
 # ----------------------------------------------------------------------------
-def _oracle_problem(w, H_host, rows):
+_BLAS_THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+
+
+def host_cores() -> int:
+    """Cores this process may run on (its affinity mask, not the machine's count)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _oracle_problem(w, H_host):
     import numpy as np
     from oracle import gsq_oracle as O
     prob = O.Problem(E=w.experts, R=w.rows, C=w.cols, grid=np.asarray(w.grid, float), group=w.group,
@@ -208,56 +269,147 @@ def _oracle_problem(w, H_host, rows):
     return prob
 
 
-def _cpu_inputs(w, rows):
-    """The workload's W rows and H (expert 0) from the seeded generators (on the
-    GPU when one is present: input preparation only, not the timed oracle)."""
+def _input_device():
     import torch
-    from paper_2604_18556_gb300 import configs as C
-    from paper_2604_18556_gb300 import inputs
-    w1 = C.shrunk(w, experts=1)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     if dev == "cpu":
         torch.set_num_threads(max(1, os.cpu_count() or 1))
-    Wt = inputs.make_weight(w1, device=dev)[0, :rows].float().cpu().numpy()
-    H = inputs.make_gram(w1, device=dev)[0].double().cpu().numpy()
-    return Wt, H
+    return dev
 
 
-def _oracle_rows_for(seconds_per_step, t_one_row):
-    return max(1, int(seconds_per_step / max(t_one_row, 1e-6)))
+def _cpu_weight(w, rows):
+    """Rows [0, rows) of expert 0's W from the seeded generator (on the GPU when
+    one is present: input preparation only, not the timed oracle)."""
+    from paper_2604_18556_gb300 import inputs
+    return inputs.make_weight(w, device=_input_device(), experts=(0, 1),
+                              rows=(0, rows))[0].float().cpu().numpy()
 
 
-def _single_thread_env():
-    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+def _cpu_gram(w):
+    """Expert 0's H (float64), prepared like the weights."""
+    from paper_2604_18556_gb300 import inputs
+    return inputs.make_gram(w, device=_input_device(), experts=(0, 1))[0].double().cpu().numpy()
+
+
+def _oracle_block(root, w, w_path, h_path, lo, hi, n_warm, n_steps, barrier, queue, idx):
+    """One spawned, single-threaded worker: the oracle's whole step on rows
+    [lo, hi) of expert 0 -- n_warm untimed steps, then, once every worker is
+    ready, n_steps timed ones.  Puts (idx, seconds of each timed step, error)."""
+    for v in _BLAS_THREAD_VARS:
         os.environ[v] = "1"
+    sys.path.insert(0, root)
+    try:
+        import numpy as np
+        from oracle import gsq_oracle as O
+        Wt = np.array(np.load(w_path, mmap_mode="r")[lo:hi])
+        H = np.load(h_path, mmap_mode="r")          # pages shared by every worker
+        prob = _oracle_problem(w, H[None])
+        st = O.init_state(prob, Wt, np.arange(lo, hi), init_bias=w.init_bias)
+        for t in range(n_warm):
+            O.step(prob, st, t, w.tau(t), w.kappa)
+        barrier.wait(timeout=900)
+        times = []
+        for t in range(n_warm, n_warm + n_steps):
+            t0 = time.perf_counter()
+            O.step(prob, st, t, w.tau(t), w.kappa)
+            times.append(time.perf_counter() - t0)
+        queue.put((idx, times, None))
+    except Exception as e:  # report instead of leaving the parent waiting
+        try:
+            barrier.abort()
+        except Exception:
+            pass
+        queue.put((idx, None, repr(e)))
 
 
-def run_oracle_sample(w, step_budget_s: float, n_steps: int, n_warm: int, Wt=None, H=None):
-    """Times the oracle's full step on a row sample.  Returns (seconds per step of
-    the full layer, rows sampled, seconds measured)."""
+def run_oracle_parallel(w, workers, rows_per_worker, n_warm, n_steps, Wt, H, timeout_s=1800):
+    """`workers` spawned single-threaded oracle processes on consecutive blocks of
+    rows_per_worker rows of Wt (the last block may be shorter), all timed over the
+    same window.  Returns (seconds per timed step of the slowest worker, rows)."""
+    import multiprocessing as mp
+    import tempfile
     import numpy as np
-    from oracle import gsq_oracle as O
-    if Wt is None:
-        Wt, H = _cpu_inputs(w, min(w.rows, 256))
-    prob = _oracle_problem(w, H[None] if H.ndim == 2 else H, None)
-    # size the sample from a probe of 16 rows (after one untimed call)
-    probe = min(16, Wt.shape[0])
-    st = O.init_state(prob, Wt[:probe], np.arange(probe), init_bias=w.init_bias)
-    O.step(prob, st.copy(), 0, w.tau(0), w.kappa)
-    t0 = time.perf_counter()
-    O.step(prob, st, 0, w.tau(0), w.kappa)
-    t_row = (time.perf_counter() - t0) / probe
-    rows = min(Wt.shape[0], _oracle_rows_for(step_budget_s, t_row))
-    st = O.init_state(prob, Wt[:rows], np.arange(rows), init_bias=w.init_bias)
-    for t in range(n_warm):
-        O.step(prob, st, t, w.tau(t), w.kappa)
-    times = []
-    for t in range(n_warm, n_warm + n_steps):
-        t0 = time.perf_counter()
-        O.step(prob, st, t, w.tau(t), w.kappa)
-        times.append(time.perf_counter() - t0)
-    per = float(np.median(times))
-    return per * (w.experts * w.rows) / rows, rows, float(sum(times))
+    rows_total = Wt.shape[0]
+    blocks = [(i * rows_per_worker, min(rows_total, (i + 1) * rows_per_worker))
+              for i in range(workers)]
+    blocks = [b for b in blocks if b[1] > b[0]]
+    ctx = mp.get_context("spawn")             # never fork a process that holds a CUDA context
+    saved = {v: os.environ.get(v) for v in _BLAS_THREAD_VARS}
+    for v in _BLAS_THREAD_VARS:
+        os.environ[v] = "1"
+    try:
+        with tempfile.TemporaryDirectory() as td:
+            wp, hp = os.path.join(td, "W.npy"), os.path.join(td, "H.npy")
+            np.save(wp, np.ascontiguousarray(Wt, dtype=np.float32))
+            np.save(hp, np.ascontiguousarray(H, dtype=np.float64))
+            barrier, queue = ctx.Barrier(len(blocks)), ctx.Queue()
+            procs = [ctx.Process(target=_oracle_block,
+                                 args=(ROOT, w, wp, hp, lo, hi, n_warm, n_steps, barrier,
+                                       queue, i), daemon=True)
+                     for i, (lo, hi) in enumerate(blocks)]
+            for p in procs:
+                p.start()
+            times, errors = {}, []
+            try:
+                for _ in procs:
+                    idx, tt, err = queue.get(timeout=timeout_s)
+                    if err:
+                        errors.append(err)
+                    else:
+                        times[idx] = tt
+            finally:
+                for p in procs:
+                    p.join(timeout=30)
+                    if p.is_alive():
+                        p.terminate()
+            if errors:
+                raise RuntimeError("oracle worker failed: " + errors[0])
+    finally:
+        for v, x in saved.items():
+            if x is None:
+                os.environ.pop(v, None)
+            else:
+                os.environ[v] = x
+    per_step = max(sum(t) for t in times.values()) / n_steps
+    return per_step, sum(hi - lo for lo, hi in blocks)
+
+
+def time_oracle(w, cores, step_s, n_warm, n_steps, single=True):
+    """The oracle's whole-layer step time on `cores` host cores: one process per
+    core on its own block of expert 0's rows; the blocks cover all R rows when
+    that keeps a step near step_s seconds, else they are a sample and the time is
+    scaled by (E R) / rows (rows are independent; every row costs the same).  The
+    per-row cost comes from a 16-row probe.  With single=True the same block is
+    also timed alone on one core.  Returns a dict for the JSON line."""
+    import math
+    R = w.rows
+    H = _cpu_gram(w)
+    probe = min(16, R)
+    t_probe, _ = run_oracle_parallel(w, 1, probe, 1, 1, _cpu_weight(w, probe), H)
+    t_row = t_probe / probe
+    rpw = max(1, min(math.ceil(R / cores), int(step_s / max(t_row, 1e-9))))
+    workers = min(cores, math.ceil(R / rpw))
+    Wt = _cpu_weight(w, min(R, workers * rpw))
+    per_step, covered = run_oracle_parallel(w, workers, rpw, n_warm, n_steps, Wt, H)
+    scale = w.experts * w.rows / covered
+    out = {"full_step_s": per_step * scale, "workers": workers, "rows": covered,
+           "rows_per_worker": rpw, "per_step_s": per_step, "scale": scale,
+           "n_warm": n_warm, "n_steps": n_steps}
+    if single:
+        n1 = max(1, min(n_steps, 2))
+        t1, c1 = run_oracle_parallel(w, 1, rpw, 1, n1, Wt[:rpw], H)
+        out["single_core_full_step_s"] = t1 * (w.experts * w.rows) / c1
+        out["single_core_rows"] = c1
+    return out
+
+
+def oracle_sample_text(w, r, cores):
+    whole = w.experts * w.rows
+    what = ("the whole layer" if r["scale"] == 1.0 else
+            f"a sample of {r['rows']} of {whole} rows, time scaled by {r['scale']:.3g}")
+    return (f"{r['workers']} single-threaded oracle processes on {cores} host cores, "
+            f"{r['rows_per_worker']} rows each ({what}); {r['n_warm']} untimed + "
+            f"{r['n_steps']} timed steps each, slowest process's time per step")
 
 
 def run_oracle_tokens_sample(w, n_steps: int, rows: int = 256, tok=(512, 4096)):
@@ -275,7 +427,7 @@ def run_oracle_tokens_sample(w, n_steps: int, rows: int = 256, tok=(512, 4096)):
     from paper_2604_18556_gb300 import inputs
     w1 = C.shrunk(w, experts=1)
     Wt = inputs.make_weight(w1)[0, :rows].float().numpy()
-    prob = _oracle_problem(w1, None, None)
+    prob = _oracle_problem(w1, None)
     per_tok = []
     measured = 0.0
     for T in tok:
@@ -299,66 +451,103 @@ def run_oracle_tokens_sample(w, n_steps: int, rows: int = 256, tok=(512, 4096)):
 
 
 def reference_arm(args, rank, world):
+    """The oracle as it stands, on the host's cores, for the same workload and
+    metric; rank 0 alone runs it under torchrun."""
     if rank != 0:
         return 0
-    _single_thread_env()
     w = _workload(args.workload)
+    cores = host_cores()
+    common = {"impl": "reference", "metric": METRIC, "unit": UNIT, "n_gpus": args.gpus,
+              "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
+              "scaling": "strong", "vs_baseline": None, "dtype": "f64", "data": "synthetic"}
     if w.calib == "batches":
+        for v in _BLAS_THREAD_VARS:
+            os.environ[v] = "1"
         full_step_s, desc, _ = run_oracle_tokens_sample(w, max(args.steps, 1))
         value = 1.0 / full_step_s
-        print(json.dumps({
-            "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": full_step_s * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": _config(w, {"oracle": "numpy float64, one thread"}),
+        print(json.dumps(dict(common, **{
+            "value": value, "ms_per_step": full_step_s * 1e3,
+            "config": _config(w, {"oracle": "numpy float64, one thread"}),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-        }), flush=True)
+        })), flush=True)
         return 0
-    per_step_budget = 1.0
-    full_step_s, rows, measured = run_oracle_sample(w, per_step_budget, args.steps, args.warmup)
-    value = 1.0 / full_step_s
-    line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": full_step_s * 1e3,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": _config(w, {"oracle": "numpy float64, one thread"}),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"{rows} of {w.experts * w.rows} rows per step (rows are "
-                                   f"independent; full-layer time = sample time x {w.rows}/{rows}); "
-                                   f"{measured:.1f} s measured"},
+    r = time_oracle(w, cores, step_s=3.0, n_warm=args.warmup, n_steps=max(args.steps, 1),
+                    single=False)
+    value = 1.0 / r["full_step_s"]
+    print(json.dumps(dict(common, **{
+        "value": value, "ms_per_step": r["full_step_s"] * 1e3,
+        "config": _config(w, {"oracle": "numpy float64, one process per host core"}),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": r["workers"], "kind": "oracle",
+                         "sample": oracle_sample_text(w, r, cores)},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-    }
-    print(json.dumps(line), flush=True)
+    })), flush=True)
     return 0
 
 
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
+def _parallelism(w, sh, world):
+    if world == 1:
+        return "1 GPU, the whole layer"
+    (e0, e1), (r0, r1) = sh.experts, sh.rows
+    part = f"experts {e0}..{e1 - 1}" if w.experts > 1 else f"rows {r0}..{r1 - 1}"
+    return (f"{world} GPUs, one layer split by {'experts' if w.experts > 1 else 'rows'} "
+            f"(rank 0 holds {part}), H replicated, no collective in the timed region")
+
+
+def _timed_replays(args, run_k_steps, stream, world, device):
+    """Times replays of exactly K steps, each bracketed by a barrier (N > 1) and a
+    synchronize, until the window covers args.min_window_ms.  Returns the list of
+    per-replay milliseconds (the same count on every rank)."""
+    import torch
+    import torch.distributed as dist
+
+    def one():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        run_k_steps()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    reps = [one()]
+    n = replays_for_window(max_over_ranks(reps[0], device), args.min_window_ms)
+    for _ in range(n - 1):
+        reps.append(one())
+    if world > 1:
+        dist.barrier()
+    return reps
+
+
 def gpu_arm(args, rank, world, local):
     import numpy as np
     import torch
     import torch.distributed as dist
 
     torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
     if world > 1:
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist.init_process_group("nccl", device_id=device)
     from paper_2604_18556_gb300 import build
     build.build()
     from paper_2604_18556_gb300 import gsq, inputs
-    from paper_2604_18556_gb300 import configs as C
 
-    w = rank_workload(_workload(args.workload), rank, world)
-    W = inputs.make_weight(w, device="cuda")
-    H = inputs.make_gram(w, device="cuda")
-    H_host = H[0].double().cpu().numpy() if world == 1 and not args.no_cpu_baseline else None
+    whole = _workload(args.workload)
+    sh = rank_shard(whole, rank, world)
+    w = sh.workload
+    W = inputs.make_weight(whole, device="cuda", experts=sh.experts, rows=sh.rows)
+    H = inputs.make_gram(whole, device="cuda", experts=sh.experts)
+    hyper = dict(init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits, lr_scales=w.lr_scales,
+                 beta1=w.beta1, beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
+                 param=w.param, index_offset=sh.index_offset)
     layer = gsq.Layer(W, H, w.grid, w.group, calib_kind="H", scale_mode=w.scale_mode, gemm="bf16",
-                      init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
-                      lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param,
-                      unstaged=args.unstaged)
+                      unstaged=args.unstaged, **hyper)
     stream = torch.cuda.current_stream()
     loss = torch.zeros(1, device="cuda")
     T = w.steps
@@ -373,104 +562,111 @@ def gpu_arm(args, rank, world, local):
     layer.sync_status()
     torch.cuda.synchronize()
 
-    # The timed steps run as one CUDA graph (captured here, untimed): K distinct
-    # steps t0..t0+K-1, so the replay does exactly the work of K eager steps
-    # without the host launch gaps.  The library's profiling events are captured
-    # as event-record nodes and time the kernels of the replay.
+    # The K timed steps are captured once as a CUDA graph (untimed): K distinct
+    # steps t0..t0+K-1, so a replay does exactly the work of K eager steps without
+    # host launch gaps.  The library's profiling events become event-record nodes
+    # and time the kernels of every replay (the record read at the end is the last
+    # replay's).  K is even, so the look-ahead D a replay leaves behind sits in the
+    # buffer its first step reads.
     graph = None
+    layer.profile_enable(True)
+    layer.profile_read()
     if not args.no_graph:
-        layer.profile_enable(True)
-        layer.profile_read()
         graph = torch.cuda.CUDAGraph()
-        t_cap = t
         with torch.cuda.graph(graph):
             for i in range(args.steps):
-                layer.step(t_cap + i, sched(t_cap + i), w.kappa, next_tau=sched(t_cap + i + 1),
+                layer.step(t + i, sched(t + i), w.kappa, next_tau=sched(t + i + 1),
                            next_kappa=w.kappa, loss=loss)
         t += args.steps
         graph.replay()      # first replay (graph upload), untimed
         torch.cuda.synchronize()
+
+    state = {"t": t}
+
+    def run_k_steps():
+        if graph is not None:
+            graph.replay()
+            return
+        for _ in range(args.steps):
+            tt = state["t"]
+            layer.step(tt, sched(tt), w.kappa, next_tau=sched(tt + 1), next_kappa=w.kappa,
+                       loss=loss)
+            state["t"] = tt + 1
+
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
-    if graph is None:
-        layer.profile_enable(True)
-        layer.profile_read()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    if graph is not None:
-        graph.replay()
-    else:
-        for _ in range(args.steps):
-            layer.step(t, sched(t), w.kappa, next_tau=sched(t + 1), next_kappa=w.kappa, loss=loss)
-            t += 1
-    e1.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    reps = _timed_replays(args, run_k_steps, stream, world, device)
     clocks = sampler.stop()
-    ms_total = e0.elapsed_time(e1)
     prof = layer.profile_read()
     layer.profile_enable(False)
     layer.sync_status()
-    ms_total = max_over_ranks(ms_total, torch.device("cuda", local))
-    ms_step = ms_total / args.steps
-    value = whole_job_steps_per_s(ms_step, world)
+    ms_step = max_over_ranks(float(np.median(reps)), device) / args.steps
+    value = layer_steps_per_s(ms_step)
+    loss_total = sum_over_ranks(float(loss.item()), device)   # reporting only, untimed
 
     hbm, tf_burst, tf_sust, peak_src = _peaks()
-    n = w.n
     bwd_n, bwd_ms = prof["backward"]
     gemm_n, gemm_ms = prof["gemm"]
     fwd_n, fwd_ms = prof["forward"]
-    flops = w.gemm_flops_per_step()
     bwd_avg = bwd_ms / max(bwd_n, 1)
     gemm_avg = gemm_ms / max(gemm_n, 1)
-    bytes_bwd = w.elementwise_bytes_per_weight() * n
-    bwd_gbs = bytes_bwd / (bwd_avg * 1e-3) / 1e9
-    gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
+    per_weight_8d = 20 * w.L + w.w_bytes() + 6 + (2 if w.param == "shift5" else 0)
+    bytes_8d = elementwise_bytes_8d(w)
+    bytes_fused = w.elementwise_bytes_per_weight() * w.n
+    traffic = committed_traffic(w.name) if world == 1 else None
+    gbs = lambda nbytes: nbytes / (bwd_avg * 1e-3) / 1e9
     kname = layer.kernel_name(gsq.GSQ_K_BACKWARD)
-    roofline = {"kernel": f"{kname} (fused backward + Lion + next forward)", "bound": "hbm",
-                "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s", "frac": bwd_gbs / hbm,
-                "traffic": committed_traffic(w.name),
-                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
-                "algorithmic_bytes_per_launch": bytes_bwd, "avg_launch_ms": bwd_avg,
-                "frac_of_8TBps": bwd_gbs / 8000.0}
+    roofline = {
+        "kernel": f"{kname} (backward + Lion + the next step's forward, one launch per step)",
+        "bound": "hbm", "achieved": gbs(bytes_8d), "peak": hbm, "unit": "GB/s",
+        "frac": gbs(bytes_8d) / hbm, "traffic": traffic,
+        "peak_source": f"{peak_src}: MEASURED_PEAKS.json hbm_gbs (copy, burst)",
+        "algorithmic_bytes_per_weight": per_weight_8d, "weights_per_launch": w.n,
+        "algorithmic_bytes_per_launch": bytes_8d, "avg_launch_ms": bwd_avg,
+        "frac_of_8TBps": gbs(bytes_8d) / 8000.0,
+        "moved_bytes_per_launch_fused": bytes_fused,
+        "frac_on_moved_bytes_fused": gbs(bytes_fused) / hbm,
+        "frac_on_ncu_traffic": None if not traffic else gbs(traffic) / hbm}
+    flops = w.gemm_flops_per_step()
+    gemm_tfs = flops / (gemm_avg * 1e-3) / 1e12
     roofline_gemm = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} (tcgen05 loss contraction)",
-                     "bound": "tensor",
-                     "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
-                     "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst,
+                     "bound": "tensor", "achieved": gemm_tfs, "peak": tf_burst, "unit": "TFLOP/s",
+                     "frac": gemm_tfs / tf_burst, "frac_of_sustained": gemm_tfs / tf_sust,
                      "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
-                     "peak_source": f"{peak_src} bf16_tflops_sustained"}
-    launches = bwd_n + gemm_n + fwd_n
+                     "peak_source": f"{peak_src}: bf16_tflops (burst; the timed window is "
+                                    f"{sum(reps):.0f} ms of replays)"}
+    launches = (bwd_n + gemm_n + fwd_n) * (len(reps) if graph is not None else 1)
 
     # method diagnostics of the state after the timed steps (not timed)
-    diag = layer.diagnose(sched(t), w.kappa)
-    diag["after_step"] = t
+    diag = layer.diagnose(sched(state["t"]), w.kappa)
+    diag["after_step"] = state["t"]
     e2e = None
     if not args.no_e2e:
-        e2e = e2e_run(args, w, W, H, gsq, torch, rank, world)
+        e2e = e2e_run(args, w, W, H, gsq, torch, device, hyper)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:     # the oracle baseline: N = 1 only
-        cpu = cpu_baseline(args, w, W, H_host)
+        cpu = cpu_baseline(args, whole)
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32 (tensor-core GEMM bf16 in, f32 acc)",
+            "scaling": "strong", "vs_baseline": None,
+            "dtype": "f32 (tensor-core GEMM bf16 in, f32 acc)",
             "data": "synthetic (seeded; shapes and statistics of Llama-3.1-8B q_proj + calibration)",
-            "config": _config(w, {"parallelism": f"{world} independent layer(s), one per GPU",
-                                  "timing": ("one CUDA-graph replay of the timed steps (captured and "
-                                             "replayed once before the timed region)")
-                                  if graph is not None else "eager launches"}),
+            "config": _config(whole, {
+                "parallelism": _parallelism(whole, sh, world),
+                "timing": (f"{len(reps)} replays of one CUDA graph of the {args.steps} timed steps "
+                           f"(each replay bracketed by a synchronize; median replay), "
+                           f"{sum(reps):.1f} ms timed in total") if graph is not None else
+                          f"{len(reps)} rounds of {args.steps} eager steps, median round"}),
+            "timed_window_ms": sum(reps), "replays": len(reps),
             "roofline": roofline, "roofline_gemm": roofline_gemm, "clocks": clocks,
-            "diagnostics": diag,
+            "diagnostics": diag, "loss_last_step": loss_total,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
-            "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
-                                   "forward": fwd_ms / args.steps},
+            "kernel_ms_per_step": {"gemm": gemm_ms / max(gemm_n, 1), "backward": bwd_avg,
+                                   "forward": fwd_ms / max(args.steps, 1)},
         }
         print(json.dumps(line), flush=True)
     del graph
@@ -483,6 +679,7 @@ def gpu_arm(args, rank, world, local):
 def gpu_arm_tokens(args, rank, world, local):
     """One step = w.micro micro-batches of w.tokens per-step tokens (gsq_step_tokens),
     Lion after the last; the token batches are resident in HBM and reused."""
+    import numpy as np
     import torch
     import torch.distributed as dist
 
@@ -493,12 +690,14 @@ def gpu_arm_tokens(args, rank, world, local):
     build.build()
     from paper_2604_18556_gb300 import gsq, inputs
 
-    w = rank_workload(_workload(args.workload), rank, world)
-    W = inputs.make_weight(w, device="cuda")
+    whole = _workload(args.workload)
+    sh = rank_shard(whole, rank, world)
+    w = sh.workload
+    W = inputs.make_weight(whole, device="cuda", experts=sh.experts, rows=sh.rows)
     Xs = [inputs.make_token_batch(w, 0, j, device="cuda") for j in range(w.micro)]
     hyper = dict(init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits, lr_scales=w.lr_scales,
                  beta1=w.beta1, beta2=w.beta2, wd_logits=w.wd_logits, wd_scales=w.wd_scales,
-                 param=w.param)
+                 param=w.param, index_offset=sh.index_offset)
     layer = gsq.Layer(W, None, w.grid, w.group, calib_kind="batches", tokens_per_batch=w.tokens,
                       scale_mode=w.scale_mode, gemm="bf16", **hyper)
     stream = torch.cuda.current_stream()
@@ -521,24 +720,22 @@ def gpu_arm_tokens(args, rank, world, local):
     time.sleep(0.3)
     layer.profile_enable(True)
     layer.profile_read()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        one_step(layer, t, Xs, loss)
-        t += 1
-    e1.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    state = {"t": t}
+
+    def run_k_steps():
+        for _ in range(args.steps):
+            one_step(layer, state["t"], Xs, loss)
+            state["t"] += 1
+
+    device = torch.device("cuda", local)
+    reps = _timed_replays(args, run_k_steps, stream, world, device)
     clocks = sampler.stop()
     prof = layer.profile_read()
     layer.profile_enable(False)
     layer.sync_status()
-    ms_step = max_over_ranks(e0.elapsed_time(e1), torch.device("cuda", local)) / args.steps
-    value = whole_job_steps_per_s(ms_step, world)
+    n_timed = args.steps * len(reps)
+    ms_step = max_over_ranks(float(np.median(reps)), device) / args.steps
+    value = layer_steps_per_s(ms_step)
 
     hbm, tf_burst, tf_sust, peak_src = _peaks()
     gemm_n, gemm_ms = prof["gemm"]
@@ -549,40 +746,42 @@ def gpu_arm_tokens(args, rank, world, local):
     flops_per_launch = w.gemm_flops_per_step() / w.micro      # Y = D X^T and G = 2 Y X
     gemm_tfs = flops_per_launch / (gemm_avg * 1e-3) / 1e12
     bytes_step = w.elementwise_bytes_per_step()
-    bwd_gbs = bytes_step / (bwd_ms / args.steps * 1e-3) / 1e9
+    bwd_gbs = bytes_step / (bwd_ms / n_timed * 1e-3) / 1e9
     roofline = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} x 2 (Y = D X^T, then G = 2 Y X; "
                           "tcgen05, bf16 in, fp32 acc)",
-                "bound": "tensor", "achieved": gemm_tfs, "peak": tf_sust, "unit": "TFLOP/s",
-                "frac": gemm_tfs / tf_sust, "frac_of_burst": gemm_tfs / tf_burst, "traffic": None,
-                "flops_per_launch": flops_per_launch, "avg_launch_ms": gemm_avg,
-                "peak_source": f"{peak_src} bf16_tflops_sustained (MEASURED_PEAKS.json)"}
+                "bound": "tensor", "achieved": gemm_tfs, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": gemm_tfs / tf_burst, "frac_of_sustained": gemm_tfs / tf_sust,
+                "traffic": None, "flops_per_launch": flops_per_launch, "avg_launch_ms": gemm_avg,
+                "peak_source": f"{peak_src}: bf16_tflops (burst; MEASURED_PEAKS.json)"}
     roofline_bwd = {"kernel": "k_backward (accumulating / Lion + next forward), all micro-batches",
                     "bound": "hbm", "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s",
                     "frac": bwd_gbs / hbm, "algorithmic_bytes_per_step": bytes_step,
-                    "ms_per_step": bwd_ms / args.steps}
+                    "ms_per_step": bwd_ms / n_timed}
     launches = gemm_n * 2 + bwd_n + tok_n + fwd_n
 
     e2e = None
     if not args.no_e2e:
-        e2e = e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step)
+        e2e = e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, device, one_step)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:     # the oracle baseline: N = 1 only
-        cpu = cpu_baseline_tokens(args, w)
+        cpu = cpu_baseline_tokens(args, whole)
     if rank == 0:
         print(json.dumps({
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32 (tensor-core GEMMs bf16 in, f32 acc)",
+            "scaling": "strong", "vs_baseline": None,
+            "dtype": "f32 (tensor-core GEMMs bf16 in, f32 acc)",
             "data": "synthetic (seeded; Llama-3.1-8B q_proj shape, per-step token batches)",
-            "config": _config(w, {"parallelism": f"{world} independent layer(s), one per GPU",
+            "timed_window_ms": sum(reps), "replays": len(reps),
+            "config": _config(whole, {"parallelism": _parallelism(whole, sh, world),
                                   "micro_batches": w.micro, "tokens_per_micro_batch": w.tokens,
                                   "l2": "token batches of "
                                         f"{w.tokens * w.cols * 4 / 2**20:.0f} MiB each, larger "
                                         "than L2"}),
             "roofline": roofline, "roofline_backward": roofline_bwd, "clocks": clocks,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
-            "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "backward": bwd_ms / args.steps,
-                                   "tokens": tok_ms / args.steps, "forward": fwd_ms / args.steps},
+            "kernel_ms_per_step": {"gemm": gemm_ms / n_timed, "backward": bwd_ms / n_timed,
+                                   "tokens": tok_ms / n_timed, "forward": fwd_ms / n_timed},
         }), flush=True)
     layer.close()
     if world > 1:
@@ -590,7 +789,7 @@ def gpu_arm_tokens(args, rank, world, local):
     return 0
 
 
-def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step):
+def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, device, one_step):
     """The whole job through the public API from pinned host buffers: W and the
     micro-batch tokens uploaded, init, K steps (every micro-batch's loss read
     back), projection + packing, packed download."""
@@ -613,12 +812,12 @@ def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, world, one_step):
     packed_host = torch.empty(packed.numel(), dtype=torch.uint8).pin_memory()
     packed_host.copy_(packed, non_blocking=True)
     torch.cuda.synchronize()
-    dt = time.perf_counter() - t0
+    dt = max_over_ranks(time.perf_counter() - t0, device)
     layer.close()
     if not bool(torch.isfinite(loss_host).all()):
         raise RuntimeError("non-finite loss in the end-to-end run")
     h2d = W_host.numel() * W_host.element_size() + sum(X.numel() * 4 for X in X_host)
-    return {"value": world * K / dt, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
+    return {"value": K / dt, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
             "d2h_bytes_per_step": (4 * K * w.micro + packed_host.numel()) / K,
             "what": f"one {K}-step job: pinned W + {w.micro} token batches uploaded, init, "
                     f"{K} steps with every loss read back, projection + packing, download"}
@@ -641,23 +840,20 @@ def cpu_baseline_tokens(args, w):
     return {"value": 1.0 / full, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
 
 
-def e2e_run(args, w, W, H, gsq, torch, rank, world):
+def e2e_run(args, w, W, H, gsq, torch, device, hyper):
     """The whole per-layer job through the public API with host buffers: pinned
     W and H copied to the GPU, init, K steps (each step's loss read back into
-    pinned memory), projection + packing, packed result copied back."""
+    pinned memory), projection + packing, packed result copied back.  Under
+    torchrun every rank runs its shard's job; the slowest rank's time counts."""
     W_host = W.cpu().pin_memory()
     H_host = H.cpu().pin_memory()
-    stream = torch.cuda.current_stream()
     K = args.steps
     loss_host = torch.zeros(K, dtype=torch.float32).pin_memory()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     Wd = W_host.to("cuda", non_blocking=True)
     Hd = H_host.to("cuda", non_blocking=True)
-    layer = gsq.Layer(Wd, Hd, w.grid, w.group, scale_mode=w.scale_mode, gemm="bf16",
-                      init_bias=w.init_bias, seed=w.seed, lr_logits=w.lr_logits,
-                      lr_scales=w.lr_scales, beta1=w.beta1, beta2=w.beta2,
-                      wd_logits=w.wd_logits, wd_scales=w.wd_scales, param=w.param)
+    layer = gsq.Layer(Wd, Hd, w.grid, w.group, scale_mode=w.scale_mode, gemm="bf16", **hyper)
     loss = torch.zeros(K, device="cuda")
     for t in range(K):
         layer.step(t, w.tau(t % w.steps), w.kappa, next_tau=w.tau((t + 1) % w.steps),
@@ -668,46 +864,32 @@ def e2e_run(args, w, W, H, gsq, torch, rank, world):
     packed_host = torch.empty(packed.numel(), dtype=torch.uint8).pin_memory()
     packed_host.copy_(packed, non_blocking=True)
     torch.cuda.synchronize()
-    dt = time.perf_counter() - t0
+    dt = max_over_ranks(time.perf_counter() - t0, device)
     layer.close()
     h2d = W_host.numel() * W_host.element_size() + H_host.numel() * H_host.element_size()
     d2h = 4 * K + packed_host.numel()
     if not bool(torch.isfinite(loss_host).all()):
         raise RuntimeError("non-finite loss in the end-to-end run")
-    return {"value": world * K / dt, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
+    return {"value": K / dt, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
             "d2h_bytes_per_step": d2h / K,
             "what": f"one {K}-step layer job: pinned W+H upload, init, {K} steps with the loss "
                     f"read back each step, projection + packing, packed download"}
 
 
-def cpu_baseline(args, w, W, H_host):
-    """Oracle step on a bounded row sample, in a single-threaded child process."""
-    import numpy as np
-    import tempfile
-    rows = min(w.rows, 1024)
-    with tempfile.TemporaryDirectory() as td:
-        np.save(os.path.join(td, "W.npy"), W[0, :rows].float().cpu().numpy())
-        np.save(os.path.join(td, "H.npy"), H_host)
-        code = (
-            "import sys, json, numpy as np; sys.path.insert(0, %r)\n"
-            "import bench\n"
-            "from paper_2604_18556_gb300 import configs as C\n"
-            "w = C.WORKLOADS[%r]\n"
-            "Wt = np.load(%r); H = np.load(%r)\n"
-            "per, rows, meas = bench.run_oracle_sample(w, %f, 6, 1, Wt, H)\n"
-            "print(json.dumps([per, rows, meas]))\n"
-        ) % (ROOT, w.name, os.path.join(td, "W.npy"), os.path.join(td, "H.npy"),
-             args.cpu_sample_seconds / 7)
-        env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
-        r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
-                           cwd=ROOT, timeout=600)
-        if r.returncode != 0:
-            return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle",
-                    "sample": f"failed: {r.stderr[-300:]}"}
-        per, srows, meas = json.loads(r.stdout.strip().splitlines()[-1])
-    return {"value": 1.0 / per, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{srows} of {w.rows} rows, 6 timed steps + 1 warm-up ({meas:.1f} s "
-                      f"measured); full-layer step = sample x {w.rows}/{srows}"}
+def cpu_baseline(args, w):
+    """The oracle on every host core (one single-threaded process per core, each on
+    its own block of rows), with the same block on one core beside it."""
+    cores = host_cores()
+    try:
+        r = time_oracle(w, cores, step_s=args.cpu_step_seconds, n_warm=1, n_steps=3, single=True)
+    except Exception as e:  # the baseline is reported, never required
+        return {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": f"failed: {e!r}"[:300]}
+    return {"value": 1.0 / r["full_step_s"], "unit": UNIT, "cores": r["workers"], "kind": "oracle",
+            "sample": oracle_sample_text(w, r, cores),
+            "single_core": {"value": 1.0 / r["single_core_full_step_s"], "unit": UNIT, "cores": 1,
+                            "sample": f"the first {r['single_core_rows']}-row block alone on one "
+                                      f"core, time scaled to the whole layer"}}
 
 
 def main():

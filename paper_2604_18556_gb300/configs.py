@@ -155,6 +155,48 @@ ORDER = ["ternary_256x512", "llama8b_q_proj", "llama8b_down_proj", "llama70b_gat
          "moe64_kquant3"]
 
 
+@dataclass(frozen=True)
+class Shard:
+    """One rank's part of a layer split across GPUs: whole experts of a
+    multi-expert layer, or a contiguous block of rows of a one-expert layer
+    (rows and experts are independent in Eq. 1 with a linear f, so the shards
+    never exchange data).  `workload` is the shard's own layer problem; the
+    input generators take `experts` and `rows` (ranges of the whole layer's
+    global indices) to produce exactly its slice of W and H; `index_offset`
+    is the flat index of its first weight in the whole layer, so it draws the
+    whole layer's noise."""
+    workload: Workload
+    experts: Tuple[int, int]
+    rows: Tuple[int, int]
+    index_offset: int
+
+
+def _block(n: int, rank: int, world: int) -> Tuple[int, int]:
+    """[lo, hi) of block `rank` when n items split into `world` contiguous blocks
+    whose sizes differ by at most one (the first n % world are one larger)."""
+    base, extra = divmod(n, world)
+    lo = rank * base + min(rank, extra)
+    return lo, lo + base + (1 if rank < extra else 0)
+
+
+def shard(w: Workload, rank: int, world: int) -> Shard:
+    """Rank `rank` of `world`: experts split across ranks when the layer has
+    several (each rank gets whole experts, every row), else rows."""
+    if not 0 <= rank < world:
+        raise ValueError(f"rank {rank} outside world {world}")
+    if world == 1:
+        return Shard(w, (0, w.experts), (0, w.rows), 0)
+    if w.experts > 1:
+        if w.experts < world:
+            raise ValueError(f"{w.experts} experts cannot feed {world} ranks")
+        e0, e1 = _block(w.experts, rank, world)
+        return Shard(replace(w, experts=e1 - e0), (e0, e1), (0, w.rows), e0 * w.rows * w.cols)
+    if w.rows < world:
+        raise ValueError(f"{w.rows} rows cannot feed {world} ranks")
+    r0, r1 = _block(w.rows, rank, world)
+    return Shard(replace(w, rows=r1 - r0), (0, 1), (r0, r1), r0 * w.cols)
+
+
 def shrunk(w: Workload, experts: int | None = None, rows: int | None = None,
            cols: int | None = None, tokens: int | None = None) -> Workload:
     """The same workload recipe at a smaller shape (for tests the oracle finishes in seconds)."""

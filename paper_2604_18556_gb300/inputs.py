@@ -36,17 +36,21 @@ def _gen(device, seed: int) -> torch.Generator:
     return g
 
 
-def make_weight(w: Workload, device="cpu") -> torch.Tensor:
-    """W as [E, R, C] in the workload's storage dtype (fp32 or bf16)."""
+def make_weight(w: Workload, device="cpu", experts=None, rows=None) -> torch.Tensor:
+    """W as [E, R, C] in the workload's storage dtype (fp32 or bf16).  experts /
+    rows: [lo, hi) ranges of the layer's global expert and row indices to return
+    (a shard's slice; default all), drawn exactly as in the whole layer."""
     out_dtype = torch.float32 if w.w_dtype == "f32" else torch.bfloat16
-    W = torch.empty((w.experts, w.rows, w.cols), dtype=out_dtype, device=device)
-    for e in range(w.experts):
+    e0, e1 = experts if experts is not None else (0, w.experts)
+    r0, r1 = rows if rows is not None else (0, w.rows)
+    W = torch.empty((e1 - e0, r1 - r0, w.cols), dtype=out_dtype, device=device)
+    for e in range(e0, e1):
         g = _gen(device, w.data_seed + _W_ID + 17 * e)
         z = torch.randn((w.rows, w.cols), generator=g, device=device, dtype=torch.float32)
         gr = _gen(device, w.data_seed + _ROWSCALE_ID + 17 * e)
         u = torch.rand((w.rows, 1), generator=gr, device=device, dtype=torch.float32)
         rho = torch.exp(math.log(0.5) + u * (math.log(2.0) - math.log(0.5)))
-        W[e] = (0.02 * z * rho).to(out_dtype)
+        W[e - e0] = (0.02 * z * rho)[r0:r1].to(out_dtype)
     return W
 
 
@@ -94,13 +98,16 @@ def make_token_batch(w: Workload, step: int, micro: int, device="cpu") -> torch.
     return X
 
 
-def make_gram(w: Workload, device="cpu", chunk: int = 8192) -> torch.Tensor:
-    """H = X^T X as [E, C, C] fp32, built chunk by chunk with TF32 off."""
+def make_gram(w: Workload, device="cpu", chunk: int = 8192, experts=None) -> torch.Tensor:
+    """H = X^T X as [E, C, C] fp32, built chunk by chunk with TF32 off; experts:
+    [lo, hi) range of global expert indices to build (default all)."""
     prev = torch.backends.cuda.matmul.allow_tf32
     torch.backends.cuda.matmul.allow_tf32 = False
+    e0, e1 = experts if experts is not None else (0, w.experts)
     try:
-        H = torch.zeros((w.experts, w.cols, w.cols), dtype=torch.float32, device=device)
-        for e in range(w.experts):
+        H = torch.zeros((e1 - e0, w.cols, w.cols), dtype=torch.float32, device=device)
+        for e in range(e0, e1):
+            He = H[e - e0]
             g = _gen(device, w.data_seed + _X_ID + 17 * e)
             ch = _outlier_channels(w, e, device) if w.outliers else None
             done = 0
@@ -109,9 +116,9 @@ def make_gram(w: Workload, device="cpu", chunk: int = 8192) -> torch.Tensor:
                 x = _token_chunk(w, g, m, device)
                 if ch is not None:
                     x[:, ch] *= w.outlier_scale
-                H[e].addmm_(x.t(), x)
+                He.addmm_(x.t(), x)
                 done += m
-            H[e] = 0.5 * (H[e] + H[e].t())
+            H[e - e0] = 0.5 * (He + He.t())
         return H
     finally:
         torch.backends.cuda.matmul.allow_tf32 = prev

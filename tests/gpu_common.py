@@ -287,3 +287,39 @@ class Case:
         nr = self.w.experts * self.w.rows
         ids = np.arange(nr) if rows is None else np.asarray(rows)
         return O.init_state(self.prob, self.W_host[ids], ids, init_bias=self.w.init_bias)
+
+
+def gather_rows(case, rows) -> O.RowState:
+    """The GPU state of the given global rows (row id = e*R + r) as an oracle
+    RowState, gathered on the device so only those rows cross to the host."""
+    g = gsq()
+    w = case.w
+    nr, L, Cc = w.experts * w.rows, w.L, w.cols
+    rows = np.asarray(rows, dtype=np.int64)
+    idx = torch.from_numpy(rows).cuda()
+    f = lambda which: case.layer.get_tensor(which, torch.float32)
+    st = O.RowState(
+        row_ids=rows, W=case.W.view(nr, Cc)[idx].float().cpu().double().numpy(),
+        logits=f(g.GSQ_T_LOGITS).view(L, nr, Cc)[:, idx].cpu().numpy(),
+        scales=f(g.GSQ_T_SCALES).view(nr, Cc // w.group)[idx].cpu().numpy(),
+        m_logits=f(g.GSQ_T_MOM_LOGITS).view(L, nr, Cc)[:, idx].cpu().numpy(),
+        m_scales=f(g.GSQ_T_MOM_SCALES).view(nr, Cc // w.group)[idx].cpu().numpy())
+    if w.param == "shift5":
+        st.j0 = case.layer.get_tensor(g.GSQ_T_J0, torch.uint8).view(nr, Cc)[idx].cpu().numpy()
+    if w.scale_mode == "kquant2":
+        d16 = case.layer.get_tensor(g.GSQ_T_KQ_D, torch.int16).view(nr, Cc // 256)[idx]
+        st.kq_d = O.f16_bits_to_f32(d16.cpu().numpy().view(np.uint16))
+        sc = case.layer.get_tensor(g.GSQ_T_KQ_SC, torch.int8).view(nr, Cc // 16)[idx]
+        st.kq_sc = sc.cpu().numpy().astype(np.int32)
+    return st
+
+
+class HostH:
+    """Expert -> float64 H lookup for the oracle holding only the experts of the
+    sampled rows (a full-size layer's H for every expert need not be on the host)."""
+
+    def __init__(self, calib, experts):
+        self.H = {int(e): calib[int(e)].double().cpu().numpy() for e in experts}
+
+    def __getitem__(self, e):
+        return self.H[int(e)]

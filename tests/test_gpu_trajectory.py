@@ -1,0 +1,219 @@
+"""Whole schedules of the paper-shaped workloads against the oracle's own trajectory.
+
+Each workload's full-size layer runs its whole schedule on the GPU -- 500 steps
+(4096 x 4096, tau 1.0 -> 0.1), 200 (4096 x 14336), 100 (28672 x 8192, then
+projection and packing), 100 (64 experts of 2048 x 7168, K-Quant, then
+projection and packing) -- with the benchmark's look-ahead sequence and the fp32
+loss contraction, whose only difference from the oracle is fp32 rounding.  The
+oracle follows a sample of rows on its own trajectory from the same initial
+state with the same noise (rows are independent given H: Eq. 1 with a linear f
+is a sum over rows, so a row subset is exact); Alg. 2's loop with Lion (§3.3).
+
+Lion moves a parameter by lr sign(c) plus its decay, so two trajectories whose
+gradients differ by rounding agree to rounding, except where sign(c) was decided
+by a difference below that rounding: such a flip moves the entry by 2 lr and
+feeds back, through D and H, into its row's later gradients.  Checks:
+  * logits: an entry either agrees within fp32 rounding drift (|d| <= lr / 4) or
+    has flipped (|d| <= 2 lr per step); flipped entries are a small fraction,
+    at most FLIP_PER_STEP x steps of all entries;
+  * projection: codes bit-exact wherever both sides' margins are >= 1e-5;
+  * scales: within 1e-4 relative (|a - b| <= 1e-4 (|b| + rms b)) except entries
+    that flipped, which differ by multiples of 2 lr_scales;
+  * packing (gate_proj, MoE): the GPU's bytes for the sampled rows equal the
+    oracle's packing of the GPU's final state (bit for bit), and their codes and
+    scales equal the oracle's own final state outside the margin exclusion and
+    the flipped scales.
+A shorter run on the performance path (bf16 tensor-core contraction, staged
+backward) checks the same with the bf16 flip rate, and the step-0 loss of the
+whole 4096 x 4096 layer is compared with the oracle's float64 loss over every
+row, on both contraction paths."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_common import TOL_BF16, TOL_F32, Case, HostH, gather_rows, gsq
+from oracle import gsq_oracle as O
+from paper_2604_18556_gb300 import configs as C
+
+pytestmark = pytest.mark.gpu
+
+# Per-step fraction of logit entries whose Lion sign may differ between the fp32
+# GPU path and the float64 oracle (|c| below the contraction's rounding), and
+# between the bf16 tensor-core path and the oracle (|c| below G's 2e-2 tolerance).
+FLIP_PER_STEP = {"f32": 1e-4, "bf16": 1e-3}
+
+
+def _sample_rows(w, k):
+    """k rows: the first and last of the layer, the last of the first expert, and
+    seeded random ones; for a multi-expert layer, rows of three experts."""
+    rng = np.random.default_rng(29)
+    if w.experts > 1:
+        experts = [0, w.experts // 2, w.experts - 1]
+        per = k // len(experts)
+        rows = []
+        for e in experts:
+            rr = {0, w.rows - 1} | set(rng.integers(0, w.rows, per - 2).tolist())
+            rows += [e * w.rows + r for r in sorted(rr)]
+        return np.array(rows, dtype=np.int64)
+    rr = {0, w.rows - 1} | set(rng.integers(0, w.rows, k - 2).tolist())
+    return np.array(sorted(rr), dtype=np.int64)
+
+
+def _diverged(gpu, orc, lr):
+    """Entries that no longer agree to rounding (a Lion flip moved one side by 2 lr)."""
+    return np.abs(np.asarray(gpu, np.float64) - np.asarray(orc, np.float64)) > 0.25 * lr
+
+
+def _check_state(w, gst, ost, steps, path, what):
+    """Logits, scales and codes of the GPU rows against the oracle's trajectory."""
+    d = np.abs(gst.logits.astype(np.float64) - ost.logits)
+    div = _diverged(gst.logits, ost.logits, w.lr_logits)
+    frac = float(div.mean())
+    print(f"{what}: {steps} steps, diverged logits {frac:.2e} ({int(div.sum())}/{div.size}), "
+          f"max drift elsewhere {float(d[~div].max()):.2e}, max |d| {float(d.max()):.2e}")
+    assert frac <= FLIP_PER_STEP[path] * steps, (what, frac)
+    assert float(d.max()) <= 2.0 * w.lr_logits * steps * 1.001, what
+    # codes: bit-exact where both margins clear the exclusion
+    gc, gm = O.project(gst.logits, j0=gst.j0, levels=w.K, mask_sign=w.param == "mask_sign")
+    oc, om = O.project(ost.logits, j0=ost.j0, levels=w.K, mask_sign=w.param == "mask_sign")
+    keep = (gm >= 1e-5) & (om >= 1e-5)
+    assert np.array_equal(gc[keep], oc[keep]), (what, int((gc[keep] != oc[keep]).sum()))
+    # scales: 1e-4 relative, except those that flipped
+    s_g, s_o = gst.scales.astype(np.float64), ost.scales.astype(np.float64)
+    rms = float(np.sqrt(np.mean(s_o * s_o)))
+    sdiv = np.abs(s_g - s_o) > TOL_F32 * (np.abs(s_o) + rms)
+    if w.lr_scales == 0.0:
+        assert np.array_equal(gst.scales, ost.scales), what      # frozen (K-Quant)
+    else:
+        print(f"{what}: scales outside 1e-4: {int(sdiv.sum())}/{sdiv.size}")
+        assert sdiv.mean() <= FLIP_PER_STEP[path] * steps * 10, (what, float(sdiv.mean()))
+        k = np.abs(s_g - s_o)[sdiv] / (2 * w.lr_scales)        # whole Lion steps apart
+        assert np.all(k <= steps * 1.001), what
+    return keep, sdiv
+
+
+def _packed_rows(w, packed, rows):
+    """The sampled rows' part of gsq_pack's output, laid out as the oracle packs
+    those rows on their own (codes section, then fp16 scales; or K-Quant records)."""
+    C_ = w.cols
+    if w.scale_mode == "kquant2":
+        rec = C_ // O.SUPER_BLOCK * O.KQ_RECORD
+        return b"".join(packed[r * rec:(r + 1) * rec] for r in rows)
+    bits = O.code_bits(w.K)
+    row_code = C_ * bits // 8
+    sec = O.code_section_bytes(w.n, w.K)
+    ng = C_ // w.group
+    codes = b"".join(packed[r * row_code:(r + 1) * row_code] for r in rows)
+    codes += b"\0" * ((-len(codes)) % 16)
+    return codes + b"".join(packed[sec + 2 * r * ng:sec + 2 * (r + 1) * ng] for r in rows)
+
+
+def _pack(w, st, codes):
+    if w.scale_mode == "kquant2":
+        return O.pack_kquant2(codes.reshape(-1), st.kq_d, st.kq_sc)
+    return O.pack_group(codes.reshape(-1), st.scales, w.K)
+
+
+def _check_pack(case, w, rows, gst, ost, keep, sdiv):
+    g = gsq()
+    packed = torch.empty(case.layer.packed_size(), dtype=torch.uint8, device="cuda")
+    case.layer.pack(packed)
+    got = _packed_rows(w, packed.cpu().numpy().tobytes(), rows)
+    gc, _ = O.project(gst.logits)
+    assert got == _pack(w, gst, gc), w.name            # state-synced: bit for bit (R23)
+    # against the oracle's own final state: unpack and compare what is unique
+    oc, _ = O.project(ost.logits)
+    n = len(rows) * w.cols
+    if w.scale_mode == "kquant2":
+        codes, d, sc = O.unpack_kquant2(got, n)
+        od = O.unpack_kquant2(_pack(w, ost, oc), n)
+        assert np.array_equal(d, od[1]) and np.array_equal(sc, od[2])
+    else:
+        codes, s16 = O.unpack_group(got, n, w.K, n // w.group)
+        o_codes, o16 = O.unpack_group(_pack(w, ost, oc), n, w.K, n // w.group)
+        ok = ~sdiv.reshape(-1)
+        assert np.array_equal(s16[ok], o16[ok])
+    assert np.array_equal(codes.reshape(oc.shape)[keep], oc[keep])
+
+
+TRAJECTORIES = [("llama8b_q_proj", 16), ("llama8b_down_proj", 12), ("llama70b_gate_proj", 16),
+                ("moe64_kquant3", 24)]
+
+
+@pytest.mark.parametrize("name,k", TRAJECTORIES)
+def test_full_schedule_trajectory_fp32(name, k):
+    w = C.WORKLOADS[name]
+    case = Case(w, gemm="f32", keep_calib_host=False)
+    rows = _sample_rows(w, k)
+    case.prob.H = HostH(case.calib, sorted(set((rows // w.rows).tolist())))
+    del case.calib
+    torch.cuda.empty_cache()
+    ost = case.oracle_init(rows)
+    gst = gather_rows(case, rows)
+    assert np.array_equal(gst.logits, ost.logits) and np.array_equal(gst.scales, ost.scales)
+    loss = torch.zeros(1, device="cuda")
+    T = w.steps
+    for t in range(T):
+        nxt = w.tau(t + 1) if t + 1 < T else 0.0
+        case.layer.step(t, w.tau(t), w.kappa, next_tau=nxt, next_kappa=w.kappa, loss=loss)
+        O.step(case.prob, ost, t, w.tau(t), w.kappa)
+        if (t + 1) % max(1, T // 5) == 0 and t + 1 < T:
+            _check_state(w, gather_rows(case, rows), ost, t + 1, "f32", f"{name} step {t + 1}")
+    case.layer.sync_status()
+    assert np.isfinite(loss.item())
+    gst = gather_rows(case, rows)
+    keep, sdiv = _check_state(w, gst, ost, T, "f32", f"{name} final")
+    if w.pack:
+        _check_pack(case, w, rows, gst, ost, keep, sdiv)
+    case.layer.close()
+
+
+def test_bf16_path_trajectory_q_proj():
+    """The performance path (bf16 tensor-core contraction, staged backward, look-ahead)
+    for the first 20 steps of the 4096 x 4096 schedule."""
+    g = gsq()
+    w = C.WORKLOADS["llama8b_q_proj"]
+    case = Case(w, gemm="bf16", keep_calib_host=False)
+    assert case.layer.kernel_name(g.GSQ_K_BACKWARD) == "k_backward_staged"
+    rows = _sample_rows(w, 16)
+    case.prob.H = HostH(case.calib, [0])
+    del case.calib
+    ost = case.oracle_init(rows)
+    loss = torch.zeros(1, device="cuda")
+    T = 20
+    for t in range(T):
+        case.layer.step(t, w.tau(t), w.kappa, next_tau=w.tau(t + 1), next_kappa=w.kappa, loss=loss)
+        O.step(case.prob, ost, t, w.tau(t), w.kappa)
+    case.layer.sync_status()
+    _check_state(w, gather_rows(case, rows), ost, T, "bf16", "q_proj bf16")
+    case.layer.close()
+
+
+def test_full_layer_step0_loss_q_proj():
+    """L_0 = tr(D H D^T) of the whole 4096 x 4096 layer (every row) against the
+    oracle's float64 loss: fp32 contraction within 1e-4, bf16 within 2e-2."""
+    w = C.WORKLOADS["llama8b_q_proj"]
+    got = {}
+    H = None
+    for gemm in ("f32", "bf16"):
+        case = Case(w, gemm=gemm, keep_calib_host=False)
+        if H is None:
+            H = case.calib[0].double().cpu().numpy()
+        loss = torch.zeros(1, device="cuda")
+        case.layer.step(0, w.tau(0), w.kappa, loss=loss)
+        case.layer.sync_status()
+        got[gemm] = float(loss.item())
+        W_host = case.W_host
+        prob = case.prob
+        case.layer.close()
+        del case
+        torch.cuda.empty_cache()
+    prob.H = H[None]
+    ids = np.arange(w.rows)
+    st = O.init_state(prob, W_host, ids, init_bias=w.init_bias)
+    fw = O.forward(prob, st, 0, w.tau(0), w.kappa)
+    ref, _ = O.loss_and_grad(prob, ids, fw.D)
+    rel = {k: abs(v - ref) / ref for k, v in got.items()}
+    print(f"full-layer step-0 loss: oracle {ref:.9e}, fp32 {got['f32']:.9e} (rel {rel['f32']:.2e}), "
+          f"bf16 {got['bf16']:.9e} (rel {rel['bf16']:.2e})")
+    assert rel["f32"] <= TOL_F32 and rel["bf16"] <= TOL_BF16, rel

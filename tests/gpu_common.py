@@ -108,6 +108,29 @@ def bf16_operand_bounds(ref, prob, zmax):
     return dD, np.stack(dH), 2.0 * (1 + 4 * u) * dG
 
 
+def bf16_criterion(G, ref_G, g_bound, what, tol=TOL_BF16):
+    """The 2e-2 relative criterion on the bf16 path's G, made visible.  Prints the
+    worst elementwise error in units of tol (|b| + rms b), the fraction of entries
+    beyond it and the tensor-norm relative error; asserts that every entry beyond
+    the criterion is one where the operands' own worst-case error (g_bound: D and
+    H each one bf16 rounding from the oracle's, bf16_operand_bounds) already
+    exceeds it -- cancellation in G, not an error of the kernel.  Returns the
+    worst ratio."""
+    a = np.asarray(G, np.float64).reshape(-1)
+    b = np.asarray(ref_G, np.float64).reshape(-1)
+    gb = np.asarray(g_bound, np.float64).reshape(-1)
+    scale = tol * (np.abs(b) + np.sqrt(np.mean(b * b)))
+    ratio = np.abs(a - b) / scale
+    beyond = ratio > 1.0
+    norm_rel = float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+    worst = float(ratio.max()) if ratio.size else 0.0
+    print(f"bf16 criterion {what}: worst |dG| = {worst:.3f} x 2e-2 (|G| + rms G), "
+          f"{int(beyond.sum())}/{beyond.size} entries beyond, ||dG||/||G|| = {norm_rel:.2e}")
+    explained = gb[beyond] > scale[beyond]
+    assert explained.all(), (what, int((~explained).sum()), worst)
+    return worst
+
+
 def grad_bounds(ref, prob, tol, q=None, g_bound=None):
     """Elementwise bounds for the logit and scale gradients when the only
     reduced-precision input is G (the bf16 tensor-core GEMM): both gradients

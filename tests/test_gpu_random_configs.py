@@ -14,7 +14,8 @@ import pytest
 import torch
 
 from gpu_common import (TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound, assert_grad_close,
-                        bf16_operand_bounds, check_lion, gsq, mask_sign_grad_bounds)
+                        bf16_criterion, bf16_operand_bounds, check_lion, gsq,
+                        mask_sign_grad_bounds)
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 
@@ -112,6 +113,8 @@ def test_random_config(i):
             rows = slice(e * w.rows, (e + 1) * w.rows)
             assert_gemm_bound(Gg[rows], Dg[rows], Hg[e], f"G expert {e}")
         assert np.all(np.abs(Gg - res.G) <= gb), "G"
+        bf16_criterion(Gg, res.G, gb, f"case {i} ({w.name}, {w.experts}x{w.rows}x{w.cols}, "
+                                      f"calib {w.calib})")
         if w.param == "mask_sign":
             bl, bs = mask_sign_grad_bounds(res, case.prob, tau, kappa, TOL_BF16, gb)
             assert np.all(np.abs(got_l - res.d_logits) <= bl * 1.0001 + 1e-30), "dL/dlogits"

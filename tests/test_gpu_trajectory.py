@@ -38,9 +38,12 @@ from paper_2604_18556_gb300 import configs as C
 pytestmark = pytest.mark.gpu
 
 # Per-step fraction of logit entries whose Lion sign may differ between the fp32
-# GPU path and the float64 oracle (|c| below the contraction's rounding), and
-# between the bf16 tensor-core path and the oracle (|c| below G's 2e-2 tolerance).
-FLIP_PER_STEP = {"f32": 1e-4, "bf16": 1e-3}
+# GPU path and the float64 oracle (|c| below the fp32 contraction's rounding, about
+# C 2^-24 of sum |d h|), and between the bf16 tensor-core path and the oracle (|c|
+# below G's 2e-2 tolerance).  Measured on GB300: 1e-7 to 5e-7 per step on the four
+# fp32 schedules, 3e-4 per step on the bf16 path; the allowances are ten and three
+# times the largest of those.
+FLIP_PER_STEP = {"f32": 5e-6, "bf16": 1e-3}
 
 
 def _sample_rows(w, k):

@@ -118,11 +118,16 @@ __device__ __forceinline__ void bwd_quad(const EwParams& P, const float (&q)[kMa
     const float2 dj = make_float2(round_d(dd.x, P.d_bf16), round_d(dd.y, P.d_bf16));
     loss2 = fma2(mul2(f2(0.5f), dj), Gq[pr], loss2);
     ds2 = fma2(Gq[pr], wt, ds2);
-    const float2 A = mul2(f2(P.kappa_over_tau * s), Gq[pr]);
+    float2 A = mul2(f2(P.kappa_over_tau * s), Gq[pr]);
+    if (Rx::kScaled) A = mul2(A, rx.dscale());
+    // Lion mixes (1 - b1) and (1 - b2) of each gradient into c and the momentum:
+    // both factors ride on A, one product per pair instead of one per logit
+    const float2 A1 = mul2(A, f2(1.0f - P.b1)), A2 = mul2(A, f2(1.0f - P.b2));
 #pragma unroll
     for (int k = 0; k < K; ++k) {
       // dL/dl_k = (kappa/tau) G s dw~/dl_k
-      float2 dl = mul2(A, rx.dsoft(k));
+      const float2 dk = rx.dsoft(k);
+      float2 dl = mul2(A, dk);
       if (kAcc) {  // gradient accumulation: (this micro-batch + earlier ones) * scale
         const float2 a = reinterpret_cast<const float2*>(P.acc_in_l + k * P.n)[2 * qc + pr];
         dl = mul2(add2(dl, a), f2(P.acc_scale));
@@ -134,10 +139,12 @@ __device__ __forceinline__ void bwd_quad(const EwParams& P, const float (&q)[kMa
         // Lion, decoupled decay: c = b1 m + (1-b1) g; l <- l - lr wd l - lr sign(c);
         // m <- b2 m + (1-b2) g.  The decay is one fma on l (no rounded 1 - lr wd).
         const float2 mo = make_float2(m[k][2 * pr], m[k][2 * pr + 1]);
-        const float2 c = fma2(f2(P.b1), mo, mul2(f2(1.0f - P.b1), dl));
+        const float2 c = kAcc ? fma2(f2(P.b1), mo, mul2(f2(1.0f - P.b1), dl))
+                              : fma2(f2(P.b1), mo, mul2(A1, dk));
         const float2 ln = add2(fma2(f2(-P.lrwd_l), l2[k], l2[k]),
                                make_float2(-lr_sign(P.lr_l, c.x), -lr_sign(P.lr_l, c.y)));
-        const float2 mn = fma2(f2(P.b2), mo, mul2(f2(1.0f - P.b2), dl));
+        const float2 mn = kAcc ? fma2(f2(P.b2), mo, mul2(f2(1.0f - P.b2), dl))
+                               : fma2(f2(P.b2), mo, mul2(A2, dk));
         l[k][2 * pr] = ln.x; l[k][2 * pr + 1] = ln.y;
         m[k][2 * pr] = mn.x; m[k][2 * pr + 1] = mn.y;
       }

@@ -1,4 +1,4 @@
-// Device code shared by the elementwise kernels and the fused step kernel:
+// Device code shared by the forward and backward elementwise kernels:
 // counter-based Gumbel / logistic noise (Philox4x32-10), packed fp32 pair
 // arithmetic, the tempered softmax of a categorical relaxation and the binary
 // mask x sign relaxation, with their Jacobians (App. B).  Internal linkage:
@@ -75,8 +75,8 @@ __device__ __forceinline__ float2 exp2_2(float2 a) { return make_float2(fast_exp
 // the bits of u moves the exponent boundary to sqrt(2) (the integer-offset
 // reduction of fdlibm-style logf).  Then log2 m = (2 / ln 2) atanh(y),
 // y = (m - 1)/(m + 1), by the odd series 2(y + y^3/3 + y^5/5 + ...)
-// (Abramowitz & Stegun 4.1.27); |y| <= 0.1716, so terms through y^9 leave a
-// relative remainder below 2e-9.
+// (Abramowitz & Stegun 4.1.27); |y| <= 0.1716, so terms through y^7 leave a
+// relative remainder below y^8/9 = 8.3e-8 (under 1.5 ulp of fp32).
 // Arithmetic right shift by 23 of one 32-bit lane.  Written in PTX: with
 // nvcc 13.0 for sm_103a the C++ form of the two lanes' shifts below was
 // combined into one operation on the register pair that corrupted lane x.
@@ -88,7 +88,7 @@ __device__ __forceinline__ int sar23(uint32_t x) {
 
 __device__ __forceinline__ float2 log2_unit2(float2 u) {
   constexpr float c1 = 2.8853900817779268f;  // 2 / ln 2
-  constexpr float c3 = c1 / 3.0f, c5 = c1 / 5.0f, c7 = c1 / 7.0f, c9 = c1 / 9.0f;
+  constexpr float c3 = c1 / 3.0f, c5 = c1 / 5.0f, c7 = c1 / 7.0f;
   const uint32_t b0 = __float_as_uint(u.x), b1 = __float_as_uint(u.y);
   const int e0 = sar23(b0 - 0x3F3504F3u);
   const int e1 = sar23(b1 - 0x3F3504F3u);
@@ -96,8 +96,7 @@ __device__ __forceinline__ float2 log2_unit2(float2 u) {
                                __uint_as_float(b1 + static_cast<uint32_t>(e1) * 0xFF800000u));
   const float2 y = mul2(add2(m, f2(-1.0f)), rcp2(add2(m, f2(1.0f))));
   const float2 y2 = mul2(y, y);
-  float2 poly = fma2(y2, f2(c9), f2(c7));
-  poly = fma2(y2, poly, f2(c5));
+  float2 poly = fma2(y2, f2(c7), f2(c5));
   poly = fma2(y2, poly, f2(c3));
   poly = fma2(y2, poly, f2(c1));
   return fma2(y, poly, make_float2(static_cast<float>(e0), static_cast<float>(e1)));
@@ -142,13 +141,6 @@ __device__ __forceinline__ void draw_noise_pair(const PhiloxKeys& keys, uint32_t
   }
 }
 
-// Noise of weights i0 (even) and i0 + 1 (the elementwise kernels' pairs).
-template <int K>
-__device__ __forceinline__ void draw_noise2(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
-                                            int noise, float2 (&h)[K]) {
-  draw_noise_pair<K>(keys, t, i0, i0 + 1, noise, h);
-}
-
 // Level value of every logit for two weights.  Full parameterisation: the grid
 // (the same for every weight).  Local shift (§3.2): logit d of a weight with
 // initial index j0 stands for grid[clip(j0 + d - 2, 0, nlev - 1)]; the grid is
@@ -190,12 +182,14 @@ struct Levels2<K, true> {
 // Tempered softmax over the levels and the soft value (Alg. 1), two weights:
 //   p_k = exp((kappa l_k + g_k)/tau) / sum_j (...),  w~ = sum_k p_k q_k,
 // evaluated as p_k = 2^((z'_k - z'_max)/tau) / sum_j 2^(...) with z' from the
-// draw above (kappa_log2 = kappa log2 e).  w~ is carried as q_m + delta,
+// draw above (kappa_log2 = kappa log2 e); the numerators and 1/sum are kept
+// apart (the backward folds 1/sum into its per-weight factor).  w~ is carried as q_m + delta,
 // delta = sum_j p_j (q_j - q_m), m = argmax z', so q_k - w~ = (q_k - q_m) - delta
 // keeps full relative accuracy when p is nearly one-hot.
 template <int K>
 struct Soft2 {
-  float2 p[K];
+  float2 p[K];   // 2^((z'_k - z'_max)/tau): p_k before the division by their sum
+  float2 inv;    // 1 / sum
   float2 qm;
   float2 delta;
 };
@@ -228,8 +222,7 @@ __device__ __forceinline__ void relax2(const float2 (&l)[K], const float2 (&h)[K
     delta = fma2(s.p[k], add2(qv[k], neg2(qm)), delta);
   }
   const float2 inv = rcp2(sum);
-#pragma unroll
-  for (int k = 0; k < K; ++k) s.p[k] = mul2(s.p[k], inv);
+  s.inv = inv;
   s.qm = qm;
   s.delta = mul2(delta, inv);
 }
@@ -274,36 +267,36 @@ __device__ __forceinline__ float lr_sign(float lr, float c) {
 //   L             logits per weight (planes of the logit tensors)
 //   noise(...)    the step's draws for the pair, in log2 units
 //   relax(...)    w~ of the pair; keeps what dsoft() needs
-//   dsoft(k)      dw~/dl_k divided by kappa/tau
+//   dsoft(k)      dw~/dl_k divided by kappa/tau, times 1/dscale()
+//   kScaled       whether dscale() is not 1
 //   value(...)    w~ only (forward)
 // ---------------------------------------------------------------------------
 // Categorical GS over the K grid levels (Alg. 1), or over 5 local shifts.
 template <int K, bool kShift>
 struct CatRelax {
   static constexpr int L = K;
+  static constexpr bool kScaled = true;
   Levels2<K, kShift> qv;
   Soft2<K> sm;
   __device__ __forceinline__ CatRelax(const float (&q)[kMaxLevels], const float* sgrid, int nlev,
                                       uint32_t ja, uint32_t jb)
       : qv(q, sgrid, nlev, ja, jb) {}
+  // weights i0 (even) and i0 + 1
   __device__ static __forceinline__ void noise(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
                                                int on, float2 (&h)[L]) {
-    draw_noise2<K>(keys, t, i0, on, h);
-  }
-  // weights ia (row r) and ib (row r + 1) of one column (the fused step kernel)
-  __device__ static __forceinline__ void noise_rows(const PhiloxKeys& keys, uint32_t t, uint64_t ia,
-                                                    uint64_t ib, int on, float2 (&h)[L]) {
-    draw_noise_pair<K>(keys, t, ia, ib, on, h);
+    draw_noise_pair<K>(keys, t, i0, i0 + 1, on, h);
   }
   __device__ __forceinline__ float2 relax(const float2 (&l)[L], const float2 (&h)[L],
                                           float kappa_log2, float inv_tau) {
     relax2<K>(l, h, kappa_log2, inv_tau, qv, sm);
     return add2(sm.qm, sm.delta);
   }
-  // softmax Jacobian (App. B): dw~/dl_k = (kappa/tau) p_k (q_k - w~)
+  // softmax Jacobian (App. B): dw~/dl_k = (kappa/tau) p_k (q_k - w~), here with the
+  // numerator of p_k; dscale() is the 1/sum that completes it
   __device__ __forceinline__ float2 dsoft(int k) const {
     return mul2(sm.p[k], add2(add2(qv[k], neg2(sm.qm)), neg2(sm.delta)));
   }
+  __device__ __forceinline__ float2 dscale() const { return sm.inv; }
   __device__ __forceinline__ float2 value(const float2 (&l)[L], const float2 (&h)[L],
                                           float kappa_log2, float inv_tau) const {
     return soft_value2<K>(l, h, kappa_log2, inv_tau, qv);
@@ -339,31 +332,6 @@ __device__ __forceinline__ void draw_logistic2(const PhiloxKeys& keys, uint32_t 
   logistic_from_words2(a.x, a.z, a.y, a.w, h);
 }
 
-// Logistic draws of the same weights as draw_logistic2 for two weights of one
-// column in rows r and r + 1 (flat indices ia, ib = ia + C), with lanes holding
-// consecutive columns and the lane parity equal to the column parity (C even).
-// A block serves a column pair (c even, c + 1): the even lane computes the block
-// of row r, the odd lane that of row r + 1, and each hands its partner the two
-// words of the partner's column.  Every lane of the warp must call it.
-__device__ __forceinline__ void draw_logistic_rows(const PhiloxKeys& keys, uint32_t t, uint64_t ia,
-                                                   uint64_t ib, int on, float2 (&h)[2]) {
-  if (!on) {
-    h[0] = h[1] = f2(0.0f);
-    return;
-  }
-  const bool odd = (ia & 1u) != 0;
-  const uint64_t base = odd ? ib - 1 : ia;  // block counter: the even column of the pair
-  const uint4 a = philox4x32_10(static_cast<uint32_t>(base), static_cast<uint32_t>(base >> 32), t,
-                                0u, keys);
-  // even lane: keeps words 0, 1 (its own column, row r), sends 2, 3 (odd column, row r);
-  // odd lane: keeps words 2, 3 (its own column, row r + 1), sends 0, 1 (even column, row r + 1)
-  const uint32_t s0 = odd ? a.x : a.z, s1 = odd ? a.y : a.w;
-  const uint32_t r0 = __shfl_xor_sync(0xffffffffu, s0, 1), r1 = __shfl_xor_sync(0xffffffffu, s1, 1);
-  const uint32_t mr = odd ? r0 : a.x, br = odd ? r1 : a.y;      // row r: mask, sign words
-  const uint32_t mr1 = odd ? a.z : r0, br1 = odd ? a.w : r1;    // row r + 1
-  logistic_from_words2(mr, mr1, br, br1, h);
-}
-
 // Ternary mask x sign (§3.1, Alg. 2): w~ = a m~ b~ on the grid {-a, 0, a}, with
 // m~ = GS({0,1}, (-l_m, l_m)) and b~ = GS({-1,1}, (-l_b, l_b)); each binary GS
 // is a sigmoid of the noisy logit 2l (§3 notation paragraph):
@@ -373,6 +341,7 @@ __device__ __forceinline__ void draw_logistic_rows(const PhiloxKeys& keys, uint3
 // dm~/dl_m = 2 (kappa/tau) p0 p1, db~/dl_b = 4 (kappa/tau) p0 p1.
 struct MaskSignRelax {
   static constexpr int L = 2;
+  static constexpr bool kScaled = false;
   float a;
   float2 mt, bt, gm, gb;
   __device__ __forceinline__ MaskSignRelax(const float (&q)[kMaxLevels], const float*, int, uint32_t,
@@ -381,10 +350,6 @@ struct MaskSignRelax {
   __device__ static __forceinline__ void noise(const PhiloxKeys& keys, uint32_t t, uint64_t i0,
                                                int on, float2 (&h)[L]) {
     draw_logistic2(keys, t, i0, on, h);
-  }
-  __device__ static __forceinline__ void noise_rows(const PhiloxKeys& keys, uint32_t t, uint64_t ia,
-                                                    uint64_t ib, int on, float2 (&h)[L]) {
-    draw_logistic_rows(keys, t, ia, ib, on, h);
   }
   struct Bin {
     float2 hi, lo, y;   // max(p0,p1), min(p0,p1), y
@@ -417,6 +382,7 @@ struct MaskSignRelax {
   __device__ __forceinline__ float2 dsoft(int k) const {
     return k == 0 ? mul2(f2(a), mul2(bt, gm)) : mul2(f2(a), mul2(mt, gb));
   }
+  __device__ __forceinline__ float2 dscale() const { return f2(1.0f); }
   __device__ __forceinline__ float2 value(const float2 (&l)[L], const float2 (&h)[L],
                                           float kappa_log2, float inv_tau) const {
     const Bin m = binary(l[0], h[0], kappa_log2, inv_tau);

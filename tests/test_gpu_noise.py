@@ -25,18 +25,19 @@ SEED = 0x0123456789ABCDEF    # both key words nonzero
 TAU = 1e-6
 
 
-def _layer(grid, param):
+def _layer(grid, param, rows=R, index_offset=0):
     g = gsq()
     torch.manual_seed(3)
-    W = (0.02 * torch.randn(1, R, C, device="cuda")).bfloat16()
+    W = (0.02 * torch.randn(1, rows, C, device="cuda")).bfloat16()
     H = torch.zeros(1, C, C, device="cuda")
-    layer = g.Layer(W, H, grid, 128, gemm="bf16", param=param, seed=SEED)
-    layer.set_tensor(g.GSQ_T_SCALES, torch.ones(R * C // 128, device="cuda"))
+    layer = g.Layer(W, H, grid, 128, gemm="bf16", param=param, seed=SEED,
+                    index_offset=index_offset)
+    layer.set_tensor(g.GSQ_T_SCALES, torch.ones(rows * C // 128, device="cuda"))
     return layer
 
 
-def _soft_values(layer, t):
-    what = torch.empty(R * C, device="cuda")
+def _soft_values(layer, t, rows=R):
+    what = torch.empty(rows * C, device="cuda")
     layer.forward(t, TAU, 0.0, what=what)
     torch.cuda.synchronize()
     return what.cpu().numpy().astype(np.float64)
@@ -79,3 +80,32 @@ def test_logistic_draw_signs_match_the_oracle_words(t):
     assert np.array_equal(code[ok].astype(np.int64), expect[ok]), \
         int(np.sum(code[ok].astype(np.int64) != expect[ok]))
     assert (~ok).mean() < 1e-3, (~ok).mean()
+
+
+ROWS_OFF = 256                     # 1,048,576 weights per shard
+N_OFF = ROWS_OFF * C
+
+
+@pytest.mark.parametrize("index_offset", [(1 << 32) + 5 * N_OFF, (1 << 32) - N_OFF // 2 - 4096,
+                                          (3 << 32) - 12 * C])
+def test_largest_gumbel_draw_of_a_shard_far_into_the_counter_space(index_offset):
+    """A shard whose flat indices have a nonzero high word, and shards whose indices
+    cross a multiple of 2^32 (the counter's high word changes inside the launch):
+    every weight's draw must still be the oracle's for its whole-layer index."""
+    K = 8
+    t = 4242
+    layer = _layer(tuple(float(k) for k in range(K)), "full", rows=ROWS_OFF,
+                   index_offset=index_offset)
+    v = _soft_values(layer, t, rows=ROWS_OFF)
+    layer.close()
+    code = np.rint(v)
+    ok = np.abs(v - code) < 1e-6
+    idx = np.uint64(index_offset) + np.arange(N_OFF, dtype=np.uint64)
+    j = (P.level_words(SEED, t, idx, K) & np.uint32(0x7FFFFF)).astype(np.int64)
+    top = j.max(axis=0)
+    expect = j.argmax(axis=0)
+    tie = (j == top[None]).sum(axis=0) > 1
+    keep = ok & ~tie
+    assert np.array_equal(code[keep].astype(np.int64), expect[keep]), \
+        int(np.sum(code[keep].astype(np.int64) != expect[keep]))
+    assert (~keep).mean() < 1e-3, (~keep).mean()

@@ -529,6 +529,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           bulk_commit();
         }
         ++chunks;
+        // Pace the drain over the next tile's MMAs: drained back to back, the staging
+        // writes and store reads of a whole accumulator slowed the tensor pipe
+        // (measured on GB300, 4096^3: 88.4 us back to back, 87.2 us with 600 ns
+        // between chunks, 87.7 us with 1.5 us).  Not after this CTA's last tile.
+        if (tile + npairs < tiles) __nanosleep(600);
       }
       tc_fence_before();
       __syncwarp();

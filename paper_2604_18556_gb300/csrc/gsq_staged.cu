@@ -24,9 +24,9 @@ namespace {
 // The last warp to finish reading a stage (a shared counter) issues the copies
 // of the block's tile two ahead into it, so no warp waits for another.  A
 // partial last tile is read with direct loads by the block whose turn it is.
-// Logit momenta are staged for L <= 5 logits, where two stages of two resident
-// blocks fit in shared memory; otherwise they are loaded directly at the top of
-// the iteration and arrive while the noise is drawn.  Stores stay direct.
+// The plan decides which streams besides the logits are staged (plan 3, the
+// default up to 4 logits, loads the logit momenta directly: they arrive while
+// the noise is drawn).  Stores stay direct.
 // Every wait is bounded (2 s of %globaltimer); on expiry the block records an
 // error code, waits (bounded) for its own copies in flight and returns.
 // ---------------------------------------------------------------------------

@@ -618,8 +618,13 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   }
   // CTA pairs by default (at the same tile width measured 1-4% faster than single CTAs on the 4096 x 4096,
   // 4096 x 14336 and 64-expert layers); GSQ_GEMM_PAIR=0 selects single CTAs
+  // (1: pairs or clusters of two pairs by the wave rule of tc_gemm_cluster_mode);
+  // GSQ_GEMM_PAIR=1 forces plain pairs, =2 clusters of two pairs
   L->gemm_pair = 1;
-  if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) L->gemm_pair = std::atoi(gp) == 0 ? 0 : 1;
+  if (const char* gp = std::getenv("GSQ_GEMM_PAIR")) {
+    const int v = std::atoi(gp);
+    L->gemm_pair = v == 0 ? 0 : (v == 2 ? 2 : 3);
+  }
   // Test hook for the bounded device-side waits: GSQ_TEST_STALL=backward makes the staged
   // backward skip one stage fill, =gemm makes the tensor-core GEMM skip its first k-block;
   // the waits on it give up after 2 s and gsq_sync_status reports GSQ_ERR_TIMEOUT.
@@ -1171,7 +1176,11 @@ const char* gsq_kernel_name(gsq_layer* L, int32_t kind) {
   if (!valid(L)) return nullptr;
   if (kind == GSQ_K_GEMM) {
     if (!L->shape.d_bf16) return "k_simt_gemm";
-    return L->gemm_pair ? "k_tc_gemm_pair" : "k_tc_gemm";
+    int mode = L->gemm_pair;
+    if (mode == 1)
+      mode = tc_gemm_cluster_mode(static_cast<int>(L->shape.E), static_cast<int>(L->shape.R),
+                                  static_cast<int>(L->shape.C), L->tile_n, L->num_sms);
+    return mode == 2 ? "k_tc_gemm_quad" : (mode ? "k_tc_gemm_pair" : "k_tc_gemm");
   }
   if (kind == GSQ_K_BACKWARD) {
     return L->grid_bwd_staged > 0 ? "k_backward_staged" : "k_backward";

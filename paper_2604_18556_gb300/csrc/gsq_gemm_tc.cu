@@ -558,6 +558,242 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicExch(&args.flags->error, 0x7C04u);
 }
 
+// ---------------------------------------------------------------------------
+// Clusters of two CTA pairs (four CTAs) on the same column tile and adjacent
+// 256-row tiles: pair p of the cluster (cluster ranks 2p, 2p + 1) computes row
+// tile 2 mc + p, both pairs column tile n.  Both pairs need the same BN rows of
+// B, so each CTA loads a quarter of them (BN/4 rows) and multicasts it to the
+// CTA of the other pair that holds the same half: CTA (p, q) loads rows
+// q BN/2 + p BN/4 .. + BN/4 into both CTAs (0, q) and (1, q) at the matching
+// offset of their B half.  A (each pair's own rows) is loaded as in
+// k_tc_gemm_pair.  An SM then requests 16 KiB + BN/4 x 128 B per k-block from
+// L2 instead of 16 KiB + BN/2 x 128 B.  Barriers: each pair's full barrier (in
+// its leader) counts the bytes landing in both its CTAs, whichever CTA issued
+// them; a stage is free again only when both pairs' MMAs have read it (the
+// empty barriers take one commit from each pair's leader, multicast to all
+// four CTAs); accumulator barriers stay per pair.  Waits are bounded as in
+// k_tc_gemm_pair; a CTA that gives up records 0x7C05.
+// ---------------------------------------------------------------------------
+template <int BN>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    k_tc_gemm_quad(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmBq,
+                   const __grid_constant__ CUtensorMap tmO, const TcArgs args) {
+  using Cfg = Tc2Cfg<BN>;
+  constexpr int STAGES = Cfg::kStages;
+  constexpr int STAGE_BYTES = Cfg::kStageBytes;
+  constexpr int BQ = BN / 4;  // rows of B each CTA loads and multicasts
+  static_assert(BQ % 8 == 0, "B quarters must be whole 8-row swizzle atoms");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* epi = smem + STAGES * STAGE_BYTES;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(epi + Cfg::kEpiBytes);
+  uint64_t* empty_bar = full_bar + STAGES;
+  uint64_t* tfull_bar = empty_bar + STAGES;
+  uint64_t* tempty_bar = tfull_bar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t crank = cluster_ctarank();   // 0..3
+  const uint32_t pp = crank >> 1;             // pair within the cluster
+  const uint32_t q = crank & 1u;              // CTA within the pair (0: leader)
+  const uint32_t leader = crank & ~1u;
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << (2 * pp));
+  const uint16_t half_mask = static_cast<uint16_t>((1u << q) | (1u << (q + 2)));
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar + s, 1);
+      mbar_init(empty_bar + s, 2);  // one commit from each pair's leader
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar + a, 1);
+      mbar_init(tempty_bar + a, 8);  // one arrival per epilogue warp of the pair
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmBq)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmO)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(Cfg::kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // every CTA's barriers exist before any copy or arrival reaches them
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int Mt = (args.M + TC2_BM - 1) / TC2_BM;
+  const int Mt2 = (Mt + 1) / 2;  // row-tile pairs per expert
+  const int Nt = (args.N + BN - 1) / BN;
+  const int KB = (args.K + TC_BK - 1) / TC_BK;
+  const int tiles = args.E * Mt2 * Nt;  // cluster tiles
+  const int cl = blockIdx.x >> 2, ncl = gridDim.x >> 2;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (every CTA) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      const uint32_t fb_base = mapa_shared(smem_u32(full_bar), leader);
+      for (int tile = cl; ok && tile < tiles; tile += ncl) {
+        int e, mc, n;
+        tile_coords(tile, Mt2, Nt, args.group_n, e, mc, n);
+        const int m = 2 * mc + static_cast<int>(pp);
+        const int arow = e * args.M + m * TC2_BM + static_cast<int>(q) * TC_BM;
+        const int brow = e * args.N + n * BN + static_cast<int>(q) * Cfg::kBHalf +
+                         static_cast<int>(pp) * BQ;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(empty_bar + stage, phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + stage * STAGE_BYTES;
+          uint8_t* sbq = sa + TC_A_BYTES + pp * (BQ * TC_BK * 2);
+          const uint32_t fb = fb_base + static_cast<uint32_t>(stage * sizeof(uint64_t));
+          if (!(args.stall && tile == cl && kb == 0)) {
+            if (q == 0) mbar_expect_tx(full_bar + stage, 2 * STAGE_BYTES);
+            tma_load_2d_pair(sa, &tmA, fb, kb * TC_BK, arow);
+            tma_load_2d_pair_mc(sbq, &tmBq, fb, kb * TC_BK, brow, half_mask);
+          }
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        const unsigned long long t0 = global_ns();
+        while (global_ns() - t0 < 200000ull) __nanosleep(1000);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && q == 0) {
+      // ---------------- MMA issuer (each pair's leader) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = cl; ok && tile < tiles; tile += ncl) {
+        if (!mbar_wait(tempty_bar + acc, acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride);
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(full_bar + stage, phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint64_t da = sw128_desc(sa);
+          const uint64_t db = sw128_desc(sa + TC_A_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, Cfg::kIdesc, (kb | k) != 0 ? 1u : 0u);
+          umma_commit_mask(empty_bar + stage, 0xF);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit_mask(tfull_bar + acc, pair_mask);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 of every CTA), as in k_tc_gemm_pair ------------
+    const int quarter = warp & 3;
+    uint8_t* wbuf = epi + quarter * 2 * Cfg::kEpiChunk;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    int chunks = 0;
+    const uint32_t te_base = mapa_shared(smem_u32(tempty_bar), leader);
+    for (int tile = cl; tile < tiles; tile += ncl) {
+      if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
+      tc_fence_after();
+      int e, mc, n;
+      tile_coords(tile, Mt2, Nt, args.group_n, e, mc, n);
+      const int m = 2 * mc + static_cast<int>(pp);
+      const int row0 = m * TC2_BM + static_cast<int>(q) * TC_BM + quarter * 32;
+      const int col0 = n * BN;
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride) +
+                             (static_cast<uint32_t>(quarter * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld32(taddr + c, v);
+        if (m >= Mt || row0 >= args.M || col0 + c >= args.N) continue;  // nothing of it is stored
+        uint8_t* buf = wbuf + (chunks & 1) * Cfg::kEpiChunk;
+        if (chunks >= 2) {
+          if (lane == 0) bulk_wait_read_1();
+          __syncwarp();
+        }
+        if (args.out_bf16) {
+          uint8_t* rowp = buf + lane * 64;
+          const int sw = (lane >> 1) & 3;
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            uint32_t w[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const __nv_bfloat162 b2 = __floats2bfloat162_rn(args.alpha * v[8 * p + 2 * h],
+                                                              args.alpha * v[8 * p + 2 * h + 1]);
+              w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+            }
+            *reinterpret_cast<uint4*>(rowp + 16 * (p ^ sw)) = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        } else {
+          uint8_t* rowp = buf + lane * 128;
+          const int sw = lane & 7;
+#pragma unroll
+          for (int p = 0; p < 8; ++p)
+            *reinterpret_cast<float4*>(rowp + 16 * (p ^ sw)) =
+                make_float4(args.alpha * v[4 * p], args.alpha * v[4 * p + 1],
+                            args.alpha * v[4 * p + 2], args.alpha * v[4 * p + 3]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tmO, buf, col0 + c, row0, e);
+          bulk_commit();
+        }
+        ++chunks;
+        if (tile + ncl < tiles) __nanosleep(600);  // pace the drain (k_tc_gemm_pair)
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(te_base + static_cast<uint32_t>(acc * sizeof(uint64_t)));
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while the cluster's MMAs, copies or arrivals may touch it
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(Cfg::kTmemCols));
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(&args.flags->error, 0x7C05u);
+}
+
 bool tc_supported_impl(int device) {
   cudaDeviceProp prop;
   if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return false;
@@ -657,6 +893,61 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+template <int BN>
+cudaError_t launch_tc_gemm_quad_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
+  using Cfg = Tc2Cfg<BN>;
+  cudaError_t ea = cudaFuncSetAttribute(k_tc_gemm_quad<BN>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  if (ea != cudaSuccess) return ea;
+  CUtensorMap ta, tbq, to;
+  if (g.K % 8 != 0 || g.N % 4 != 0) return cudaErrorInvalidValue;
+  if (g.out_bf16 && g.N % 8 != 0) return cudaErrorInvalidValue;
+  if ((reinterpret_cast<uintptr_t>(g.out) & 15) != 0) return cudaErrorInvalidValue;
+  if (!encode_kmajor_bf16(&ta, g.A, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.M, TC_BM) ||
+      !encode_kmajor_bf16(&tbq, g.B, static_cast<uint64_t>(g.K),
+                          static_cast<uint64_t>(g.E) * g.N, BN / 4) ||
+      !encode_out_map(&to, g.out, g.E, g.M, g.N, g.out_bf16))
+    return cudaErrorInvalidValue;
+  TcArgs a;
+  a.E = g.E;
+  a.M = g.M;
+  a.N = g.N;
+  a.K = g.K;
+  a.group_n = g.group_n > 0 ? g.group_n : (g.N + BN - 1) / BN;
+  a.out = g.out;
+  a.out_bf16 = g.out_bf16;
+  a.alpha = g.alpha;
+  a.flags = g.flags;
+  a.stall = g.stall;
+  const int Mt = (g.M + TC2_BM - 1) / TC2_BM, Nt = (g.N + BN - 1) / BN;
+  const int64_t tiles = static_cast<int64_t>(g.E) * ((Mt + 1) / 2) * Nt;
+  int clusters = num_sms / 4;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 4;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(TC_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(4 * clusters, 1, 1);
+  int max_clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&max_clusters, k_tc_gemm_quad<BN>, &cfg) != cudaSuccess ||
+      max_clusters < 1) {
+    cudaGetLastError();
+    return launch_tc_gemm_pair_bn<BN>(g, num_sms, s);  // no 4-CTA cluster fits: pairs
+  }
+  if (max_clusters < clusters) clusters = max_clusters;
+  if (tiles < clusters) clusters = static_cast<int>(tiles);
+  cfg.gridDim = dim3(4 * clusters, 1, 1);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_quad<BN>, ta, tbq, to, a);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 }  // namespace
 
 bool tc_gemm_supported(int device) { return tc_supported_impl(device); }
@@ -692,8 +983,70 @@ int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair) {
   return cost(224) <= 1.1 * cost(256) ? 224 : 256;
 }
 
+namespace {
+
+// Resident clusters of `csize` CTAs of `kernel` (its shared memory attribute set), 0 on error.
+template <class Kern>
+int resident_clusters(Kern kernel, int smem, int csize, int num_sms) {
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = csize;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(TC_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(csize * (num_sms / csize), 1, 1);
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n < num_sms / csize ? n : num_sms / csize;
+}
+
+template <int BN>
+int cluster_mode_bn(int E, int M, int N, int num_sms) {
+  const int pairs = resident_clusters(k_tc_gemm_pair<BN>, Tc2Cfg<BN>::kSmemBytes, 2, num_sms);
+  const int quads = resident_clusters(k_tc_gemm_quad<BN>, Tc2Cfg<BN>::kSmemBytes, 4, num_sms);
+  if (pairs < 1 || quads < 1) return 3;
+  const int64_t mt = (M + TC2_BM - 1) / TC2_BM, nt = (N + BN - 1) / BN;
+  const int64_t pw = (static_cast<int64_t>(E) * mt * nt + pairs - 1) / pairs;
+  const int64_t qw = (static_cast<int64_t>(E) * ((mt + 1) / 2) * nt + quads - 1) / quads;
+  // Clusters read 23% less operand data per SM and ran each tile 5-8% faster on
+  // GB300, where fewer 4-CTA clusters than 76 pairs are resident: 64 experts
+  // 2048 x 7168, 200 waves against 189, 2.6% faster; 28672 x 8192, 50 against
+  // 48, 0.5-0.9% faster; 4096 x 14336, 13 against 12, 3.6% slower; 4096 x 4096,
+  // 5 against 4, 19% slower.  So clusters when they cost at most 6% more waves;
+  // a contraction of a few waves keeps the pairs.
+  if (pw < 4) return 3;
+  return static_cast<double>(qw) <= 1.06 * static_cast<double>(pw) ? 2 : 3;
+}
+
+}  // namespace
+
+int tc_gemm_cluster_mode(int E, int M, int N, int bn, int num_sms) {
+  if (num_sms < 4) return 3;
+  if (bn == 128) return cluster_mode_bn<128>(E, M, N, num_sms);
+  if (bn == 224) return cluster_mode_bn<224>(E, M, N, num_sms);
+  return cluster_mode_bn<256>(E, M, N, num_sms);
+}
+
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
   const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms, g.pair);
+  const int mode = g.pair == 1 ? tc_gemm_cluster_mode(g.E, g.M, g.N, bn, num_sms) : g.pair;
+  if (mode == 2 && num_sms >= 4) {
+    if (bn == 128) return launch_tc_gemm_quad_bn<128>(g, num_sms, s);
+    if (bn == 224) return launch_tc_gemm_quad_bn<224>(g, num_sms, s);
+    return launch_tc_gemm_quad_bn<256>(g, num_sms, s);
+  }
   if (g.pair && num_sms >= 2) {
     if (bn == 128) return launch_tc_gemm_pair_bn<128>(g, num_sms, s);
     if (bn == 224) return launch_tc_gemm_pair_bn<224>(g, num_sms, s);

@@ -232,12 +232,17 @@ struct TcGemm {
   DevFlags* flags;
   int tile_n;   // 0: choose 128 or 256 by wave balance
   int group_n;  // tile-order column group; <= 0: one group (m fastest across all columns)
-  int pair;     // 1: CTA pairs (cta_group::2, 256-row tiles over two SMs)
+  int pair;     // 0: single CTAs; 3: CTA pairs (cta_group::2, 256-row tiles over two SMs);
+                // 2: clusters of two pairs sharing B by multicast; 1: pairs or clusters of
+                // pairs, whichever tc_gemm_cluster_mode picks for the shape
   int stall;    // test hook (GSQ_TEST_STALL=gemm): the first k-block is never loaded
 };
 bool tc_gemm_supported(int device);
 
 int tc_gemm_tile_n(int E, int M, int N, int num_sms, int pair);
+// 2 (clusters of two CTA pairs) or 3 (CTA pairs) for an E x M x N contraction with
+// tiles BN wide: clusters unless their resident count costs more than 6% more waves.
+int tc_gemm_cluster_mode(int E, int M, int N, int bn, int num_sms);
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s);
 
 }  // namespace gsq

@@ -179,6 +179,30 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
       : "memory");
 }
 
+// The same arrival on the mbarrier at bar's offset in every CTA of `mask`
+// (cluster ranks), for clusters of several pairs.
+__device__ __forceinline__ void umma_commit_mask(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+      "[%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+
+// TMA 2D load of one box, written at dst's offset into the shared memory of
+// every CTA in `mask` (cluster ranks); each destination's bytes are counted on
+// the mbarrier at bar_cluster's offset in that destination's pair leader
+// (bar_cluster: this CTA's pair leader's barrier).
+__device__ __forceinline__ void tma_load_2d_pair_mc(void* dst, const CUtensorMap* map,
+                                                    uint32_t bar_cluster, int x, int y,
+                                                    uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes."
+      "multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y), "h"(mask)
+      : "memory");
+}
+
 // ---- TMA tensor stores (shared -> global), tracked as bulk groups ----------
 // Makes this thread's generic-proxy writes to shared memory visible to the
 // async proxy that a following TMA store reads through.

@@ -20,6 +20,7 @@ W = C.shrunk(C.WORKLOADS["llama8b_q_proj"], rows=999, cols=1280, tokens=2048)
 @pytest.mark.parametrize("stall,pair,code,kernel", [
     ("backward", "1", 0x7C03, "k_backward_staged"),
     ("gemm", "1", 0x7C04, "k_tc_gemm_pair"),
+    ("gemm", "2", 0x7C05, "k_tc_gemm_quad"),
     ("gemm", "0", 0x7C01, "k_tc_gemm"),
 ])
 def test_bounded_wait_reports_timeout(stall, pair, code, kernel, monkeypatch):

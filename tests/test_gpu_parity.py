@@ -280,3 +280,34 @@ def test_tc_gemm_cta_pairs(name, tile_n, monkeypatch):
         sel = rows // w.rows == e
         assert_gemm_bound(G[sel], D[sel], H[e], f"pairs, tile N = {tile_n}, expert {e}")
     assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())
+
+
+CLUSTER_CASES = dict(PAIR_CASES, **{
+    # 700 rows: three 256-row tiles, so the last cluster tile has one pair with rows
+    "q_proj_odd_tiles": C.shrunk(W["llama8b_q_proj"], rows=700, cols=1024, tokens=2048),
+})
+
+
+@pytest.mark.parametrize("tile_n", ["128", "224", "256"])
+@pytest.mark.parametrize("name", ["q_proj", "gate_proj", "moe_kquant", "q_proj_multi_wave",
+                                  "q_proj_odd_tiles"])
+def test_tc_gemm_pair_clusters(name, tile_n, monkeypatch):
+    """Clusters of two CTA pairs sharing each tile of H by TMA multicast: every tile width,
+    ragged shapes (an odd number of 256-row tiles leaves the second pair of the last
+    cluster tile without rows), several experts, against exact products of the kernel's
+    own bf16 operands, and the loss as 1/2 sum D G."""
+    monkeypatch.setenv("GSQ_GEMM_TILE_N", tile_n)
+    monkeypatch.setenv("GSQ_GEMM_PAIR", "2")
+    w = CLUSTER_CASES[name]
+    case = Case(w, gemm="bf16")
+    assert case.layer.kernel_name(gsq().GSQ_K_GEMM) == "k_tc_gemm_quad"
+    loss = torch.zeros(1, device="cuda")
+    case.layer.step(0, TAU.get(name, 0.55), 1.0, loss=loss)
+    torch.cuda.synchronize()
+    case.layer.sync_status()
+    D, H, G = case.D(), case.H_operand(), case.G()
+    rows = np.arange(w.experts * w.rows)
+    for e in range(w.experts):
+        sel = rows // w.rows == e
+        assert_gemm_bound(G[sel], D[sel], H[e], f"pair clusters, tile N = {tile_n}, expert {e}")
+    assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())

@@ -427,7 +427,7 @@ GSQ_API const char* gsq_version(void);
 
 /* Name of the kernel that gsq_step launches for the part `kind` of a
  * non-exporting step of this layer (GSQ_K_GEMM: "k_tc_gemm_pair",
- * "k_tc_gemm" or "k_simt_gemm"; GSQ_K_BACKWARD: "k_backward_staged" or
+ * "k_tc_gemm_quad" (clusters of two CTA pairs), "k_tc_gemm" or "k_simt_gemm"; GSQ_K_BACKWARD: "k_backward_staged" or
  * "k_backward"), so timings can be
  * attributed (the paper has no counterpart: a reporting aid).  Static string
  * owned by the library; NULL for an invalid handle or another kind. */

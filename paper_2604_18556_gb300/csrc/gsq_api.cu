@@ -1170,7 +1170,7 @@ gsq_status gsq_destroy(gsq_layer* L) {
 
 const char* gsq_last_error(void) { return g_last_error.c_str(); }
 
-const char* gsq_version(void) { return "0.1.0"; }
+const char* gsq_version(void) { return "0.2.0"; }
 
 const char* gsq_kernel_name(gsq_layer* L, int32_t kind) {
   if (!valid(L)) return nullptr;

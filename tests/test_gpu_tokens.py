@@ -36,7 +36,22 @@ def _batches(w, step):
 @pytest.mark.parametrize("gemm", ["f32", "bf16"])
 @pytest.mark.parametrize("name", list(CASES))
 def test_token_steps_match_oracle(name, gemm):
-    w = CASES[name]
+    _check_token_steps(CASES[name], gemm)
+
+
+@pytest.mark.parametrize("mode,kernel", [("0", "k_tc_gemm"), ("1", "k_tc_gemm_pair"),
+                                         ("2", "k_tc_gemm_quad")])
+def test_token_steps_on_every_contraction_kernel(mode, kernel, monkeypatch):
+    """Both token contractions (Y = D X^T with bf16 output, G = 2 Y X with fp32 output)
+    on single CTAs, CTA pairs and clusters of two pairs sharing operand tiles by TMA
+    multicast, against the oracle."""
+    monkeypatch.setenv("GSQ_GEMM_PAIR", mode)
+    w = dataclasses.replace(CASES["full"], rows=600)   # three 256-row tiles: a ragged cluster
+    case = _check_token_steps(w, "bf16")
+    assert case.layer.kernel_name(gsq().GSQ_K_GEMM) == kernel
+
+
+def _check_token_steps(w, gemm):
     case = Case(w, gemm=gemm)
     tol = TOL_F32 if gemm == "f32" else TOL_BF16
     rng = np.random.default_rng(5)
@@ -70,6 +85,8 @@ def test_token_steps_match_oracle(name, gemm):
                                (gpu.m_scales, st.m_scales, "scale momentum")):
                 d = np.linalg.norm(a.astype(np.float64) - b) / np.linalg.norm(b)
                 assert d <= tol, (what, d)
+    case.layer.sync_status()
+    return case
 
 
 def test_token_steps_enforce_order_and_mode():

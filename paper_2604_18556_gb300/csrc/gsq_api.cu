@@ -642,6 +642,11 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     const int v = std::atoi(gn);
     if (v >= 0 && v <= 1024) L->group_n = v;
   }
+  // An H-based layer's loss contraction has one shape: settle pairs or clusters of pairs
+  // once here rather than on every launch (token layers decide per contraction).
+  if (L->gemm_pair == 1 && sh.d_bf16 && !sh.batches)
+    L->gemm_pair = tc_gemm_cluster_mode(static_cast<int>(sh.E), static_cast<int>(sh.R),
+                                        static_cast<int>(sh.C), L->tile_n, L->num_sms);
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   DevFlags* flags = reinterpret_cast<DevFlags*>(L->ws + lay.flags);

@@ -10,7 +10,10 @@ tau annealed 1.0 -> 0.1 over 500 steps).  Prints one JSON line.
 
 The K timed steps are captured once as a CUDA graph; the graph is replayed
 until the timed window covers at least --min-window-ms, each replay (exactly K
-steps) bracketed by a synchronize, and the median replay gives ms_per_step.
+steps) bracketed by a synchronize, and the median replay gives ms_per_step.  The
+per-kernel times behind the rooflines come from a second graph of K steps with
+the library's event records around every kernel, replayed in a window of its
+own (those records slow a step by about 15 us, so they stay out of the headline).
 
 --impl reference times the CPU oracle (the plain float64 restatement of the
 method) on the host's cores: one single-threaded process per core, each
@@ -534,10 +537,12 @@ def _parallelism(w, sh, world):
             f"(rank 0 holds {part}), H replicated, no collective in the timed region")
 
 
-def _timed_replays(args, run_k_steps, stream, world, device):
+def _timed_replays(args, run_k_steps, stream, world, device, min_window_ms=None):
     """Times replays of exactly K steps, each bracketed by a barrier (N > 1) and a
-    synchronize, until the window covers args.min_window_ms.  Returns the list of
-    per-replay milliseconds (the same count on every rank)."""
+    synchronize, until the window covers min_window_ms (default args.min_window_ms).
+    Returns the list of per-replay milliseconds (the same count on every rank)."""
+    if min_window_ms is None:
+        min_window_ms = args.min_window_ms
     import torch
     import torch.distributed as dist
 
@@ -553,7 +558,7 @@ def _timed_replays(args, run_k_steps, stream, world, device):
         return e0.elapsed_time(e1)
 
     reps = [one()]
-    n = replays_for_window(max_over_ranks(reps[0], device), args.min_window_ms)
+    n = replays_for_window(max_over_ranks(reps[0], device), min_window_ms)
     for _ in range(n - 1):
         reps.append(one())
     if world > 1:
@@ -598,44 +603,69 @@ def gpu_arm(args, rank, world, local):
     layer.sync_status()
     torch.cuda.synchronize()
 
-    # The K timed steps are captured once as a CUDA graph (untimed): K distinct
-    # steps t0..t0+K-1, so a replay does exactly the work of K eager steps without
-    # host launch gaps.  The library's profiling events become event-record nodes
-    # and time the kernels of every replay (the record read at the end is the last
-    # replay's).  K is even, so the look-ahead D a replay leaves behind sits in the
-    # buffer its first step reads.
-    graph = None
-    layer.profile_enable(True)
-    layer.profile_read()
-    if not args.no_graph:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
+    # The K timed steps are captured as CUDA graphs (untimed): K distinct steps
+    # t0..t0+K-1, so a replay does exactly the work of K eager steps without host
+    # launch gaps.  Two graphs: the headline times one with nothing but the step's
+    # kernels; the per-kernel split comes from a second graph of K further steps
+    # with the library's profiling events as event-record nodes around every
+    # kernel, replayed in a window of its own (the record read at the end is the
+    # last replay's).  Those records add gaps between the kernels, so that window
+    # runs slower and its per-kernel averages over-state each kernel a little: the
+    # roofline fractions drawn from them are conservative.  K is even, so the
+    # look-ahead D a replay leaves behind sits in the buffer its first step reads.
+    def capture(t0):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
             for i in range(args.steps):
-                layer.step(t + i, sched(t + i), w.kappa, next_tau=sched(t + i + 1),
+                layer.step(t0 + i, sched(t0 + i), w.kappa, next_tau=sched(t0 + i + 1),
                            next_kappa=w.kappa, loss=loss)
-        t += args.steps
-        graph.replay()      # first replay (graph upload), untimed
+        g.replay()          # first replay (graph upload), untimed
         torch.cuda.synchronize()
+        return g
+
+    graph = graph_prof = None
+    layer.profile_enable(False)
+    if not args.no_graph:
+        graph = capture(t)
+        t += args.steps
+        layer.profile_enable(True)
+        graph_prof = capture(t)
+        t += args.steps
+        layer.profile_enable(False)
 
     state = {"t": t}
 
-    def run_k_steps():
-        if graph is not None:
-            graph.replay()
-            return
+    def eager_k_steps():
         for _ in range(args.steps):
             tt = state["t"]
             layer.step(tt, sched(tt), w.kappa, next_tau=sched(tt + 1), next_kappa=w.kappa,
                        loss=loss)
             state["t"] = tt + 1
 
+    def run_k_steps():
+        if graph is not None:
+            graph.replay()
+        else:
+            eager_k_steps()
+
+    def run_k_steps_profiled():
+        if graph_prof is not None:
+            graph_prof.replay()
+        else:
+            eager_k_steps()
+
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
     reps = _timed_replays(args, run_k_steps, stream, world, device)
-    clocks = sampler.stop()
+    if graph_prof is None:   # eager steps record their events from here on (a captured
+        layer.profile_enable(True)   # graph holds the events recorded at its capture)
+        layer.profile_read()
+    prof_reps = _timed_replays(args, run_k_steps_profiled, stream, world, device,
+                               min_window_ms=min(200.0, args.min_window_ms))
     prof = layer.profile_read()
     layer.profile_enable(False)
+    clocks = sampler.stop()
     layer.sync_status()
     ms_step = max_over_ranks(float(np.median(reps)), device) / args.steps
     value = layer_steps_per_s(ms_step)
@@ -670,9 +700,12 @@ def gpu_arm(args, rank, world, local):
                      "bound": "tensor", "achieved": gemm_tfs, "peak": tf_burst, "unit": "TFLOP/s",
                      "frac": gemm_tfs / tf_burst, "frac_of_sustained": gemm_tfs / tf_sust,
                      "flops_per_launch": flops, "avg_launch_ms": gemm_avg,
-                     "peak_source": f"{peak_src}: bf16_tflops (burst; the timed window is "
-                                    f"{sum(reps):.0f} ms of replays)"}
-    launches = (bwd_n + gemm_n + fwd_n) * (len(reps) if graph is not None else 1)
+                     "peak_source": f"{peak_src}: bf16_tflops (burst; the timed windows are "
+                                    f"{sum(reps):.0f} + {sum(prof_reps):.0f} ms of replays)"}
+    # kernels of the headline window: the profiled graph's last replay holds one replay's
+    # launches; eager steps launch a GEMM and a backward kernel per step
+    launches = ((bwd_n + gemm_n + fwd_n) * len(reps) if graph is not None
+                else 2 * args.steps * len(reps))
 
     # method diagnostics of the state after the timed steps (not timed)
     diag = layer.diagnose(sched(state["t"]), w.kappa)
@@ -695,9 +728,14 @@ def gpu_arm(args, rank, world, local):
                 "parallelism": _parallelism(whole, sh, world),
                 "timing": (f"{len(reps)} replays of one CUDA graph of the {args.steps} timed steps "
                            f"(each replay bracketed by a synchronize; median replay), "
-                           f"{sum(reps):.1f} ms timed in total") if graph is not None else
-                          f"{len(reps)} rounds of {args.steps} eager steps, median round"}),
+                           f"{sum(reps):.1f} ms timed in total; the per-kernel split from "
+                           f"{len(prof_reps)} replays of a second graph of {args.steps} steps "
+                           f"with event records around every kernel") if graph is not None else
+                          f"{len(reps)} rounds of {args.steps} eager steps, median round; the "
+                          f"per-kernel split from {len(prof_reps)} further rounds with event "
+                          f"records around every kernel"}),
             "timed_window_ms": sum(reps), "replays": len(reps),
+            "ms_per_step_with_kernel_events": float(np.median(prof_reps)) / args.steps,
             "roofline": roofline, "roofline_gemm": roofline_gemm, "clocks": clocks,
             "diagnostics": diag, "loss_last_step": loss_total,
             "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
@@ -754,8 +792,6 @@ def gpu_arm_tokens(args, rank, world, local):
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
-    layer.profile_enable(True)
-    layer.profile_read()
     state = {"t": t}
 
     def run_k_steps():
@@ -763,13 +799,19 @@ def gpu_arm_tokens(args, rank, world, local):
             one_step(layer, state["t"], Xs, loss)
             state["t"] += 1
 
+    # the headline from rounds with nothing but the step's kernels; the per-kernel
+    # split from further rounds with the library's event records around every kernel
     device = torch.device("cuda", local)
     reps = _timed_replays(args, run_k_steps, stream, world, device)
-    clocks = sampler.stop()
+    layer.profile_enable(True)
+    layer.profile_read()
+    prof_reps = _timed_replays(args, run_k_steps, stream, world, device,
+                               min_window_ms=min(200.0, args.min_window_ms))
     prof = layer.profile_read()
     layer.profile_enable(False)
+    clocks = sampler.stop()
     layer.sync_status()
-    n_timed = args.steps * len(reps)
+    n_timed = args.steps * len(prof_reps)     # steps of the profiled rounds
     ms_step = max_over_ranks(float(np.median(reps)), device) / args.steps
     value = layer_steps_per_s(ms_step)
 
@@ -793,7 +835,8 @@ def gpu_arm_tokens(args, rank, world, local):
                     "bound": "hbm", "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s",
                     "frac": bwd_gbs / hbm, "algorithmic_bytes_per_step": bytes_step,
                     "ms_per_step": bwd_ms / n_timed}
-    launches = gemm_n * 2 + bwd_n + tok_n + fwd_n
+    # kernels of the headline rounds (a GEMM profile entry covers both token GEMMs)
+    launches = (gemm_n * 2 + bwd_n + tok_n + fwd_n) * len(reps) // max(len(prof_reps), 1)
 
     e2e = None
     if not args.no_e2e:
@@ -809,7 +852,12 @@ def gpu_arm_tokens(args, rank, world, local):
             "dtype": "f32 (tensor-core GEMMs bf16 in, f32 acc)",
             "data": "synthetic (seeded; Llama-3.1-8B q_proj shape, per-step token batches)",
             "timed_window_ms": sum(reps), "replays": len(reps),
+            "ms_per_step_with_kernel_events": float(np.median(prof_reps)) / args.steps,
             "config": _config(whole, {"parallelism": _parallelism(whole, sh, world),
+                                  "timing": f"{len(reps)} rounds of {args.steps} eager steps, "
+                                            f"median round; the per-kernel split from "
+                                            f"{len(prof_reps)} further rounds with event records "
+                                            f"around every kernel",
                                   "micro_batches": w.micro, "tokens_per_micro_batch": w.tokens,
                                   "l2": "token batches of "
                                         f"{w.tokens * w.cols * 4 / 2**20:.0f} MiB each, larger "

@@ -273,6 +273,7 @@ struct gsq_layer {
   int group_n; // column group of the GEMM's tile order
   int gemm_pair;      // 1: the loss GEMM runs on CTA pairs (cta_group::2)
   int test_stall;     // test hook (GSQ_TEST_STALL): 1 staged backward, 2 tensor-core GEMM
+  bool pdl;           // step kernels launched as programmatic dependents of the one before
   bool g_valid; // the G buffer holds the last step's G
   size_t d_cur; // offset of the buffer holding the latest D written
   // pending forward (D valid for these arguments)
@@ -455,6 +456,7 @@ gsq_status launch_gemm(gsq_layer* L, size_t doff, cudaStream_t s) {
     g.tile_n = L->tile_n;
     g.group_n = L->group_n;
     g.pair = L->gemm_pair;
+    g.pdl = L->pdl ? 1 : 0;
     e = launch_tc_gemm(g, L->num_sms, s);
   } else {
     SimtGemm g;
@@ -637,6 +639,11 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
     const int v = std::atoi(tn);
     if (v == 128 || v == 224 || v == 256) L->tile_n = v;
   }
+  // The step's tensor-core GEMMs and backward kernels are launched as programmatic
+  // dependents: each is scheduled while the kernel before it drains and waits for it
+  // (griddepcontrol) before touching memory. GSQ_PDL=0 launches them plainly.
+  L->pdl = true;
+  if (const char* pv = std::getenv("GSQ_PDL")) L->pdl = std::atoi(pv) != 0;
   L->group_n = kGemmGroupN;
   if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)
     const int v = std::atoi(gn);
@@ -775,8 +782,8 @@ gsq_status gsq_step(gsq_layer* L, uint64_t step, float tau, float kappa, float n
   cudaError_t e;
   prof_begin(L, GSQ_K_BACKWARD, s, slot);
   e = (!export_mode && L->grid_bwd_staged > 0)
-          ? launch_backward_staged(p, L->grid_bwd_staged, L->staged_plan, s)
-          : launch_backward(p, L->grid_bwd, s);
+          ? launch_backward_staged(p, L->grid_bwd_staged, L->staged_plan, s, L->pdl)
+          : launch_backward(p, L->grid_bwd, s, L->pdl);
   prof_end(L, slot, s);
   if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
   L->g_valid = true;
@@ -843,6 +850,7 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
     g.tile_n = 0;
     g.group_n = L->group_n;
     g.pair = L->gemm_pair;
+    g.pdl = L->pdl ? 1 : 0;
     g.E = E;
     if (e == cudaSuccess) {  // Y[e] = D[e] X[e]^T  (N = T, K = C), bf16 out
       g.M = R; g.N = T; g.K = C;
@@ -909,7 +917,7 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
   }
   p.loss_out = loss_dev;
   prof_begin(L, GSQ_K_BACKWARD, s, slot);
-  e = launch_backward(p, L->grid_bwd, s);
+  e = launch_backward(p, L->grid_bwd, s, L->pdl);
   prof_end(L, slot, s);
   if (e != cudaSuccess) return cuda_fail(e, "backward kernel");
   L->g_valid = true;

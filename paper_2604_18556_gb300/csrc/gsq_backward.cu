@@ -14,6 +14,8 @@ namespace {
 template <class Rx, bool kExport, bool kShift, bool kAcc>
 __global__ void __launch_bounds__(kEwThreads, BwdOcc<Rx::L>::value) k_backward(const EwParams P) {
   constexpr int K = Rx::L;
+  grid_dep_wait();
+  grid_dep_launch();
   float q[kMaxLevels];
   load_grid(P, q);
   __shared__ float sgrid[kMaxLevels];
@@ -66,20 +68,30 @@ int ew_backward_grid(int K, int num_sms, int mode) {
   return g;
 }
 
-cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s) {
+cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s, bool pdl) {
   const bool export_mode = (p.grad_logits != nullptr) || (p.grad_scales != nullptr);
   const bool acc = p.acc_in_l != nullptr;
+  cudaLaunchAttribute attr[1];
+  pdl_attr(attr[0]);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kEwThreads, 1, 1);
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaError_t le = cudaSuccess;
   const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
     using Rx = typename decltype(rx)::type;
     constexpr bool SH = decltype(sh)::value;
     if (export_mode)
-      acc ? k_backward<Rx, true, SH, true><<<grid, kEwThreads, 0, s>>>(p)
-          : k_backward<Rx, true, SH, false><<<grid, kEwThreads, 0, s>>>(p);
+      le = acc ? cudaLaunchKernelEx(&cfg, k_backward<Rx, true, SH, true>, p)
+               : cudaLaunchKernelEx(&cfg, k_backward<Rx, true, SH, false>, p);
     else
-      acc ? k_backward<Rx, false, SH, true><<<grid, kEwThreads, 0, s>>>(p)
-          : k_backward<Rx, false, SH, false><<<grid, kEwThreads, 0, s>>>(p);
+      le = acc ? cudaLaunchKernelEx(&cfg, k_backward<Rx, false, SH, true>, p)
+               : cudaLaunchKernelEx(&cfg, k_backward<Rx, false, SH, false>, p);
   });
-  return e != cudaSuccess ? e : cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 }  // namespace gsq

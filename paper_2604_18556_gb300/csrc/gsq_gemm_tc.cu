@@ -157,6 +157,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dep_wait();  // A, B and the output may belong to the stream's previous kernel until here
+  grid_dep_launch();
 
   const int Mt = (args.M + TC_BM - 1) / TC_BM;
   const int Nt = (args.N + TC_BN - 1) / TC_BN;
@@ -385,6 +387,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   cluster_sync();  // both CTAs' barriers exist before any copy or arrival reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dep_wait();  // A, B and the output may belong to the stream's previous kernel until here
+  grid_dep_launch();
 
   const int Mt = (args.M + TC2_BM - 1) / TC2_BM;
   const int Nt = (args.N + BN - 1) / BN;
@@ -627,6 +631,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   cluster_sync();  // every CTA's barriers exist before any copy or arrival reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dep_wait();  // A, B and the output may belong to the stream's previous kernel until here
+  grid_dep_launch();
 
   const int Mt = (args.M + TC2_BM - 1) / TC2_BM;
   const int Mt2 = (Mt + 1) / 2;  // row-tile pairs per expert
@@ -833,8 +839,17 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   const int Mt = (g.M + TC_BM - 1) / TC_BM, Nt = (g.N + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  k_tc_gemm<BN><<<grid, TC_THREADS, TcCfg<BN>::kSmemBytes, s>>>(ta, tb, a);
-  return cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  pdl_attr(attr[0]);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(TC_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = TcCfg<BN>::kSmemBytes;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = g.pdl ? 1 : 0;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm<BN>, ta, tb, a);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <int BN>
@@ -869,7 +884,8 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
   int pairs = num_sms / 2;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  pdl_attr(attr[1]);
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
@@ -889,6 +905,7 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   if (max_clusters < pairs) pairs = max_clusters;
   if (tiles < pairs) pairs = static_cast<int>(tiles);
   cfg.gridDim = dim3(2 * pairs, 1, 1);
+  cfg.numAttrs = g.pdl ? 2 : 1;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_pair<BN>, ta, tb, to, a);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -924,7 +941,8 @@ cudaError_t launch_tc_gemm_quad_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   const int64_t tiles = static_cast<int64_t>(g.E) * ((Mt + 1) / 2) * Nt;
   int clusters = num_sms / 4;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  pdl_attr(attr[1]);
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 4;
   attr[0].val.clusterDim.y = 1;
@@ -944,6 +962,7 @@ cudaError_t launch_tc_gemm_quad_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   if (max_clusters < clusters) clusters = max_clusters;
   if (tiles < clusters) clusters = static_cast<int>(tiles);
   cfg.gridDim = dim3(4 * clusters, 1, 1);
+  cfg.numAttrs = g.pdl ? 2 : 1;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_quad<BN>, ta, tbq, to, a);
   return e != cudaSuccess ? e : cudaGetLastError();
 }

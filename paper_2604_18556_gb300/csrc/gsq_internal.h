@@ -14,6 +14,23 @@ constexpr int kSuperBlock = 256;  // K-Quant-like super-block (fp16 d)
 constexpr int kKqRecord = 110;    // bytes per packed super-block
 constexpr int kEwThreads = 256;   // threads per block of the elementwise kernels
 
+// Programmatic dependent launch. A kernel launched with the programmatic stream
+// serialization attribute (set by pdl_attr) may be scheduled while the kernel before it on
+// the stream is still running; grid_dep_wait() returns once that kernel has completed and
+// its writes are visible, so it comes before every access to global memory the kernel
+// before may read or write. grid_dep_launch() lets the next such kernel be scheduled onto
+// SMs this one frees. Without the attribute both are no-ops (PTX griddepcontrol, sm_90+).
+#ifdef __CUDACC__
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+#endif
+inline void pdl_attr(cudaLaunchAttribute& a) {
+  a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  a.val.programmaticStreamSerializationAllowed = 1;
+}
+
 // Device-side status words, one 256-byte slot of the workspace.
 struct DevFlags {
   unsigned int blocks_done;  // last-block-done counter of the loss reduction
@@ -91,13 +108,15 @@ gsq_status set_last_error(gsq_status st, const char* msg);
 
 // ---- launchers (gsq_elementwise.cu; backward: gsq_backward.cu, gsq_staged.cu) --
 cudaError_t launch_forward(const EwParams& p, int grid, cudaStream_t s);
-cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s);
+// pdl: launched with pdl_attr (the kernels wait for the one before them first).
+cudaError_t launch_backward(const EwParams& p, int grid, cudaStream_t s, bool pdl = false);
 // TMA-staged backward for non-export, non-accumulating steps: its grid for a
 // layer (resident blocks x SMs) and staging plan, 0 where it does not apply;
 // and its launch.
 int ew_staged_grid(int K, int mode, int w_bf16, int log2_group, int scales_frozen, int num_sms,
                    int* plan);
-cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s);
+cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s,
+                                   bool pdl = false);
 int ew_grid_size(int K, int which, int num_sms, int mode);  // which: 0 forward, 1 backward
 int ew_backward_grid(int K, int num_sms, int mode);          // gsq_backward.cu
 
@@ -236,6 +255,8 @@ struct TcGemm {
                 // 2: clusters of two pairs sharing B by multicast; 1: pairs or clusters of
                 // pairs, whichever tc_gemm_cluster_mode picks for the shape
   int stall;    // test hook (GSQ_TEST_STALL=gemm): the first k-block is never loaded
+  int pdl;      // 1: tensor-core kernels launched with pdl_attr (prologue overlaps the
+                // previous kernel's tail; operands read after grid_dep_wait)
 };
 bool tc_gemm_supported(int device);
 

@@ -91,6 +91,8 @@ __global__ void __launch_bounds__(kEwThreads, Plan::kOcc)
   __shared__ unsigned int done[2], issued[2];
   __shared__ int abort_flag;
   __shared__ float sgrid[kMaxLevels];
+  grid_dep_wait();
+  grid_dep_launch();
   float q[kMaxLevels];
   load_grid(P, q);
   const int tid = threadIdx.x, lane = tid & 31;
@@ -300,7 +302,8 @@ int ew_staged_grid(int K, int mode, int w_bf16, int log2_group, int scales_froze
   return g;
 }
 
-cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s) {
+cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaStream_t s,
+                                   bool pdl) {
   if (p.grad_logits || p.grad_scales || p.acc_in_l || p.acc_in_s) return cudaErrorInvalidValue;
   if (p.log2_group < 2 || p.log2_group > 7) return cudaErrorInvalidValue;
   // bulk copies need 16-byte aligned sources (tile offsets are multiples of 16 B)
@@ -309,6 +312,15 @@ cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaSt
       !a16(p.m_scales) || (p.j0 && !a16(p.j0)) || ((p.n * 4) & 15))
     return cudaErrorInvalidValue;
   bool launched = false;
+  cudaLaunchAttribute attr[1];
+  pdl_attr(attr[0]);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kEwThreads, 1, 1);
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaError_t le = cudaSuccess;
   const cudaError_t e = with_relax(p.K, p.mode, [&](auto rx, auto sh) {
     using Rx = typename decltype(rx)::type;
     constexpr bool SH = decltype(sh)::value;
@@ -316,13 +328,14 @@ cudaError_t launch_backward_staged(const EwParams& p, int grid, int plan, cudaSt
       using Plan = decltype(pl);
       const BwdStage S = stage_layout(Rx::L, Plan::kStageM, Plan::kStageGW, p.w_bf16, p.log2_group,
                                       p.scales_frozen, SH ? 1 : 0);
-      k_backward_staged<Rx, SH, Plan><<<grid, kEwThreads, 2 * S.bytes, s>>>(p, S);
+      cfg.dynamicSmemBytes = 2 * S.bytes;
+      le = cudaLaunchKernelEx(&cfg, k_backward_staged<Rx, SH, Plan>, p, S);
       launched = true;
     });
   });
   if (e != cudaSuccess) return e;
   if (!launched) return cudaErrorInvalidValue;
-  return cudaGetLastError();
+  return le != cudaSuccess ? le : cudaGetLastError();
 }
 
 }  // namespace gsq

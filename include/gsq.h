@@ -28,6 +28,12 @@
  *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).
  *     Work is enqueued on it; calls return without waiting for the GPU except
  *     where a function says it synchronises.
+ *   - The tensor-core and backward kernels of gsq_step and gsq_step_tokens are
+ *     launched as programmatic dependents of the kernel before them on the
+ *     stream: they may be scheduled while it drains, and wait for it to complete
+ *     (griddepcontrol.wait) before their first global memory access, so stream
+ *     order holds as for plain launches, also inside a captured CUDA graph.
+ *     With the environment variable GSQ_PDL=0 they are launched plainly.
  *   - Argument errors are detected on the host before anything is enqueued.
  *     Launch errors are reported as GSQ_ERR_CUDA.
  *   - Fault injection for host-side tests: with the environment variable

@@ -821,11 +821,13 @@ def gpu_arm_tokens(args, rank, world, local):
     tok_n, tok_ms = prof["tokens"]
     fwd_n, fwd_ms = prof["forward"]
     gemm_avg = gemm_ms / max(gemm_n, 1)
-    flops_per_launch = w.gemm_flops_per_step() / w.micro      # Y = D X^T and G = 2 Y X
+    gram = layer.tensor_size(gsq.GSQ_T_H) > 0     # the layer contracts through X^T X
+    flops_per_launch = w.gemm_flops_per_step(gram) / w.micro   # both GEMMs of a micro-batch
     gemm_tfs = flops_per_launch / (gemm_avg * 1e-3) / 1e12
     bytes_step = w.elementwise_bytes_per_step()
     bwd_gbs = bytes_step / (bwd_ms / n_timed * 1e-3) / 1e9
-    roofline = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} x 2 (Y = D X^T, then G = 2 Y X; "
+    route = "H = X^T X, then G = 2 D H" if gram else "Y = D X^T, then G = 2 Y X"
+    roofline = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} x 2 ({route}; "
                           "tcgen05, bf16 in, fp32 acc)",
                 "bound": "tensor", "achieved": gemm_tfs, "peak": tf_burst, "unit": "TFLOP/s",
                 "frac": gemm_tfs / tf_burst, "frac_of_sustained": gemm_tfs / tf_sust,

@@ -265,7 +265,12 @@ GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float ka
  * (another order returns GSQ_ERR_STATE).  Micro-batch j of step t:
  *   forward   fresh noise with the counter t*n_micro + j (every forward pass
  *             draws anew), W^_j, D_j = W^_j - W;
- *   loss      Y = D_j X^T, G = 2 Y X  (X = X_dev, this micro-batch's tokens),
+ *   loss      G = 2 D_j X^T X (X = X_dev, this micro-batch's tokens), as
+ *             Y = D_j X^T, G = 2 Y X, or on the tensor cores, where it costs fewer
+ *             flops (C (T + R) < 2 R T at the descriptor's n_tokens = T), through
+ *             the micro-batch's Gram matrix H = X^T X (bf16), G = 2 D_j H;
+ *             GSQ_TOKEN_ROUTE=direct|gram in the environment at gsq_init_layer
+ *             (and gsq_workspace_size) forces one;
  *             L_j = 1/2 sum D_j*G = sum over the tokens of ||D_j x||^2;
  *   backward  the gradients of L_j, added into an accumulator;
  *   update    after the last micro-batch only: Lion with the mean gradient
@@ -319,7 +324,9 @@ enum {
   GSQ_T_D = 4,          /* last forward's D = W^ - W, [E][R][C], bf16 or fp32  */
   GSQ_T_G = 5,          /* last step's dL/dW^, fp32 [E][R][C]                  */
   GSQ_T_W = 6,          /* stored copy of W, [E][R][C], w_dtype                */
-  GSQ_T_H = 7,          /* GEMM operand H (symmetrised), [E][C][C], bf16/fp32  */
+  GSQ_T_H = 7,          /* GEMM operand H (symmetrised), [E][C][C], bf16/fp32; *
+                         * per-step tokens: the last micro-batch's X^T X (bf16) *
+                         * on the Gram route, size 0 otherwise                  */
   GSQ_T_KQ_D = 8,       /* fp16 bits [E*R*C/256] (KQUANT2 only)                */
   GSQ_T_KQ_SC = 9,      /* int8 [E*R*C/16] (KQUANT2 only)                      */
   GSQ_T_J0 = 10         /* uint8 [E][R][C] initial grid index (SHIFT5 only);   *

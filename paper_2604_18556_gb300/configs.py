@@ -86,12 +86,23 @@ class Workload:
         write logits, logit momentum (4L each), D for the next step (2)."""
         return 16 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
 
-    def gemm_flops_per_step(self) -> int:
-        """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or
-        per micro-batch Y = D X^T and G = 2 Y X (4 R C T per expert)."""
+    def gram_route(self) -> bool:
+        """Per-step tokens on the tensor cores contract through each micro-batch's Gram
+        matrix (H = X^T X, then G = 2 D H) when that costs fewer flops than Y = D X^T,
+        G = 2 Y X: C (T + R) < 2 R T."""
+        return self.calib == "batches" and self.cols * (self.tokens + self.rows) < 2 * self.rows * self.tokens
+
+    def gemm_flops_per_step(self, gram=None) -> int:
+        """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or per
+        micro-batch Y = D X^T and G = 2 Y X (4 R C T per expert) or, on the Gram route
+        (gram: the layer's choice; None: the cost rule), H = X^T X and G = 2 D H
+        (2 C^2 T + 2 R C^2 per expert)."""
+        E, R, Cc = self.experts, self.rows, self.cols
         if self.calib == "batches":
-            return 4 * self.experts * self.rows * self.cols * self.tokens * self.micro
-        return 2 * self.experts * self.rows * self.cols * self.cols
+            if self.gram_route() if gram is None else gram:
+                return 2 * E * (Cc * Cc * self.tokens + R * Cc * Cc) * self.micro
+            return 4 * E * R * Cc * self.tokens * self.micro
+        return 2 * E * R * Cc * Cc
 
     def elementwise_bytes_per_step(self) -> int:
         """Algorithmic HBM bytes of one step's fused elementwise kernels, all

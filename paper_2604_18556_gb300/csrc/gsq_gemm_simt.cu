@@ -99,11 +99,11 @@ __global__ void k_symmetrize(const float* H, void* out, int C) {
 }
 
 // Tokens of one micro-batch to the tensor-core operands: Xb[e][t][c] and
-// Xt[e][c][t] = bf16(X[e][t][c]).  One 64 x 64 tile per block of 256 threads:
-// 16-byte loads along c, 8-byte stores of four bf16 to Xb, the tile through
-// shared memory, then 8-byte stores of four tokens to Xt.  T and C are
-// multiples of 8, so a group of four never straddles an edge.  ldt is the row
-// length of Xt.
+// Xt[e][c][t] = bf16(X[e][t][c]) (Xb null: Xt only).  One 64 x 64 tile per block
+// of 256 threads: 16-byte loads along c, 8-byte stores of four bf16 to Xb, the
+// tile through shared memory, then 8-byte stores of four tokens to Xt.  T and C
+// are multiples of 8, so a group of four never straddles an edge.  ldt is the
+// row length of Xt.
 __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat16* Xb,
                                                      __nv_bfloat16* Xt, int T, int C, int ldt) {
   __shared__ __nv_bfloat16 tile[64][68];
@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
   const int tid = threadIdx.x;
   const int q = (tid & 15) * 4, r0 = tid >> 4;  // 16 groups of four along the tile row
   const float* Xe = X + static_cast<int64_t>(e) * T * C;
-  __nv_bfloat16* Xbe = Xb + static_cast<int64_t>(e) * T * C;
+  __nv_bfloat16* Xbe = Xb ? Xb + static_cast<int64_t>(e) * T * C : nullptr;
   __nv_bfloat16* Xte = Xt + static_cast<int64_t>(e) * C * ldt;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -120,7 +120,7 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
     if (t < T && c < C) v = __ldcs(reinterpret_cast<const float4*>(Xe + static_cast<int64_t>(t) * C + c));
     const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
-    if (t < T && c < C) {
+    if (Xbe && t < T && c < C) {
       uint2 raw;
       raw.x = *reinterpret_cast<const uint32_t*>(&lo);
       raw.y = *reinterpret_cast<const uint32_t*>(&hi);

@@ -87,10 +87,13 @@ def test_workspace_size_formula(lib):
                           lr_scales=w.lr_scales,
                           param_mode=lib.PARAM_MODES[w.param])
         n, L = w.n, w.L
+        # per-step tokens contract through each micro-batch's Gram matrix X^T X where that
+        # costs fewer flops than Y = D X^T, G = 2 Y X: C (T + R) < 2 R T
+        gram = w.calib == "batches" and w.cols * (w.tokens + w.rows) < 2 * w.rows * w.tokens
         # every buffer is 256-byte aligned and followed by a 256-byte canary
         bufs = [256, 8 * 16384, 4 * L * n, 4 * L * n, 4 * n // w.group, 4 * n // w.group,
                 n * w.w_bytes()]
-        if w.calib != "batches":
+        if w.calib != "batches" or gram:
             bufs.append(w.experts * w.cols ** 2 * 2)               # H (bf16)
         bufs.append(2 * n)                                         # D (bf16)
         if w.calib != "batches":
@@ -104,7 +107,9 @@ def test_workspace_size_formula(lib):
             bufs.append(n)                                         # j0, one byte per weight
         if w.calib == "batches":                                   # bf16 X, X^T, Y; accumulators
             et = w.experts * w.tokens
-            bufs += [2 * et * w.cols, 2 * et * w.cols, 2 * et * w.rows, 4 * L * n, 4 * n // w.group]
+            bufs += ([2 * et * w.cols] if gram else
+                     [2 * et * w.cols, 2 * et * w.cols, 2 * et * w.rows])
+            bufs += [4 * L * n, 4 * n // w.group]
         bufs += [n, 8 * 17]                                        # initial codes; diagnostics
         expect = sum(_align(b) + 256 for b in bufs)
         assert lib.gsq_workspace_size(d) == expect, w.name

@@ -13,7 +13,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_common import TOL_BF16, TOL_F32, Case, assert_close, check_lion, gsq
+from gpu_common import TOL_BF16, TOL_F32, Case, assert_close, assert_gemm_bound, check_lion, gsq
 from oracle import gsq_oracle as O
 from paper_2604_18556_gb300 import configs as C
 from paper_2604_18556_gb300 import inputs
@@ -33,22 +33,60 @@ def _batches(w, step):
     return [inputs.make_token_batch(w, step, j, device="cuda") for j in range(w.micro)]
 
 
-@pytest.mark.parametrize("gemm", ["f32", "bf16"])
+@pytest.mark.parametrize("gemm,route", [("f32", "direct"), ("bf16", "direct"), ("bf16", "gram")])
 @pytest.mark.parametrize("name", list(CASES))
-def test_token_steps_match_oracle(name, gemm):
+def test_token_steps_match_oracle(name, gemm, route, monkeypatch):
+    """route: the tensor-core contraction as Y = D X^T, G = 2 Y X ("direct") or through the
+    micro-batch's Gram matrix H = X^T X, G = 2 D H ("gram"); the fp32 path is direct."""
+    monkeypatch.setenv("GSQ_TOKEN_ROUTE", route)
     _check_token_steps(CASES[name], gemm)
 
 
+@pytest.mark.parametrize("route", ["direct", "gram"])
 @pytest.mark.parametrize("mode,kernel", [("0", "k_tc_gemm"), ("1", "k_tc_gemm_pair"),
                                          ("2", "k_tc_gemm_quad")])
-def test_token_steps_on_every_contraction_kernel(mode, kernel, monkeypatch):
-    """Both token contractions (Y = D X^T with bf16 output, G = 2 Y X with fp32 output)
-    on single CTAs, CTA pairs and clusters of two pairs sharing operand tiles by TMA
-    multicast, against the oracle."""
+def test_token_steps_on_every_contraction_kernel(mode, kernel, route, monkeypatch):
+    """Both token contractions of either route (Y = D X^T with bf16 output and G = 2 Y X
+    with fp32 output; or H = X^T X with bf16 output and G = 2 D H) on single CTAs, CTA
+    pairs and clusters of two pairs sharing operand tiles by TMA multicast, against the
+    oracle."""
     monkeypatch.setenv("GSQ_GEMM_PAIR", mode)
+    monkeypatch.setenv("GSQ_TOKEN_ROUTE", route)
     w = dataclasses.replace(CASES["full"], rows=600)   # three 256-row tiles: a ragged cluster
     case = _check_token_steps(w, "bf16")
     assert case.layer.kernel_name(gsq().GSQ_K_GEMM) == kernel
+
+
+@pytest.mark.parametrize("mode", ["0", "1", "2"])
+def test_gram_route_contractions(mode, monkeypatch):
+    """The Gram route on the kernels' own bf16 operands, two experts: the micro-batch's
+    H = X^T X (fp32 accumulation of the bf16 tokens, then one rounding to bf16) within
+    the accumulation bound plus that rounding, G = 2 D H within the accumulation bound
+    of the bf16 D and H, and the loss as 1/2 sum D G."""
+    monkeypatch.setenv("GSQ_TOKEN_ROUTE", "gram")
+    monkeypatch.setenv("GSQ_GEMM_PAIR", mode)
+    w = dataclasses.replace(BASE, experts=2, rows=600, micro=1)
+    case = Case(w, gemm="bf16")
+    g = gsq()
+    X = inputs.make_token_batch(w, 0, 0, device="cuda")
+    loss = torch.zeros(1, device="cuda")
+    case.layer.step_tokens(0, 0, 1, w.tau(0), X, loss=loss)   # no look-ahead: D stays
+    torch.cuda.synchronize()
+    case.layer.sync_status()
+    Cc, T = w.cols, X.shape[1]
+    Hj = case.tensor(g.GSQ_T_H, torch.bfloat16).float().view(w.experts, Cc, Cc).cpu().numpy()
+    Xb = X.bfloat16().double().cpu().numpy()
+    D, G = case.D(), case.G()
+    rows = np.arange(w.experts * w.rows)
+    for e in range(w.experts):
+        exact = Xb[e].T @ Xb[e]
+        absum = np.abs(Xb[e]).T @ np.abs(Xb[e])
+        bound = 1.01 * T * 2.0 ** -24 * absum + 2.0 ** -8 * np.abs(exact) + 1e-30
+        worst = float((np.abs(Hj[e] - exact) / bound).max())
+        assert worst <= 1.0, ("H = X^T X", e, worst)
+        sel = rows // w.rows == e
+        assert_gemm_bound(G[sel], D[sel], Hj[e], f"G = 2 D H, expert {e}")
+    assert abs(loss.item() - 0.5 * np.sum(D.astype(np.float64) * G)) <= 1e-5 * abs(loss.item())
 
 
 def _check_token_steps(w, gemm):

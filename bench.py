@@ -822,11 +822,13 @@ def gpu_arm_tokens(args, rank, world, local):
     fwd_n, fwd_ms = prof["forward"]
     gemm_avg = gemm_ms / max(gemm_n, 1)
     gram = layer.tensor_size(gsq.GSQ_T_H) > 0     # the layer contracts through X^T X
-    flops_per_launch = w.gemm_flops_per_step(gram) / w.micro   # both GEMMs of a micro-batch
+    sym = os.environ.get("GSQ_TOKEN_SYM", "1") != "0"   # ... formed from its upper triangle
+    flops_per_launch = w.gemm_flops_per_step(gram, sym) / w.micro   # a micro-batch's GEMMs
     gemm_tfs = flops_per_launch / (gemm_avg * 1e-3) / 1e12
     bytes_step = w.elementwise_bytes_per_step()
     bwd_gbs = bytes_step / (bwd_ms / n_timed * 1e-3) / 1e9
-    route = "H = X^T X, then G = 2 D H" if gram else "Y = D X^T, then G = 2 Y X"
+    route = ("H = X^T X" + (" (upper triangle, mirrored)" if sym else "") + ", then G = 2 D H"
+             if gram else "Y = D X^T, then G = 2 Y X")
     roofline = {"kernel": f"{layer.kernel_name(gsq.GSQ_K_GEMM)} x 2 ({route}; "
                           "tcgen05, bf16 in, fp32 acc)",
                 "bound": "tensor", "achieved": gemm_tfs, "peak": tf_burst, "unit": "TFLOP/s",
@@ -837,8 +839,9 @@ def gpu_arm_tokens(args, rank, world, local):
                     "bound": "hbm", "achieved": bwd_gbs, "peak": hbm, "unit": "GB/s",
                     "frac": bwd_gbs / hbm, "algorithmic_bytes_per_step": bytes_step,
                     "ms_per_step": bwd_ms / n_timed}
-    # kernels of the headline rounds (a GEMM profile entry covers both token GEMMs)
-    launches = (gemm_n * 2 + bwd_n + tok_n + fwd_n) * len(reps) // max(len(prof_reps), 1)
+    # kernels of the headline rounds (a GEMM profile entry covers a micro-batch's GEMMs)
+    per_gemm = 3 if gram and sym else 2      # the GEMMs of a micro-batch (and the mirror)
+    launches = (gemm_n * per_gemm + bwd_n + tok_n + fwd_n) * len(reps) // max(len(prof_reps), 1)
 
     e2e = None
     if not args.no_e2e:

@@ -92,16 +92,17 @@ class Workload:
         G = 2 Y X: C (T + R) < 2 R T."""
         return self.calib == "batches" and self.cols * (self.tokens + self.rows) < 2 * self.rows * self.tokens
 
-    def gemm_flops_per_step(self, gram=None) -> int:
+    def gemm_flops_per_step(self, gram=None, sym=True) -> int:
         """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or per
         micro-batch Y = D X^T and G = 2 Y X (4 R C T per expert) or, on the Gram route
         (gram: the layer's choice; None: the cost rule), H = X^T X and G = 2 D H
-        (2 C^2 T + 2 R C^2 per expert)."""
-        E, R, Cc = self.experts, self.rows, self.cols
+        (2 C^2 T + 2 R C^2 per expert; C (C + 1) T for H's upper triangle when sym)."""
+        E, R, Cc, T = self.experts, self.rows, self.cols, self.tokens
         if self.calib == "batches":
             if self.gram_route() if gram is None else gram:
-                return 2 * E * (Cc * Cc * self.tokens + R * Cc * Cc) * self.micro
-            return 4 * E * R * Cc * self.tokens * self.micro
+                h = Cc * (Cc + 1) * T if sym else 2 * Cc * Cc * T
+                return E * (h + 2 * R * Cc * Cc) * self.micro
+            return 4 * E * R * Cc * T * self.micro
         return 2 * E * R * Cc * Cc
 
     def elementwise_bytes_per_step(self) -> int:

@@ -290,6 +290,7 @@ struct gsq_layer {
   int gemm_pair;      // 1: the loss GEMM runs on CTA pairs (cta_group::2)
   int test_stall;     // test hook (GSQ_TEST_STALL): 1 staged backward, 2 tensor-core GEMM
   bool pdl;           // step kernels launched as programmatic dependents of the one before
+  bool token_sym;     // Gram route of per-step tokens: X^T X from its upper triangle
   bool g_valid; // the G buffer holds the last step's G
   size_t d_cur; // offset of the buffer holding the latest D written
   // pending forward (D valid for these arguments)
@@ -661,6 +662,10 @@ gsq_status gsq_init_layer(const gsq_layer_desc* desc, void* workspace, size_t by
   // (griddepcontrol) before touching memory. GSQ_PDL=0 launches them plainly.
   L->pdl = true;
   if (const char* pv = std::getenv("GSQ_PDL")) L->pdl = std::atoi(pv) != 0;
+  // The Gram route forms X^T X from the tiles of its upper triangle and mirrors them
+  // (half the flops); GSQ_TOKEN_SYM=0 computes every tile.
+  L->token_sym = true;
+  if (const char* sv = std::getenv("GSQ_TOKEN_SYM")) L->token_sym = std::atoi(sv) != 0;
   L->group_n = kGemmGroupN;
   if (const char* gn = std::getenv("GSQ_GEMM_GROUP_N")) {  // tile-order column group (0: none)
     const int v = std::atoi(gn);
@@ -872,14 +877,17 @@ gsq_status gsq_step_tokens(gsq_layer* L, uint64_t step, uint32_t micro, uint32_t
     g.E = E;
     if (sh.gram) {
       void* Hj = L->ws + L->lay.H;
-      if (e == cudaSuccess) {  // H[e] = X[e]^T X[e]  (M = N = C, K = T), bf16 out
-        g.M = C; g.N = C; g.K = T;
+      if (e == cudaSuccess) {  // H[e] = X[e]^T X[e]  (M = N = C, K = T), bf16 out: the
+        g.M = C; g.N = C; g.K = T;  // tiles of the upper triangle, then its mirror below
         g.A = Xt;
         g.B = Xt;
         g.out = Hj;
         g.out_bf16 = 1;
         g.alpha = 1.0f;
+        g.sym = L->token_sym ? 1 : 0;
         e = launch_tc_gemm(g, L->num_sms, s);
+        if (e == cudaSuccess && g.sym) e = launch_mirror_upper_bf16(Hj, E, C, s);
+        g.sym = 0;
       }
       if (e == cudaSuccess) {  // G[e] = 2 D[e] H[e]  (N = C, K = C; H symmetric), fp32 out
         g.M = R; g.N = C; g.K = C;

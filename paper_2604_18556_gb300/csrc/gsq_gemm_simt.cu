@@ -98,6 +98,28 @@ __global__ void k_symmetrize(const float* H, void* out, int C) {
   }
 }
 
+// H[e][i][j] = H[e][j][i] for i > j (bf16): the lower triangle from the upper one,
+// through a 32x32 shared tile; blocks wholly above the diagonal return at once.  A
+// block reads only the upper triangle and writes only the lower one, so blocks
+// never race.
+__global__ void k_mirror_upper_bf16(__nv_bfloat16* H, int C) {
+  const int bi = blockIdx.y, bj = blockIdx.x;  // destination tile: rows bi, columns bj
+  if (bj > bi) return;
+  __shared__ __nv_bfloat16 t[32][34];
+  __nv_bfloat16* He = H + static_cast<int64_t>(blockIdx.z) * C * C;
+  const int i0 = bi * 32, j0 = bj * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  for (int r = ty; r < 32; r += 8) {  // source tile: rows j0.., columns i0..
+    const int i = j0 + r, j = i0 + tx;
+    if (i < C && j < C) t[r][tx] = He[static_cast<int64_t>(i) * C + j];
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int i = i0 + r, j = j0 + tx;
+    if (i < C && j < C && i > j) He[static_cast<int64_t>(i) * C + j] = t[tx][r];
+  }
+}
+
 // Tokens of one micro-batch to the tensor-core operands: Xb[e][t][c] and
 // Xt[e][c][t] = bf16(X[e][t][c]) (Xb null: Xt only).  One 64 x 64 tile per block
 // of 256 threads: 16-byte loads along c, 8-byte stores of four bf16 to Xb, the
@@ -191,6 +213,14 @@ cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_b
     k_symmetrize<true><<<grid, block, 0, s>>>(H, out, C);
   else
     k_symmetrize<false><<<grid, block, 0, s>>>(H, out, C);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mirror_upper_bf16(void* H, int E, int C, cudaStream_t s) {
+  if (E <= 0 || C <= 0) return cudaSuccess;
+  dim3 grid((C + 31) / 32, (C + 31) / 32, E);
+  dim3 block(32, 8);
+  k_mirror_upper_bf16<<<grid, block, 0, s>>>(static_cast<__nv_bfloat16*>(H), C);
   return cudaGetLastError();
 }
 

@@ -111,7 +111,18 @@ struct TcArgs {
   int out_bf16;
   float alpha;
   DevFlags* flags;
+  int sym_per_e;  // > 0: symmetric output, only the upper-triangle tiles (tile_coords_upper)
 };
+
+// Output tile `tile` of the launch: the full order of tile_coords, or the upper
+// triangle of a symmetric output.
+__device__ __forceinline__ void tile_at(const TcArgs& a, int tile, int Mt, int Nt, int BM, int BN,
+                                        int& e, int& m, int& n) {
+  if (a.sym_per_e > 0)
+    tile_coords_upper(tile, Mt, Nt, BM, BN, a.sym_per_e, e, m, n);
+  else
+    tile_coords(tile, Mt, Nt, a.group_n, e, m, n);
+}
 
 template <int BN>
 __global__ void __launch_bounds__(TC_THREADS, 1)
@@ -164,7 +175,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int Nt = (args.N + TC_BN - 1) / TC_BN;
   const int KB = (args.K + TC_BK - 1) / TC_BK;
   static_assert(TC_STAGES >= 2, "pipeline depth");
-  const int tiles = args.E * Mt * Nt;
+  const int tiles = args.E * (args.sym_per_e > 0 ? args.sym_per_e : Mt * Nt);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -177,7 +188,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
         int e, m, n;
-        tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+        tile_at(args, tile, Mt, Nt, TC_BM, TC_BN, e, m, n);
         const int arow = e * args.M + m * TC_BM;
         const int brow = e * args.N + n * TC_BN;
         for (int kb = 0; kb < KB; ++kb) {
@@ -253,7 +264,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
       tc_fence_after();
       int e, m, n;
-      tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+      tile_at(args, tile, Mt, Nt, TC_BM, TC_BN, e, m, n);
       const int row = m * TC_BM + quarter * 32 + lane;
       const int col0 = n * TC_BN;
       const int64_t obase = (static_cast<int64_t>(e) * args.M + row) * args.N;
@@ -393,7 +404,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int Mt = (args.M + TC2_BM - 1) / TC2_BM;
   const int Nt = (args.N + BN - 1) / BN;
   const int KB = (args.K + TC_BK - 1) / TC_BK;
-  const int tiles = args.E * Mt * Nt;
+  const int tiles = args.E * (args.sym_per_e > 0 ? args.sym_per_e : Mt * Nt);
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
 
   if (warp == 0) {
@@ -404,7 +415,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       bool ok = true;
       for (int tile = pair; ok && tile < tiles; tile += npairs) {
         int e, m, n;
-        tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+        tile_at(args, tile, Mt, Nt, TC2_BM, BN, e, m, n);
         const int arow = e * args.M + m * TC2_BM + static_cast<int>(rank) * TC_BM;
         const int brow = e * args.N + n * BN + static_cast<int>(rank) * Cfg::kBHalf;
         for (int kb = 0; kb < KB; ++kb) {
@@ -488,7 +499,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!mbar_wait(tfull_bar + acc, acc_phase, abort_flag)) break;
       tc_fence_after();
       int e, m, n;
-      tile_coords(tile, Mt, Nt, args.group_n, e, m, n);
+      tile_at(args, tile, Mt, Nt, TC2_BM, BN, e, m, n);
       const int row0 = m * TC2_BM + static_cast<int>(rank) * TC_BM + quarter * 32;
       const int col0 = n * BN;
       const uint32_t taddr = tmem_base + static_cast<uint32_t>(acc * Cfg::kAccStride) +
@@ -812,6 +823,15 @@ double wave_balance(int64_t tiles, int num_sms) {
   return static_cast<double>(tiles) / static_cast<double>(waves * num_sms);
 }
 
+// Tiles of one expert's upper triangle (tile_coords_upper) for an M x M output in
+// BM x BN tiles.
+int upper_tiles(int M, int BM, int BN) {
+  const int Mt = (M + BM - 1) / BM, Nt = (M + BN - 1) / BN;
+  int count = 0;
+  for (int m = 0; m < Mt; ++m) count += Nt - (m * BM) / BN;
+  return count;
+}
+
 template <int BN>
 cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   // set on every launch: the attribute belongs to the current device
@@ -836,8 +856,9 @@ cudaError_t launch_tc_gemm_bn(const TcGemm& g, int num_sms, cudaStream_t s) {
   a.alpha = g.alpha;
   a.flags = g.flags;
   a.stall = g.stall;
+  a.sym_per_e = g.sym ? upper_tiles(g.M, TC_BM, BN) : 0;
   const int Mt = (g.M + TC_BM - 1) / TC_BM, Nt = (g.N + BN - 1) / BN;
-  const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
+  const int64_t tiles = static_cast<int64_t>(g.E) * (g.sym ? a.sym_per_e : Mt * Nt);
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
   cudaLaunchAttribute attr[1];
   pdl_attr(attr[0]);
@@ -880,8 +901,9 @@ cudaError_t launch_tc_gemm_pair_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   a.alpha = g.alpha;
   a.flags = g.flags;
   a.stall = g.stall;
+  a.sym_per_e = g.sym ? upper_tiles(g.M, TC2_BM, BN) : 0;
   const int Mt = (g.M + TC2_BM - 1) / TC2_BM, Nt = (g.N + BN - 1) / BN;
-  const int64_t tiles = static_cast<int64_t>(g.E) * Mt * Nt;
+  const int64_t tiles = static_cast<int64_t>(g.E) * (g.sym ? a.sym_per_e : Mt * Nt);
   int pairs = num_sms / 2;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
@@ -937,6 +959,7 @@ cudaError_t launch_tc_gemm_quad_bn(const TcGemm& g, int num_sms, cudaStream_t s)
   a.alpha = g.alpha;
   a.flags = g.flags;
   a.stall = g.stall;
+  a.sym_per_e = 0;  // clusters compute every tile (symmetric outputs run on pairs)
   const int Mt = (g.M + TC2_BM - 1) / TC2_BM, Nt = (g.N + BN - 1) / BN;
   const int64_t tiles = static_cast<int64_t>(g.E) * ((Mt + 1) / 2) * Nt;
   int clusters = num_sms / 4;
@@ -1058,9 +1081,26 @@ int tc_gemm_cluster_mode(int E, int M, int N, int bn, int num_sms) {
   return cluster_mode_bn<256>(E, M, N, num_sms);
 }
 
+// Tile width of a symmetric output's upper triangle: 224 or 256, whichever costs fewer
+// waves x width (4096 x 4096 on pairs: 136 tiles 256 wide, 2 waves, against 173 tiles
+// 224 wide, 3 waves).
+int sym_tile_n(int E, int M, int num_sms, int pair) {
+  const int units = pair ? (num_sms / 2 > 0 ? num_sms / 2 : 1) : (num_sms > 0 ? num_sms : 1);
+  const int bm = pair ? TC2_BM : TC_BM;
+  auto cost = [&](int bn) {
+    const int64_t tiles = static_cast<int64_t>(E) * upper_tiles(M, bm, bn);
+    return static_cast<double>((tiles + units - 1) / units) * bn;
+  };
+  return cost(256) <= cost(224) ? 256 : 224;
+}
+
 cudaError_t launch_tc_gemm(const TcGemm& g, int num_sms, cudaStream_t s) {
-  const int bn = g.tile_n ? g.tile_n : tc_gemm_tile_n(g.E, g.M, g.N, num_sms, g.pair);
-  const int mode = g.pair == 1 ? tc_gemm_cluster_mode(g.E, g.M, g.N, bn, num_sms) : g.pair;
+  if (g.sym && g.M != g.N) return cudaErrorInvalidValue;
+  const int bn = g.tile_n ? g.tile_n
+                          : (g.sym ? sym_tile_n(g.E, g.M, num_sms, g.pair)
+                                   : tc_gemm_tile_n(g.E, g.M, g.N, num_sms, g.pair));
+  int mode = g.pair == 1 ? tc_gemm_cluster_mode(g.E, g.M, g.N, bn, num_sms) : g.pair;
+  if (g.sym && mode == 2) mode = 3;  // the upper-triangle order runs on pairs
   if (mode == 2 && num_sms >= 4) {
     if (bn == 128) return launch_tc_gemm_quad_bn<128>(g, num_sms, s);
     if (bn == 224) return launch_tc_gemm_quad_bn<224>(g, num_sms, s);

@@ -232,6 +232,9 @@ cudaError_t launch_simt_gemm(const SimtGemm& g, cudaStream_t s);
 // H_out[e] = (H[e] + H[e]^T) / 2 converted to bf16 (out_bf16=1) or fp32.
 cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_bf16,
                               cudaStream_t s);
+// H[e][i][j] = H[e][j][i] for i > j, bf16 [E][C][C] in place (the lower triangle of a
+// symmetric output whose upper triangle a TcGemm with sym = 1 computed).
+cudaError_t launch_mirror_upper_bf16(void* H, int E, int C, cudaStream_t s);
 // Xb[e] = bf16(X[e]) ([T][C]) and Xt[e] = bf16(X[e])^T ([C][ldt], first T columns).
 cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
                                cudaStream_t s);
@@ -257,6 +260,9 @@ struct TcGemm {
   int stall;    // test hook (GSQ_TEST_STALL=gemm): the first k-block is never loaded
   int pdl;      // 1: tensor-core kernels launched with pdl_attr (prologue overlaps the
                 // previous kernel's tail; operands read after grid_dep_wait)
+  int sym;      // 1: symmetric output (M = N, out = A A^T with B = A): only the tiles
+                // of the upper triangle are computed; launch_mirror_upper_bf16 fills
+                // the rest (clusters of pairs fall back to pairs)
 };
 bool tc_gemm_supported(int device);
 

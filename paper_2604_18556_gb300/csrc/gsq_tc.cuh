@@ -318,5 +318,24 @@ __device__ __forceinline__ void tile_coords(int tile, int Mt, int Nt, int GN, in
   n = n0 + (rr - m * gw);
 }
 
+// Upper-triangle tile order for a symmetric output (out = A A^T, M = N): per expert
+// only the tiles holding an element with row <= column, row block m from its first
+// such column tile floor(m BM / BN) on, row by row; per_e of them per expert.  The
+// elements below the diagonal inside those tiles are computed as well; the caller
+// overwrites the lower triangle with the mirror of the upper one.
+__device__ __forceinline__ void tile_coords_upper(int tile, int Mt, int Nt, int BM, int BN,
+                                                  int per_e, int& e, int& m, int& n) {
+  e = tile / per_e;
+  int r = tile - e * per_e;
+  m = 0;
+  while (m < Mt - 1) {
+    const int cnt = Nt - (m * BM) / BN;
+    if (r < cnt) break;
+    r -= cnt;
+    ++m;
+  }
+  n = (m * BM) / BN + r;
+}
+
 }  // namespace
 }  // namespace gsq

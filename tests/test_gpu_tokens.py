@@ -57,15 +57,20 @@ def test_token_steps_on_every_contraction_kernel(mode, kernel, route, monkeypatc
     assert case.layer.kernel_name(gsq().GSQ_K_GEMM) == kernel
 
 
+@pytest.mark.parametrize("sym", ["1", "0"], ids=["upper_triangle", "every_tile"])
 @pytest.mark.parametrize("mode", ["0", "1", "2"])
-def test_gram_route_contractions(mode, monkeypatch):
+@pytest.mark.parametrize("cols", [384, 1152])
+def test_gram_route_contractions(cols, mode, sym, monkeypatch):
     """The Gram route on the kernels' own bf16 operands, two experts: the micro-batch's
     H = X^T X (fp32 accumulation of the bf16 tokens, then one rounding to bf16) within
-    the accumulation bound plus that rounding, G = 2 D H within the accumulation bound
-    of the bf16 D and H, and the loss as 1/2 sum D G."""
+    the accumulation bound plus that rounding, and exactly symmetric, whether formed
+    from the tiles of its upper triangle and mirrored (default) or from every tile;
+    G = 2 D H within the accumulation bound of the bf16 D and H; the loss as 1/2 sum
+    D G.  1,152 inputs: ragged tiles on both sides of the diagonal."""
     monkeypatch.setenv("GSQ_TOKEN_ROUTE", "gram")
+    monkeypatch.setenv("GSQ_TOKEN_SYM", sym)
     monkeypatch.setenv("GSQ_GEMM_PAIR", mode)
-    w = dataclasses.replace(BASE, experts=2, rows=600, micro=1)
+    w = dataclasses.replace(BASE, experts=2, rows=600, cols=cols, micro=1)
     case = Case(w, gemm="bf16")
     g = gsq()
     X = inputs.make_token_batch(w, 0, 0, device="cuda")
@@ -79,6 +84,7 @@ def test_gram_route_contractions(mode, monkeypatch):
     D, G = case.D(), case.G()
     rows = np.arange(w.experts * w.rows)
     for e in range(w.experts):
+        assert np.array_equal(Hj[e], Hj[e].T), ("H = X^T X not symmetric", e)
         exact = Xb[e].T @ Xb[e]
         absum = np.abs(Xb[e]).T @ np.abs(Xb[e])
         bound = 1.01 * T * 2.0 ** -24 * absum + 2.0 ** -8 * np.abs(exact) + 1e-30

@@ -98,25 +98,42 @@ __global__ void k_symmetrize(const float* H, void* out, int C) {
   }
 }
 
-// H[e][i][j] = H[e][j][i] for i > j (bf16): the lower triangle from the upper one,
-// through a 32x32 shared tile; blocks wholly above the diagonal return at once.  A
-// block reads only the upper triangle and writes only the lower one, so blocks
-// never race.
-__global__ void k_mirror_upper_bf16(__nv_bfloat16* H, int C) {
-  const int bi = blockIdx.y, bj = blockIdx.x;  // destination tile: rows bi, columns bj
-  if (bj > bi) return;
-  __shared__ __nv_bfloat16 t[32][34];
-  __nv_bfloat16* He = H + static_cast<int64_t>(blockIdx.z) * C * C;
-  const int i0 = bi * 32, j0 = bj * 32;
-  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
-  for (int r = ty; r < 32; r += 8) {  // source tile: rows j0.., columns i0..
-    const int i = j0 + r, j = i0 + tx;
-    if (i < C && j < C) t[r][tx] = He[static_cast<int64_t>(i) * C + j];
+// H[e][i][j] = H[e][j][i] for i > j (bf16, C even): the lower triangle from the upper
+// one.  One block per 64 x 64 destination tile on or below the diagonal (blocks
+// enumerated over the triangle): the source tile above the diagonal is read with
+// 4-byte loads of two columns into shared memory, the destination written with 4-byte
+// stores of two columns.  A block reads only the upper triangle and writes only the
+// lower one (a diagonal tile reads all of itself before writing), so blocks never race.
+__global__ void __launch_bounds__(256) k_mirror_upper_bf16(__nv_bfloat16* H, int C) {
+  const int x = blockIdx.x;
+  int bi = static_cast<int>((sqrtf(8.0f * static_cast<float>(x) + 1.0f) - 1.0f) * 0.5f);
+  while ((bi + 1) * (bi + 2) / 2 <= x) ++bi;
+  while (bi * (bi + 1) / 2 > x) --bi;
+  const int bj = x - bi * (bi + 1) / 2;  // destination tile: rows bi, columns bj <= bi
+  __shared__ __align__(4) __nv_bfloat16 t[64][66];
+  __nv_bfloat16* He = H + static_cast<int64_t>(blockIdx.y) * C * C;
+  const int i0 = bi * 64, j0 = bj * 64;
+  for (int k = threadIdx.x; k < 64 * 32; k += 256) {  // source rows j0.., columns i0..
+    const int r = k >> 5, c = (k & 31) * 2;
+    const int gi = j0 + r, gj = i0 + c;
+    if (gi < C && gj < C)
+      *reinterpret_cast<uint32_t*>(&t[r][c]) =
+          *reinterpret_cast<const uint32_t*>(He + static_cast<int64_t>(gi) * C + gj);
   }
   __syncthreads();
-  for (int r = ty; r < 32; r += 8) {
-    const int i = i0 + r, j = j0 + tx;
-    if (i < C && j < C && i > j) He[static_cast<int64_t>(i) * C + j] = t[tx][r];
+  for (int k = threadIdx.x; k < 64 * 32; k += 256) {  // destination rows i0.., columns j0..
+    const int r = k >> 5, c = (k & 31) * 2;
+    const int gi = i0 + r, gj = j0 + c;
+    if (gi >= C || gj >= C || gi <= gj) continue;
+    __nv_bfloat16* dst = He + static_cast<int64_t>(gi) * C + gj;
+    if (gi > gj + 1) {
+      __nv_bfloat162 v;
+      v.x = t[c][r];
+      v.y = t[c + 1][r];
+      *reinterpret_cast<__nv_bfloat162*>(dst) = v;
+    } else {
+      *dst = t[c][r];
+    }
   }
 }
 
@@ -218,9 +235,10 @@ cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_b
 
 cudaError_t launch_mirror_upper_bf16(void* H, int E, int C, cudaStream_t s) {
   if (E <= 0 || C <= 0) return cudaSuccess;
-  dim3 grid((C + 31) / 32, (C + 31) / 32, E);
-  dim3 block(32, 8);
-  k_mirror_upper_bf16<<<grid, block, 0, s>>>(static_cast<__nv_bfloat16*>(H), C);
+  if (C % 2 != 0) return cudaErrorInvalidValue;
+  const int nb = (C + 63) / 64;
+  dim3 grid(nb * (nb + 1) / 2, E);
+  k_mirror_upper_bf16<<<grid, 256, 0, s>>>(static_cast<__nv_bfloat16*>(H), C);
   return cudaGetLastError();
 }
 

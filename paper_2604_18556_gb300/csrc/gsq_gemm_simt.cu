@@ -138,11 +138,11 @@ __global__ void __launch_bounds__(256) k_mirror_upper_bf16(__nv_bfloat16* H, int
 }
 
 // Tokens of one micro-batch to the tensor-core operands: Xb[e][t][c] and
-// Xt[e][c][t] = bf16(X[e][t][c]) (Xb null: Xt only).  One 64 x 64 tile per block
-// of 256 threads: 16-byte loads along c, 8-byte stores of four bf16 to Xb, the
-// tile through shared memory, then 8-byte stores of four tokens to Xt.  T and C
-// are multiples of 8, so a group of four never straddles an edge.  ldt is the
-// row length of Xt.
+// Xt[e][c][t] = bf16(X[e][t][c]).  One 64 x 64 tile per block of 256 threads:
+// 16-byte loads along c, 8-byte stores of four bf16 to Xb, the tile through
+// shared memory, then 8-byte stores of four tokens to Xt.  T and C are
+// multiples of 8, so a group of four never straddles an edge.  ldt is the row
+// length of Xt.
 __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat16* Xb,
                                                      __nv_bfloat16* Xt, int T, int C, int ldt) {
   __shared__ __nv_bfloat16 tile[64][68];
@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
   const int tid = threadIdx.x;
   const int q = (tid & 15) * 4, r0 = tid >> 4;  // 16 groups of four along the tile row
   const float* Xe = X + static_cast<int64_t>(e) * T * C;
-  __nv_bfloat16* Xbe = Xb ? Xb + static_cast<int64_t>(e) * T * C : nullptr;
+  __nv_bfloat16* Xbe = Xb + static_cast<int64_t>(e) * T * C;
   __nv_bfloat16* Xte = Xt + static_cast<int64_t>(e) * C * ldt;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -159,7 +159,7 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
     if (t < T && c < C) v = __ldcs(reinterpret_cast<const float4*>(Xe + static_cast<int64_t>(t) * C + c));
     const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
-    if (Xbe && t < T && c < C) {
+    if (t < T && c < C) {
       uint2 raw;
       raw.x = *reinterpret_cast<const uint32_t*>(&lo);
       raw.y = *reinterpret_cast<const uint32_t*>(&hi);
@@ -181,6 +181,41 @@ __global__ void __launch_bounds__(256) k_tokens_bf16(const float* X, __nv_bfloat
       *reinterpret_cast<uint2*>(Xte + static_cast<int64_t>(c) * ldt + t) = raw;
     }
   }
+}
+
+// Tokens of one micro-batch to X^T alone: Xt[e][c][t] = bf16(X[e][t][c]), without
+// shared memory.  Each thread reads 8 consecutive tokens x 4 channels (eight 16-byte
+// loads; the 16 lanes of a half-warp cover 64 channels of one token row) and writes
+// each channel's 8 tokens with one 16-byte store.  A block covers 128 tokens x 64
+// channels.  T and C are multiples of 8, so a thread's tokens and channels are all
+// inside or all outside the layer.
+__global__ void __launch_bounds__(256) k_tokens_t_bf16(const float* X, __nv_bfloat16* Xt, int T,
+                                                       int C, int ldt) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int c = blockIdx.x * 64 + (lane & 15) * 4;
+  const int t0 = blockIdx.y * 128 + warp * 16 + (lane >> 4) * 8;
+  if (c >= C || t0 >= T) return;
+  const float* Xe = X + static_cast<int64_t>(blockIdx.z) * T * C;
+  __nv_bfloat16* Xte = Xt + static_cast<int64_t>(blockIdx.z) * C * ldt;
+  float4 v[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    v[i] = __ldcs(reinterpret_cast<const float4*>(Xe + static_cast<int64_t>(t0 + i) * C + c));
+  auto pack = [](float a, float b) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  };
+  __nv_bfloat16* o = Xte + static_cast<int64_t>(c) * ldt + t0;
+  *reinterpret_cast<uint4*>(o) = make_uint4(pack(v[0].x, v[1].x), pack(v[2].x, v[3].x),
+                                            pack(v[4].x, v[5].x), pack(v[6].x, v[7].x));
+  *reinterpret_cast<uint4*>(o + ldt) = make_uint4(pack(v[0].y, v[1].y), pack(v[2].y, v[3].y),
+                                                  pack(v[4].y, v[5].y), pack(v[6].y, v[7].y));
+  *reinterpret_cast<uint4*>(o + 2 * static_cast<int64_t>(ldt)) =
+      make_uint4(pack(v[0].z, v[1].z), pack(v[2].z, v[3].z), pack(v[4].z, v[5].z),
+                 pack(v[6].z, v[7].z));
+  *reinterpret_cast<uint4*>(o + 3 * static_cast<int64_t>(ldt)) =
+      make_uint4(pack(v[0].w, v[1].w), pack(v[2].w, v[3].w), pack(v[4].w, v[5].w),
+                 pack(v[6].w, v[7].w));
 }
 
 // One block per canary (256 bytes = 64 words): write the pattern, or compare.
@@ -208,6 +243,12 @@ cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T,
                                cudaStream_t s) {
   if (E <= 0 || T <= 0 || C <= 0) return cudaSuccess;
   if (T % 8 != 0 || C % 8 != 0 || ldt % 4 != 0) return cudaErrorInvalidValue;
+  if (!Xb) {  // X^T alone
+    if (ldt % 8 != 0) return cudaErrorInvalidValue;  // 16-byte stores
+    dim3 grid_t((C + 63) / 64, (T + 127) / 128, E);
+    k_tokens_t_bf16<<<grid_t, 256, 0, s>>>(X, static_cast<__nv_bfloat16*>(Xt), T, C, ldt);
+    return cudaGetLastError();
+  }
   dim3 grid((C + 63) / 64, (T + 63) / 64, E);
   k_tokens_bf16<<<grid, 256, 0, s>>>(X, static_cast<__nv_bfloat16*>(Xb),
                                      static_cast<__nv_bfloat16*>(Xt), T, C, ldt);

@@ -235,7 +235,8 @@ cudaError_t launch_symmetrize(const float* H, void* out, int E, int C, int out_b
 // H[e][i][j] = H[e][j][i] for i > j, bf16 [E][C][C] in place (the lower triangle of a
 // symmetric output whose upper triangle a TcGemm with sym = 1 computed).
 cudaError_t launch_mirror_upper_bf16(void* H, int E, int C, cudaStream_t s);
-// Xb[e] = bf16(X[e]) ([T][C]) and Xt[e] = bf16(X[e])^T ([C][ldt], first T columns).
+// Xb[e] = bf16(X[e]) ([T][C]) and Xt[e] = bf16(X[e])^T ([C][ldt], first T columns);
+// Xb null: Xt alone (ldt a multiple of 8).
 cudaError_t launch_tokens_bf16(const float* X, void* Xb, void* Xt, int E, int T, int C, int ldt,
                                cudaStream_t s);
 

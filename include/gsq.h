@@ -267,8 +267,9 @@ GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float ka
  *             draws anew), W^_j, D_j = W^_j - W;
  *   loss      G = 2 D_j X^T X (X = X_dev, this micro-batch's tokens), as
  *             Y = D_j X^T, G = 2 Y X, or on the tensor cores, where it costs fewer
- *             flops (C (T + R) < 2 R T at the descriptor's n_tokens = T), through
- *             the micro-batch's Gram matrix H = X^T X (bf16), G = 2 D_j H;
+ *             flops (C (T + 2R) < 4 R T at the descriptor's n_tokens = T), through
+ *             the micro-batch's Gram matrix H = X^T X (bf16, formed from the tiles
+ *             of its upper triangle and mirrored), G = 2 D_j H;
  *             GSQ_TOKEN_ROUTE=direct|gram in the environment at gsq_init_layer
  *             (and gsq_workspace_size) forces one;
  *             L_j = 1/2 sum D_j*G = sum over the tokens of ||D_j x||^2;

@@ -86,11 +86,15 @@ class Workload:
         write logits, logit momentum (4L each), D for the next step (2)."""
         return 16 * self.L + 4 + self.w_bytes() + 2 + (1 if self.param == "shift5" else 0)
 
-    def gram_route(self) -> bool:
+    def gram_route(self, sym=True) -> bool:
         """Per-step tokens on the tensor cores contract through each micro-batch's Gram
         matrix (H = X^T X, then G = 2 D H) when that costs fewer flops than Y = D X^T,
-        G = 2 Y X: C (T + R) < 2 R T."""
-        return self.calib == "batches" and self.cols * (self.tokens + self.rows) < 2 * self.rows * self.tokens
+        G = 2 Y X: C (T + 2R) < 4 R T with H formed from its upper triangle (sym), else
+        C (T + R) < 2 R T."""
+        if self.calib != "batches":
+            return False
+        C_, T, R = self.cols, self.tokens, self.rows
+        return C_ * (T + 2 * R) < 4 * R * T if sym else C_ * (T + R) < 2 * R * T
 
     def gemm_flops_per_step(self, gram=None, sym=True) -> int:
         """Loss contraction flops of one step: G = 2 D H (2 R C^2 per expert), or per
@@ -99,7 +103,7 @@ class Workload:
         (2 C^2 T + 2 R C^2 per expert; C (C + 1) T for H's upper triangle when sym)."""
         E, R, Cc, T = self.experts, self.rows, self.cols, self.tokens
         if self.calib == "batches":
-            if self.gram_route() if gram is None else gram:
+            if self.gram_route(sym) if gram is None else gram:
                 h = Cc * (Cc + 1) * T if sym else 2 * Cc * Cc * T
                 return E * (h + 2 * R * Cc * Cc) * self.micro
             return 4 * E * R * Cc * T * self.micro

@@ -127,13 +127,16 @@ Shape shape_of(const gsq_layer_desc& d) {
   s.mask_sign = d.param_mode == GSQ_PARAM_MASK_SIGN;
   s.L = s.shift ? 5 : (s.mask_sign ? 2 : s.K);
   // Per-step tokens on the tensor cores: G = 2 D X^T X either as Y = D X^T, G = 2 Y X
-  // (4 R T C flops per expert) or through the micro-batch's Gram matrix, H = X^T X,
-  // G = 2 D H (2 C^2 T + 2 R C^2 flops), whichever costs fewer flops at the
-  // descriptor's token count (4096 x 4096 with 32,768 tokens: 1.24 against 2.2 TFLOP).
-  // GSQ_TOKEN_ROUTE=direct|gram forces one.
+  // (4 R T C flops per expert) or through the micro-batch's Gram matrix, H = X^T X
+  // from the tiles of its upper triangle (C^2 T; every tile with GSQ_TOKEN_SYM=0:
+  // 2 C^2 T), then G = 2 D H (2 R C^2), whichever costs fewer flops at the
+  // descriptor's token count (4096 x 4096 with 32,768 tokens: 0.69 against 2.2
+  // TFLOP).  GSQ_TOKEN_ROUTE=direct|gram forces one.
   s.gram = false;
   if (s.batches && s.d_bf16) {
-    s.gram = s.C * (s.T + s.R) < 2 * s.R * s.T;
+    const char* sv = std::getenv("GSQ_TOKEN_SYM");
+    const bool sym = !(sv && std::atoi(sv) == 0);
+    s.gram = sym ? s.C * (s.T + 2 * s.R) < 4 * s.R * s.T : s.C * (s.T + s.R) < 2 * s.R * s.T;
     if (const char* v = std::getenv("GSQ_TOKEN_ROUTE")) {
       if (std::strcmp(v, "direct") == 0) s.gram = false;
       if (std::strcmp(v, "gram") == 0) s.gram = true;

@@ -87,9 +87,10 @@ def test_workspace_size_formula(lib):
                           lr_scales=w.lr_scales,
                           param_mode=lib.PARAM_MODES[w.param])
         n, L = w.n, w.L
-        # per-step tokens contract through each micro-batch's Gram matrix X^T X where that
-        # costs fewer flops than Y = D X^T, G = 2 Y X: C (T + R) < 2 R T
-        gram = w.calib == "batches" and w.cols * (w.tokens + w.rows) < 2 * w.rows * w.tokens
+        # per-step tokens contract through each micro-batch's Gram matrix X^T X (formed from
+        # its upper triangle) where that costs fewer flops than Y = D X^T, G = 2 Y X:
+        # C (T + 2R) < 4 R T
+        gram = w.calib == "batches" and w.cols * (w.tokens + 2 * w.rows) < 4 * w.rows * w.tokens
         # every buffer is 256-byte aligned and followed by a 256-byte canary
         bufs = [256, 8 * 16384, 4 * L * n, 4 * L * n, 4 * n // w.group, 4 * n // w.group,
                 n * w.w_bytes()]

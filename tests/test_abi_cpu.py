@@ -121,6 +121,33 @@ def test_workspace_size_formula(lib):
     assert lib.gsq_workspace_size(d) < 100e9
 
 
+@pytest.mark.parametrize("sym", ["1", "0"])
+def test_token_route_follows_the_flop_rule(lib, sym, monkeypatch):
+    """A per-step-token layer on the tensor cores contracts through each micro-batch's
+    Gram matrix exactly where that costs fewer flops than Y = D X^T, G = 2 Y X:
+    C (T + 2R) < 4 R T with X^T X formed from its upper triangle, C (T + R) < 2 R T with
+    every tile.  The route shows in the workspace (X^T and H against X, X^T and Y)."""
+    monkeypatch.setenv("GSQ_TOKEN_SYM", sym)
+    rule = ((lambda R, C, T: C * (T + 2 * R) < 4 * R * T) if sym == "1"
+            else (lambda R, C, T: C * (T + R) < 2 * R * T))
+    shapes = [(4096, 4096, 32768), (2048, 4096, 32768), (1024, 4096, 32768), (512, 4096, 32768),
+              (4096, 4096, 2048), (4096, 1024, 8192), (136, 384, 328), (600, 384, 328)]
+    picked = set()
+    for R, C, T in shapes:
+        d = lib.make_desc(experts=1, rows=R, cols=C, grid=(-1.5, -0.5, 0.5, 1.5), group_size=128,
+                          calib_kind=lib.GSQ_CALIB_BATCHES, n_tokens=T)
+        sizes = {}
+        for route in ("gram", "direct"):
+            monkeypatch.setenv("GSQ_TOKEN_ROUTE", route)
+            sizes[route] = lib.gsq_workspace_size(d)
+        monkeypatch.delenv("GSQ_TOKEN_ROUTE")
+        assert sizes["gram"] != sizes["direct"], (R, C, T)
+        want = "gram" if rule(R, C, T) else "direct"
+        picked.add(want)
+        assert lib.gsq_workspace_size(d) == sizes[want], (R, C, T, want)
+    assert picked == {"gram", "direct"}
+
+
 @pytest.mark.parametrize("kw,status", [
     (dict(cols=260), 2),                         # C % 8
     (dict(cols=192, group_size=128), 2),         # C % G

@@ -878,6 +878,22 @@ def gpu_arm_tokens(args, rank, world, local):
     return 0
 
 
+def make_read_back(torch):
+    """Per-step read-back of a step's loss into pinned host memory on a copy stream of
+    its own: the copy waits for the step (an event on the compute stream) but does not
+    hold the next step's kernels behind it."""
+    copy_stream = torch.cuda.Stream()
+
+    def read_back(dst_host, src_dev):
+        done = torch.cuda.Event()
+        done.record()
+        copy_stream.wait_event(done)
+        with torch.cuda.stream(copy_stream):
+            dst_host.copy_(src_dev, non_blocking=True)
+            src_dev.record_stream(copy_stream)
+    return read_back
+
+
 def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, device, one_step):
     """The whole job through the public API from pinned host buffers: W and the
     micro-batch tokens uploaded, init, K steps (every micro-batch's loss read
@@ -886,6 +902,7 @@ def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, device, one_step):
     X_host = [X.cpu().pin_memory() for X in Xs]
     K = args.steps
     loss_host = torch.zeros(K, w.micro, dtype=torch.float32).pin_memory()
+    read_back = make_read_back(torch)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     Wd = W_host.to("cuda", non_blocking=True)
@@ -895,7 +912,7 @@ def e2e_run_tokens(args, w, W, Xs, hyper, gsq, torch, device, one_step):
     loss = torch.zeros(K, w.micro, device="cuda")
     for t in range(K):
         one_step(layer, t, Xd, loss[t])
-        loss_host[t].copy_(loss[t], non_blocking=True)
+        read_back(loss_host[t], loss[t])
     packed = torch.empty(layer.packed_size(), dtype=torch.uint8, device="cuda")
     layer.pack(packed)
     packed_host = torch.empty(packed.numel(), dtype=torch.uint8).pin_memory()
@@ -933,6 +950,7 @@ def e2e_run(args, w, W, H, gsq, torch, device, hyper):
     H_host = H.cpu().pin_memory()
     K = args.steps
     loss_host = torch.zeros(K, dtype=torch.float32).pin_memory()
+    read_back = make_read_back(torch)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     Wd = W_host.to("cuda", non_blocking=True)
@@ -942,7 +960,7 @@ def e2e_run(args, w, W, H, gsq, torch, device, hyper):
     for t in range(K):
         layer.step(t, w.tau(t % w.steps), w.kappa, next_tau=w.tau((t + 1) % w.steps),
                    next_kappa=w.kappa, loss=loss[t:t + 1])
-        loss_host[t:t + 1].copy_(loss[t:t + 1], non_blocking=True)
+        read_back(loss_host[t:t + 1], loss[t:t + 1])
     packed = torch.empty(layer.packed_size(), dtype=torch.uint8, device="cuda")
     layer.pack(packed)
     packed_host = torch.empty(packed.numel(), dtype=torch.uint8).pin_memory()

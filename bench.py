@@ -883,14 +883,14 @@ def make_read_back(torch):
     its own: the copy waits for the step (an event on the compute stream) but does not
     hold the next step's kernels behind it."""
     copy_stream = torch.cuda.Stream()
+    done = torch.cuda.Event()   # one event, recorded again every step: a wait takes the
+                                # record current when it is enqueued
 
-    def read_back(dst_host, src_dev):
-        done = torch.cuda.Event()
+    def read_back(dst_host, src_dev):   # src_dev stays alive until the job's final sync
         done.record()
         copy_stream.wait_event(done)
         with torch.cuda.stream(copy_stream):
             dst_host.copy_(src_dev, non_blocking=True)
-            src_dev.record_stream(copy_stream)
     return read_back
 
 

@@ -162,3 +162,39 @@ def test_full_size_token_microbatch_sampled_rows():
     assert np.array_equal(st1.logits, st0.logits) and np.array_equal(st1.scales, st0.scales)
     case.layer.sync_status()
     case.layer.close()
+
+
+def test_full_layer_loss_against_oracle():
+    """The headline layer whole (4096 x 4096, K = 4, the benchmark's launch configuration):
+    the loss of one step against the oracle's float64 loss over every row, within the
+    2e-2 relative tolerance for a loss taken through the bf16 GEMM (it lands far
+    inside), and D and G over all 16.8 M weights.  The oracle starts from the GPU's own
+    initial state (initialisation has its own bit-exact tests)."""
+    g = gsq()
+    w = C.WORKLOADS["llama8b_q_proj"]
+    case = Case(w, gemm="bf16")                 # keeps H (float64) for the oracle
+    nr, K, Cc = w.rows, w.L, w.cols
+    tau0 = w.tau(0)
+    f = lambda which: case.layer.get_tensor(which, torch.float32)
+    st = O.RowState(row_ids=np.arange(nr, dtype=np.int64), W=case.W_host.astype(np.float64),
+                    logits=f(g.GSQ_T_LOGITS).view(K, nr, Cc).cpu().numpy(),
+                    scales=f(g.GSQ_T_SCALES).view(nr, Cc // w.group).cpu().numpy(),
+                    m_logits=f(g.GSQ_T_MOM_LOGITS).view(K, nr, Cc).cpu().numpy(),
+                    m_scales=f(g.GSQ_T_MOM_SCALES).view(nr, Cc // w.group).cpu().numpy())
+    loss = torch.zeros(1, device="cuda")
+    case.layer.step(0, tau0, w.kappa, loss=loss)          # no look-ahead: D stays
+    torch.cuda.synchronize()
+    case.layer.sync_status()
+    D = case.layer.get_tensor(g.GSQ_T_D, torch.bfloat16).view(nr, Cc).double().cpu().numpy()
+    G = f(g.GSQ_T_G).view(nr, Cc).double().cpu().numpy()
+    case.layer.close()
+
+    fw = O.forward(case.prob, st, 0, tau0, w.kappa)
+    L, Gr = O.loss_and_grad(case.prob, st.row_ids, fw.D)
+    rel = abs(loss.item() - L) / L
+    print(f"full-layer loss: GPU {loss.item():.6e}, oracle {L:.6e}, relative {rel:.2e}")
+    assert rel <= TOL_BF16, rel
+    assert_close(D, fw.D, TOL_BF16, "D, every weight")
+    gerr = float(np.linalg.norm(G - Gr) / np.linalg.norm(Gr))
+    print(f"G over every weight: relative norm error {gerr:.2e}")
+    assert gerr <= TOL_BF16, gerr

@@ -271,7 +271,8 @@ GSQ_API gsq_status gsq_step(gsq_layer* layer, uint64_t step, float tau, float ka
  *             the micro-batch's Gram matrix H = X^T X (bf16, formed from the tiles
  *             of its upper triangle and mirrored), G = 2 D_j H;
  *             GSQ_TOKEN_ROUTE=direct|gram in the environment at gsq_init_layer
- *             (and gsq_workspace_size) forces one;
+ *             (and gsq_workspace_size) forces one, GSQ_TOKEN_SYM=0 forms every tile
+ *             of H (the rule then reads C (T + R) < 2 R T);
  *             L_j = 1/2 sum D_j*G = sum over the tokens of ||D_j x||^2;
  *   backward  the gradients of L_j, added into an accumulator;
  *   update    after the last micro-batch only: Lion with the mean gradient

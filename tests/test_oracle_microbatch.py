@@ -101,3 +101,23 @@ def test_resampled_noise_cuts_gradient_variance():
                                          update=False).d_logits[1, 0, 3])
     ratio = np.var(eight) / np.var(one)
     assert 0.6 / 8 < ratio < 1.6 / 8, ratio
+
+
+def test_token_loss_through_the_gram_matrix():
+    """The micro-batch's loss and gradient through its Gram matrix, H = X^T X, equal the
+    token-literal ones (Eq. 1 with a linear f: sum_t ||D x_t||^2 = tr(D X^T X D^T) and
+    2 (D X^T) X = 2 D (X^T X)): the identity the GPU's Gram route rests on, on a
+    micro-batch with more tokens than inputs and with fewer."""
+    for T, C in ((40, 16), (6, 32)):
+        prob, st, batches = _setup(C=C, T=T, M=1, seed=T)
+        X = batches[0]
+        px = O.Problem(E=1, R=prob.R, C=C, grid=GRID, group=16, seed=5, X=X)
+        ph = O.Problem(E=1, R=prob.R, C=C, grid=GRID, group=16, seed=5,
+                       H=np.einsum("etc,etd->ecd", X, X))
+        fw = O.forward(px, st, 2, 0.6, 1.0)
+        ids = np.arange(prob.R)
+        Lx, Gx = O.loss_and_grad(px, ids, fw.D)
+        Lh, Gh = O.loss_and_grad(ph, ids, fw.D)
+        assert abs(Lx - Lh) <= 1e-12 * Lx
+        np.testing.assert_allclose(Gh, Gx, rtol=1e-11, atol=1e-14 * np.abs(Gx).max())
+        assert abs(O.loss_bruteforce(st.W, fw.What, X[0]) - Lh) <= 1e-12 * Lh
